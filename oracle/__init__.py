@@ -1,0 +1,212 @@
+"""CPU oracle for the MC compressed MoE layer -- TEST INFRASTRUCTURE ONLY.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` /
+``--impl reference`` legs of ``bench.py`` may import this package.  The product
+library never imports it, and it imports nothing from the product library.
+
+The arithmetic lives in ``mc_oracle.c`` (plain C, fp64, one weight at a time);
+this module compiles it with gcc on first use and marshals numpy arrays.  Every
+function states the passage of the paper it follows:
+
+* ``gate_logits`` / ``route``   -- Sec. 2.1 Eq. 1 (top-2 gate), Sec. 2.3.1 Eq. 5
+  (ODP), Sec. 2.3.2 (token protection).
+* ``permute``                   -- the token/expert correspondence of Eq. 1.
+* ``gemv`` / ``dequant_f32``    -- Sec. 2.1 (Eq. 2 integer grid), App. A.2 (1-bit).
+* ``expert``                    -- the Mixtral SwiGLU expert E_i of Eq. 1.
+* ``moe_layer``                 -- Eq. 1 with Eq. 5.
+* ``rmsnorm``                   -- the normalisation between stacked layers.
+
+Parity status: every function is pinned by ``tests/test_oracle_pins.py`` (closed
+forms, library routines, brute force and invariants); none is "parity unpinned".
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "mc_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_SO = os.path.join(_BUILD, "libmc_oracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile the C oracle with gcc (-O2, no fast-math, no vectorised reassociation)."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if force or not os.path.exists(_SO) or os.path.getmtime(_SO) < os.path.getmtime(_SRC):
+        tmp = _SO + ".tmp%d" % os.getpid()
+        subprocess.check_call(["gcc", "-O2", "-fPIC", "-shared", "-fno-fast-math",
+                               "-ffp-contract=off", "-o", tmp, _SRC, "-lm"])
+        os.replace(tmp, _SO)
+    return _SO
+
+
+class _Mat(ctypes.Structure):
+    _fields_ = [("rows", ctypes.c_int), ("cols", ctypes.c_int), ("group", ctypes.c_int),
+                ("bits", ctypes.c_int),
+                ("codes", ctypes.c_void_p), ("scale", ctypes.c_void_p),
+                ("zero", ctypes.c_void_p), ("dense", ctypes.c_void_p)]
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            P = ctypes.c_void_p
+            I = ctypes.c_int
+            D = ctypes.c_double
+            lib.mco_weight.restype = D
+            lib.mco_weight.argtypes = [ctypes.POINTER(_Mat), I, I]
+            lib.mco_dequant_f32.argtypes = [ctypes.POINTER(_Mat), P]
+            lib.mco_gemv.argtypes = [ctypes.POINTER(_Mat), P, P]
+            lib.mco_expert.argtypes = [ctypes.POINTER(_Mat)] * 3 + [P, P]
+            lib.mco_gate_logits.argtypes = [P, P, I, I, I, P]
+            lib.mco_route.argtypes = [P, P, I, I, I, D, P, P, P, P]
+            lib.mco_permute.restype = I
+            lib.mco_permute.argtypes = [P, P, I, I, P, P]
+            lib.mco_moe_layer.argtypes = [P, P, I, I, I, P, D, P, P, I, P, P, P, P]
+            lib.mco_rmsnorm.argtypes = [P, P, I, D, P]
+            _lib = lib
+    return _lib
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data
+
+
+def _f32(a):
+    return np.ascontiguousarray(a, dtype=np.float32)
+
+
+class QMat:
+    """One expert matrix [rows, cols]; groups of ``group`` along cols.
+
+    ``codes`` uint8 [rows, cols] (0 .. 2**bits-1), ``scale``/``zero`` fp16 or fp32
+    [rows, cols/group]; or ``bits=16`` with ``dense`` [rows, cols].
+    """
+
+    def __init__(self, rows, cols, group, bits, codes=None, scale=None, zero=None, dense=None):
+        self.rows, self.cols, self.group, self.bits = int(rows), int(cols), int(group), int(bits)
+        if bits == 16:
+            self.dense = _f32(dense).reshape(rows, cols)
+            self.codes = self.scale = self.zero = None
+        else:
+            self.codes = np.ascontiguousarray(codes, dtype=np.uint8).reshape(rows, cols)
+            self.scale = _f32(np.asarray(scale).astype(np.float32)).reshape(rows, cols // group)
+            self.zero = _f32(np.asarray(zero).astype(np.float32)).reshape(rows, cols // group)
+            self.dense = None
+
+    def c(self):
+        return _Mat(self.rows, self.cols, self.group, self.bits,
+                    _ptr(self.codes), _ptr(self.scale), _ptr(self.zero), _ptr(self.dense))
+
+
+def weight(m: QMat, r: int, k: int) -> float:
+    """Sec. 2.1 / App. A.2: the real value (q - z) * s of one weight (fp64)."""
+    cm = m.c()
+    return _load().mco_weight(ctypes.byref(cm), int(r), int(k))
+
+
+def dequant_f32(m: QMat) -> np.ndarray:
+    """Sec. 2.1: the whole matrix dequantised in fp32, ((float)q - (float)z) * (float)s."""
+    out = np.empty((m.rows, m.cols), np.float32)
+    cm = m.c()
+    _load().mco_dequant_f32(ctypes.byref(cm), _ptr(out))
+    return out
+
+
+def gemv(m: QMat, x) -> np.ndarray:
+    """y = W x with W dequantised one weight at a time, fp64."""
+    x = np.ascontiguousarray(x, dtype=np.float64)
+    y = np.empty(m.rows, np.float64)
+    cm = m.c()
+    _load().mco_gemv(ctypes.byref(cm), _ptr(x), _ptr(y))
+    return y
+
+
+def expert(w1: QMat, w3: QMat, w2: QMat, x) -> np.ndarray:
+    """Mixtral SwiGLU expert of Eq. 1: W2 (silu(W1 x) * W3 x), fp64."""
+    x = np.ascontiguousarray(x, dtype=np.float64)
+    out = np.empty(w2.rows, np.float64)
+    a, b, c = w1.c(), w3.c(), w2.c()
+    _load().mco_expert(ctypes.byref(a), ctypes.byref(b), ctypes.byref(c), _ptr(x), _ptr(out))
+    return out
+
+
+def gate_logits(x, wg) -> np.ndarray:
+    """Eq. 1 gate: l = x Wg^T in fp64.  x [T,H], wg [E,H] (bf16 values as fp32)."""
+    x, wg = _f32(x), _f32(wg)
+    T, H = x.shape
+    E = wg.shape[0]
+    out = np.empty((T, E), np.float64)
+    _load().mco_gate_logits(_ptr(x), _ptr(wg), T, H, E, _ptr(out))
+    return out
+
+
+def route(x, wg, mu: float, protect=None):
+    """Eq. 1 top-2 + renormalised softmax weights, Eq. 5 ODP, Sec. 2.3.2 protection.
+
+    Returns (idx int32 [T,2], w float32 [T,2], pruned uint8 [T]).
+    """
+    x, wg = _f32(x), _f32(wg)
+    T, H = x.shape
+    E = wg.shape[0]
+    idx = np.empty((T, 2), np.int32)
+    w = np.empty((T, 2), np.float32)
+    pr = np.empty(T, np.uint8)
+    prot = None if protect is None else np.ascontiguousarray(protect, dtype=np.uint8)
+    _load().mco_route(_ptr(x), _ptr(wg), T, H, E, float(mu), _ptr(prot),
+                      _ptr(idx), _ptr(w), _ptr(pr))
+    return idx, w, pr
+
+
+def permute(idx, pruned, E: int):
+    """Kept (token, slot) pairs grouped by expert, ascending token: (offsets[E+1], perm[P])."""
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    pruned = np.ascontiguousarray(pruned, dtype=np.uint8)
+    T = idx.shape[0]
+    offsets = np.empty(E + 1, np.int32)
+    perm = np.empty(2 * T, np.int32)
+    n = _load().mco_permute(_ptr(idx), _ptr(pruned), T, E, _ptr(offsets), _ptr(perm))
+    return offsets, perm[:n].copy()
+
+
+def moe_layer(x, wg, mats, mu: float, protect=None, tokens=None):
+    """Eq. 1 with Eq. 5 for the tokens listed (default all).
+
+    ``mats`` is a list of E triples (w1, w3, w2) of QMat.  Returns
+    (y fp64 [n_tok, H], idx, w, pruned).
+    """
+    x, wg = _f32(x), _f32(wg)
+    T, H = x.shape
+    E = wg.shape[0]
+    flat = (_Mat * (3 * E))()
+    for e in range(E):
+        for m in range(3):
+            flat[3 * e + m] = mats[e][m].c()
+    toks = np.arange(T, dtype=np.int32) if tokens is None else np.ascontiguousarray(tokens, dtype=np.int32)
+    y = np.empty((len(toks), H), np.float64)
+    idx = np.empty((T, 2), np.int32)
+    w = np.empty((T, 2), np.float32)
+    pr = np.empty(T, np.uint8)
+    prot = None if protect is None else np.ascontiguousarray(protect, dtype=np.uint8)
+    _load().mco_moe_layer(_ptr(x), _ptr(wg), T, H, E, ctypes.cast(flat, ctypes.c_void_p),
+                          float(mu), _ptr(prot), _ptr(toks), len(toks),
+                          _ptr(idx), _ptr(w), _ptr(pr), _ptr(y))
+    return y, idx, w, pr
+
+
+def rmsnorm(x, gamma, eps: float = 1e-5) -> np.ndarray:
+    """x / sqrt(mean(x^2) + eps) * gamma for one vector, fp64."""
+    x = np.ascontiguousarray(x, dtype=np.float64)
+    g = _f32(gamma)
+    out = np.empty_like(x)
+    _load().mco_rmsnorm(_ptr(x), _ptr(g), x.shape[0], float(eps), _ptr(out))
+    return out

@@ -1,0 +1,229 @@
+"""Seeded synthetic inputs for the MC MoE layer.
+
+This module is shared by the tests, the benchmark and the smoke check: it is the
+only code both the CUDA path and the CPU oracle see.  It draws random numbers and
+converts number formats; it contains none of the layer's arithmetic (no gate, no
+dequantisation, no expert, no pruning rule).
+
+Workload shapes follow the Mixtral-8x7b MoE block (H = 4096, E = 8, top-2; the
+paper's model table) with the SwiGLU width F = 14336 and the synthetic recipes
+below:
+
+* activations x ~ N(0, 1), rounded to bf16;
+* gate weight Wg ~ N(0, 0.02), rounded to bf16 (optionally tilted along a shared
+  direction so that expert loads are skewed);
+* expert codes drawn uniformly in [0, 2**b - 1] per weight (b = the expert's bit
+  width), one fp16 scale per group with the magnitude a min-max quantiser gives
+  an N(0, 0.02) group, an fp16 zero that is an integer in the code range for
+  b >= 2 and 1/2 for b = 1 (the binary format of the paper's appendix);
+  ``zero_mode="fractional"`` draws arbitrary fp16 zeros instead;
+* protect masks choose a seeded subset of tokens.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+
+import numpy as np
+
+MIXTRAL_H = 4096
+MIXTRAL_F = 14336
+MIXTRAL_E = 8
+
+
+# ----------------------------------------------------------------- formats --
+
+def f32_to_bf16_bits(a: np.ndarray) -> np.ndarray:
+    """Round-to-nearest-even float32 -> bf16, returned as uint16 bit patterns."""
+    a = np.ascontiguousarray(a, dtype=np.float32)
+    u = a.view(np.uint32).astype(np.uint64)
+    rounded = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    return rounded.astype(np.uint16)
+
+
+def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
+    """Exact bf16 (uint16 bits) -> float32."""
+    b = np.ascontiguousarray(b, dtype=np.uint16)
+    return (b.astype(np.uint32) << 16).view(np.float32)
+
+
+def fp16_bits(a: np.ndarray) -> np.ndarray:
+    """float16 array -> its uint16 bit patterns."""
+    return np.ascontiguousarray(a, dtype=np.float16).view(np.uint16)
+
+
+# ------------------------------------------------------------------ layout --
+
+@dataclass
+class Layer:
+    """All inputs of one MoE layer, host side.
+
+    x      uint16 [T, H]  bf16 bits        gate  uint16 [E, H] bf16 bits
+    bits   int8 [E]                         group int
+    codes  list over E of 3 uint8 arrays: w1 [F, H], w3 [F, H], w2 [H, F]
+    scale, zero  list over E of 3 float16 arrays [rows, cols/group]
+    protect uint8 [T] or None; mu float (Eq. 5 threshold; 0 = no pruning)
+    """
+    T: int
+    H: int
+    F: int
+    E: int
+    group: int
+    bits: np.ndarray
+    x: np.ndarray
+    gate: np.ndarray
+    codes: list
+    scale: list
+    zero: list
+    protect: np.ndarray | None = None
+    mu: float = 0.0
+    meta: dict = field(default_factory=dict)
+
+    def x_f32(self):
+        return bf16_bits_to_f32(self.x)
+
+    def gate_f32(self):
+        return bf16_bits_to_f32(self.gate)
+
+    def mat_shape(self, m: int):
+        return (self.F, self.H) if m < 2 else (self.H, self.F)
+
+    def mean_bits(self) -> float:
+        return float(np.mean(self.bits))
+
+
+def _rng(seed, *stream):
+    return np.random.default_rng([int(seed)] + [int(s) for s in stream])
+
+
+def gaussian_bf16(seed, stream, shape, std=1.0):
+    r = _rng(seed, *stream)
+    return f32_to_bf16_bits((r.standard_normal(shape, dtype=np.float32) * np.float32(std)))
+
+
+def expert_matrix(seed, e, m, rows, cols, group, bits, zero_mode="integer"):
+    """Codes, fp16 scale, fp16 zero for matrix m (0=w1, 1=w3, 2=w2) of expert e."""
+    r = _rng(seed, 1000 + e, m)
+    n = rows * cols
+    raw = np.frombuffer(r.bytes(n), dtype=np.uint8)
+    codes = (raw & np.uint8((1 << bits) - 1)).reshape(rows, cols)
+    ng = cols // group
+    levels = (1 << bits) - 1
+    # scale magnitude of a min-max quantiser on an N(0, 0.02) group of this size:
+    # the expected range of g normals is ~ 2 * 2.6 sigma at g = 64..128.
+    jitter = r.uniform(0.8, 1.25, size=(rows, ng)).astype(np.float32)
+    if bits == 1:
+        # binary format: s = 2 * alpha with alpha ~ mean |w| = 0.8 * 0.02; z = 1/2
+        scale = (np.float32(2 * 0.8 * 0.02) * jitter).astype(np.float16)
+        zero = np.full((rows, ng), 0.5, np.float16)
+    else:
+        scale = (np.float32(5.2 * 0.02 / levels) * jitter).astype(np.float16)
+        if zero_mode == "integer":
+            lo, hi = levels // 2, (levels + 1) // 2
+            zero = r.integers(lo, hi + 1, size=(rows, ng)).astype(np.float16)
+        elif zero_mode == "fractional":
+            zero = r.uniform(0.0, float(levels), size=(rows, ng)).astype(np.float16)
+        else:
+            raise ValueError(zero_mode)
+    return codes, scale, zero
+
+
+def bit_table(seed, E, total, lo=1, hi=3):
+    """A seeded per-expert bit table with the given sum, values in [lo, hi], with at
+    least one 3-bit and one 2-bit expert (the constraints of the paper's Eq. 4)."""
+    r = _rng(seed, 7)
+    for _ in range(100000):
+        b = r.integers(lo, hi + 1, size=E)
+        if b.sum() == total and (b == 3).any() and (b == 2).any():
+            return b.astype(np.int8)
+    raise ValueError("no table")
+
+
+def make_layer(T, H, F, E, group, bits, seed, *, gate_std=0.02, mu=0.0,
+               protect_frac=0.0, zero_mode="integer", skew=None, experts=True):
+    """One layer of synthetic inputs.
+
+    ``skew``: None, or (c, beta) -- x gets +c along a seeded unit direction u and
+    gate row e gets +beta*(e - (E-1)/2)/((E-1)/2) * u, which tilts expert loads.
+    ``experts=False`` skips the expert weights (routing-only tests).
+    """
+    bits = np.asarray(bits, dtype=np.int8)
+    assert bits.shape == (E,)
+    xr = _rng(seed, 1).standard_normal((T, H), dtype=np.float32)
+    gr = _rng(seed, 2).standard_normal((E, H), dtype=np.float32) * np.float32(gate_std)
+    if skew is not None:
+        c, beta = skew
+        u = _rng(seed, 3).standard_normal(H).astype(np.float32)
+        u /= np.linalg.norm(u)
+        xr = xr + np.float32(c) * u[None, :]
+        tilt = np.float32(beta) * (np.arange(E, dtype=np.float32) - (E - 1) / 2) / ((E - 1) / 2)
+        gr = gr + tilt[:, None] * u[None, :]
+    meta = {}
+    if skew is not None:
+        meta["skew_dir"] = u
+        meta["skew_c"] = float(skew[0])
+    x = f32_to_bf16_bits(xr)
+    gate = f32_to_bf16_bits(gr)
+    codes, scale, zero = [], [], []
+    if experts:
+        for e in range(E):
+            ce, se, ze = [], [], []
+            for m in range(3):
+                rows, cols = (F, H) if m < 2 else (H, F)
+                c_, s_, z_ = expert_matrix(seed, e, m, rows, cols, group, int(bits[e]), zero_mode)
+                ce.append(c_)
+                se.append(s_)
+                ze.append(z_)
+            codes.append(ce)
+            scale.append(se)
+            zero.append(ze)
+    protect = None
+    if protect_frac > 0:
+        r = _rng(seed, 4)
+        n = int(round(protect_frac * T))
+        protect = np.zeros(T, np.uint8)
+        protect[r.choice(T, size=n, replace=False)] = 1
+    return Layer(T, H, F, E, group, bits, x, gate, codes, scale, zero, protect, float(mu), meta)
+
+
+def resample_x_rows(layer: Layer, rows, seed, attempt):
+    """Redraw the listed activation rows (same recipe, new stream)."""
+    rows = np.asarray(rows, dtype=np.int64)
+    if rows.size == 0:
+        return
+    r = _rng(seed, 5, attempt)
+    new = r.standard_normal((rows.size, layer.H), dtype=np.float32)
+    skew = layer.meta.get("skew_dir")
+    if skew is not None:
+        new = new + np.float32(layer.meta["skew_c"]) * skew[None, :]
+    layer.x[rows] = f32_to_bf16_bits(new)
+
+
+def dense_expert_weights(seed, e, H, F, std=0.02):
+    """bf16 dense (unquantised, 16-bit) weights w1 [F,H], w3 [F,H], w2 [H,F]."""
+    out = []
+    for m in range(3):
+        rows, cols = (F, H) if m < 2 else (H, F)
+        out.append(gaussian_bf16(seed, (2000 + e, m), (rows, cols), std))
+    return out
+
+
+# ------------------------------------------------------------ named configs --
+
+def config_tiny(seed=1235):
+    """Tiny single layer: H 256, F 512, 8 experts, 64 tokens, group 64,
+    bits [3,2,2,1,3,2,2,3], mu 0.3, 25% of tokens protected."""
+    return make_layer(64, 256, 512, 8, 64, [3, 2, 2, 1, 3, 2, 2, 3], seed,
+                      mu=0.3, protect_frac=0.25)
+
+
+def config_decode(T=16, seed=1236, bits_total=20):
+    """Mixtral-8x7b-shaped decode layer: H 4096, F 14336, 8 experts, group 128,
+    bits from {1,2,3} with sum 20 (mean 2.5, nearest feasible to 2.54), ODP off."""
+    bits = bit_table(seed, 8, bits_total)
+    return make_layer(T, MIXTRAL_H, MIXTRAL_F, MIXTRAL_E, 128, bits, seed)
+
+
+def config_prefill(T=4096, seed=1237, bits_total=20, skew=(3.0, 0.9)):
+    """Mixtral-8x7b-shaped prefill layer with skewed expert loads, ODP off."""
+    bits = bit_table(seed, 8, bits_total)
+    return make_layer(T, MIXTRAL_H, MIXTRAL_F, MIXTRAL_E, 128, bits, seed, skew=skew)

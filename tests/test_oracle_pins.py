@@ -1,0 +1,322 @@
+"""Pins for the CPU oracle: each test checks the oracle against something other than
+itself -- a closed form from the paper, a library routine (numpy / torch), brute
+force on tiny inputs, or an invariant the method fixes.  No GPU needed.
+
+Together they are chosen so that a plausible slip in the oracle (a dropped term, a
+wrong sign or index, a transposed operand, a swapped slot, a wrong tie-break, a
+non-strict threshold) fails at least one of them; ``test_oracle_mutants.py``
+checks exactly that by compiling deliberately broken copies of the oracle.
+"""
+import itertools
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+
+
+def _rand_layer(T=12, H=32, F=48, E=4, group=16, bits=(1, 2, 3, 2), seed=7, **kw):
+    return synth.make_layer(T, H, F, E, group, list(bits), seed, **kw)
+
+
+def _mats(L):
+    return [[oracle.QMat(*L.mat_shape(m), L.group, int(L.bits[e]), L.codes[e][m],
+                         L.scale[e][m], L.zero[e][m]) for m in range(3)] for e in range(L.E)]
+
+
+# ------------------------------------------------------------------ gate ----
+
+def test_gate_logits_equal_library_matmul():
+    L = _rand_layer(T=9, H=40, E=5, bits=(1, 2, 3, 2, 1))
+    got = oracle.gate_logits(L.x_f32(), L.gate_f32())
+    want = L.x_f32().astype(np.float64) @ L.gate_f32().astype(np.float64).T
+    np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-12)
+    # orientation: logits[t, e] uses row e of the gate (a transposed gate fails)
+    assert got.shape == (9, 5)
+
+
+def test_top2_matches_full_sort():
+    """Eq. 1 top-2 against a stable sort of the fp32-rounded logits (library)."""
+    L = _rand_layer(T=200, H=24, E=8, bits=(1, 2, 3, 2, 1, 2, 3, 3), experts=False, gate_std=0.3)
+    idx, w, pr = oracle.route(L.x_f32(), L.gate_f32(), mu=0.0)
+    lg = oracle.gate_logits(L.x_f32(), L.gate_f32()).astype(np.float32)
+    order = np.argsort(-lg, axis=1, kind="stable")  # ties -> lower index first
+    np.testing.assert_array_equal(idx, order[:, :2].astype(np.int32))
+    assert not pr.any()
+
+
+def test_top2_tie_breaks_to_lower_index():
+    # identical gate rows give identical logits: lower index must win both slots
+    x = np.ones((1, 4), np.float32)
+    wg = np.array([[0, 0, 0, 0], [1, 1, 1, 1], [1, 1, 1, 1], [1, 1, 1, 1]], np.float32)
+    idx, w, _ = oracle.route(x, wg, mu=0.0)
+    assert idx.tolist() == [[1, 2]]
+    np.testing.assert_allclose(w, [[0.5, 0.5]], rtol=1e-7)
+
+
+def test_weights_are_renormalised_softmax():
+    """Weights = library softmax over all experts, restricted to top-2, renormalised."""
+    L = _rand_layer(T=64, H=24, E=8, bits=(1, 2, 3, 2, 1, 2, 3, 3), experts=False, gate_std=0.3)
+    idx, w, _ = oracle.route(L.x_f32(), L.gate_f32(), mu=0.0)
+    lg = torch.tensor(oracle.gate_logits(L.x_f32(), L.gate_f32()))
+    p = torch.softmax(lg, dim=1).numpy()
+    sel = np.take_along_axis(p, idx.astype(np.int64), axis=1)
+    np.testing.assert_allclose(w, sel / sel.sum(1, keepdims=True), rtol=2e-7, atol=1e-7)
+    np.testing.assert_allclose(w.sum(1), 1.0, rtol=1e-6)
+    assert (w[:, 0] >= w[:, 1]).all()  # slot 0 is the primary
+
+
+# ------------------------------------------------------------------- ODP ----
+
+def _ratios(L):
+    lg = torch.tensor(oracle.gate_logits(L.x_f32(), L.gate_f32()))
+    p = torch.softmax(lg, dim=1)
+    top = torch.topk(p, 2, dim=1).values.numpy()
+    return top[:, 1] / top[:, 0]
+
+
+def test_mu_zero_is_plain_top2():
+    """Eq. 5 uses a strict '<' and w1/w0 > 0, so mu = 0 prunes nothing."""
+    L = _rand_layer(T=80, E=8, bits=(1, 2, 3, 2, 1, 2, 3, 3), experts=False, gate_std=0.5)
+    i0, w0, p0 = oracle.route(L.x_f32(), L.gate_f32(), mu=0.0)
+    assert not p0.any()
+    i1, w1, p1 = oracle.route(L.x_f32(), L.gate_f32(), mu=-1.0)
+    np.testing.assert_array_equal(i0, i1)
+    np.testing.assert_array_equal(w0, w1)
+
+
+def test_mu_above_one_prunes_every_unprotected_token():
+    """w1/w0 <= 1 always, so mu > 1 prunes all but protected tokens (Sec. 2.3.2)."""
+    L = _rand_layer(T=80, E=8, bits=(1, 2, 3, 2, 1, 2, 3, 3), experts=False,
+                    gate_std=0.5, protect_frac=0.25)
+    idx, w, pr = oracle.route(L.x_f32(), L.gate_f32(), mu=1.0001, protect=L.protect)
+    np.testing.assert_array_equal(pr, 1 - L.protect)
+    # pruned: primary weight exactly 1, secondary exactly 0 (Eq. 5 as read)
+    np.testing.assert_array_equal(w[pr == 1], np.tile([1.0, 0.0], (int(pr.sum()), 1)).astype(np.float32))
+    # protected tokens keep the renormalised pair
+    np.testing.assert_allclose(w[pr == 0].sum(1), 1.0, rtol=1e-6)
+    assert (w[pr == 0][:, 1] > 0).all()
+
+
+def test_prune_set_is_ratio_below_mu():
+    """The pruned set is exactly {t unprotected : w1/w0 < mu}, checked on both sides
+    of several tokens' own ratios (a flipped ratio or a lost protection fails)."""
+    L = _rand_layer(T=60, E=8, bits=(1, 2, 3, 2, 1, 2, 3, 3), experts=False,
+                    gate_std=0.6, protect_frac=0.2)
+    ratio = _ratios(L)
+    for t in range(0, 60, 7):
+        for mu, flip in ((float(ratio[t]) * (1 - 1e-9), False), (float(ratio[t]) * (1 + 1e-9), True)):
+            _, _, pr = oracle.route(L.x_f32(), L.gate_f32(), mu=mu, protect=L.protect)
+            want = (ratio < mu) & (L.protect == 0)
+            np.testing.assert_array_equal(pr.astype(bool), want)
+            # just below its own ratio a token is kept; just above it is pruned
+            assert pr[t] == (flip and not L.protect[t])
+    # monotone in mu
+    counts = [oracle.route(L.x_f32(), L.gate_f32(), mu=m)[2].sum() for m in (0.1, 0.3, 0.5, 0.7, 0.9)]
+    assert counts == sorted(counts)
+
+
+# ----------------------------------------------------------- permutation ----
+
+def test_permutation_brute_force():
+    L = _rand_layer(T=50, E=8, bits=(1, 2, 3, 2, 1, 2, 3, 3), experts=False,
+                    gate_std=0.6, protect_frac=0.2)
+    idx, w, pr = oracle.route(L.x_f32(), L.gate_f32(), mu=0.5, protect=L.protect)
+    offsets, perm = oracle.permute(idx, pr, 8)
+    pairs = sorted((int(idx[t, s]), t, s) for t in range(50) for s in range(2)
+                   if not (s == 1 and pr[t]))
+    assert perm.tolist() == [2 * t + s for (_, t, s) in pairs]
+    for e in range(8):
+        assert offsets[e + 1] - offsets[e] == sum(1 for p in pairs if p[0] == e)
+    assert offsets[0] == 0 and offsets[-1] == 100 - pr.sum()
+
+
+# ---------------------------------------------------------------- dequant ---
+
+def test_dequant_closed_form_grid_points():
+    """Eq. 2 grid: a weight that lies on the grid of its group comes back exactly."""
+    r = np.random.default_rng(3)
+    for bits in (2, 3):
+        rows, cols, g = 6, 64, 16
+        s = r.uniform(0.01, 0.05, (rows, cols // g)).astype(np.float16)
+        z = r.integers(0, 2 ** bits, (rows, cols // g)).astype(np.float16)
+        q = r.integers(0, 2 ** bits, (rows, cols)).astype(np.uint8)
+        m = oracle.QMat(rows, cols, g, bits, q, s, z)
+        d = oracle.dequant_f32(m)
+        for rr, kk in [(0, 0), (5, 63), (3, 17), (2, 31), (4, 48)]:
+            gi = kk // g
+            want = (int(q[rr, kk]) - float(z[rr, gi])) * float(s[rr, gi])
+            assert d[rr, kk] == np.float32(want)
+            assert oracle.weight(m, rr, kk) == pytest.approx(want, rel=0, abs=0)
+    # the largest code is 2^b - 1 (R1): code 7 at 3 bits, zero 0, scale 1 -> 7
+    m = oracle.QMat(1, 8, 8, 3, np.full((1, 8), 7, np.uint8), np.ones((1, 1), np.float16),
+                    np.zeros((1, 1), np.float16))
+    assert oracle.dequant_f32(m)[0, 0] == 7.0
+
+
+def test_one_bit_sign_transform_round_trip():
+    """App. A.2: B~ = (sign(W)+1)/2 with sign(0)=+1, stored 1-bit; dequant with z=1/2,
+    s=2*alpha returns alpha*sign(W) exactly."""
+    r = np.random.default_rng(4)
+    rows, cols, g = 5, 32, 32
+    W = r.standard_normal((rows, cols)).astype(np.float32) * 0.02
+    W[0, 3] = 0.0  # sign(0) = +1
+    B = np.where(W >= 0, 1.0, -1.0)
+    Bt = ((B + 1) / 2).astype(np.uint8)
+    alpha = np.abs(W).mean(axis=1, keepdims=True).astype(np.float16)
+    m = oracle.QMat(rows, cols, g, 1, Bt, (2 * alpha.astype(np.float32)).astype(np.float16),
+                    np.full((rows, 1), 0.5, np.float16))
+    d = oracle.dequant_f32(m)
+    np.testing.assert_array_equal(d, (alpha.astype(np.float32) * B).astype(np.float32))
+    assert d[0, 3] > 0
+
+
+def test_one_bit_gemv_is_eq10_mac_free_form():
+    """Eq. 10: s*xB = s*(sum_{B~=1} x - sum_{B~=0} x), per group."""
+    r = np.random.default_rng(5)
+    rows, cols, g = 7, 96, 32
+    Bt = r.integers(0, 2, (rows, cols)).astype(np.uint8)
+    alpha = r.uniform(0.01, 0.03, (rows, cols // g)).astype(np.float16)
+    m = oracle.QMat(rows, cols, g, 1, Bt, (2 * alpha.astype(np.float32)).astype(np.float16),
+                    np.full((rows, cols // g), 0.5, np.float16))
+    x = r.standard_normal(cols)
+    y = oracle.gemv(m, x)
+    for rr in range(rows):
+        want = 0.0
+        for gi in range(cols // g):
+            sl = slice(gi * g, (gi + 1) * g)
+            xs, bs = x[sl], Bt[rr, sl]
+            want += float(alpha[rr, gi]) * (xs[bs == 1].sum() - xs[bs == 0].sum())
+        assert y[rr] == pytest.approx(want, rel=1e-12, abs=1e-12)
+
+
+def test_gemv_group_factored_identity():
+    """sum_k x_k (q_k - z) s = s (sum_k q_k x_k - z sum_k x_k) per group."""
+    r = np.random.default_rng(6)
+    for bits, g in [(2, 16), (3, 32), (1, 64)]:
+        rows, cols = 5, 128
+        q = r.integers(0, 2 ** bits, (rows, cols)).astype(np.uint8)
+        s = r.uniform(0.01, 0.05, (rows, cols // g)).astype(np.float16)
+        z = r.uniform(0, 2 ** bits - 1, (rows, cols // g)).astype(np.float16)
+        m = oracle.QMat(rows, cols, g, bits, q, s, z)
+        x = r.standard_normal(cols)
+        y = oracle.gemv(m, x)
+        qx = (q.astype(np.float64) * x).reshape(rows, cols // g, g).sum(-1)
+        X = x.reshape(cols // g, g).sum(-1)
+        want = (s.astype(np.float64) * (qx - z.astype(np.float64) * X[None, :])).sum(-1)
+        np.testing.assert_allclose(y, want, rtol=1e-11, atol=1e-12)
+
+
+def test_gemv_equals_library_matmul_of_dequantised():
+    L = _rand_layer()
+    m = _mats(L)[2][0]
+    x = np.random.default_rng(8).standard_normal(m.cols)
+    np.testing.assert_allclose(oracle.gemv(m, x), oracle.dequant_f32(m).astype(np.float64) @ x,
+                               rtol=1e-10, atol=1e-12)
+
+
+# ----------------------------------------------------------------- expert ---
+
+def _torch_expert(W1, W3, W2, x):
+    x = torch.as_tensor(x, dtype=torch.float64)
+    a = torch.nn.functional.silu(x @ torch.as_tensor(W1, dtype=torch.float64).T)
+    b = x @ torch.as_tensor(W3, dtype=torch.float64).T
+    return ((a * b) @ torch.as_tensor(W2, dtype=torch.float64).T).numpy()
+
+
+def test_expert_16bit_is_textbook_swiglu():
+    """bits = 16: the expert is the unquantised Mixtral FFN, W2 (silu(W1 x) * W3 x)."""
+    H, F = 24, 40
+    W = [synth.bf16_bits_to_f32(w) for w in synth.dense_expert_weights(9, 0, H, F, std=0.2)]
+    ms = [oracle.QMat(*w.shape, 8, 16, dense=w) for w in W]
+    x = np.random.default_rng(9).standard_normal(H)
+    np.testing.assert_allclose(oracle.expert(*ms, x), _torch_expert(*W, x), rtol=1e-10, atol=1e-12)
+
+
+def test_expert_operands_not_swapped():
+    """w1 carries the silu, w3 does not: swapping them changes the result."""
+    L = _rand_layer()
+    m = _mats(L)[0]
+    x = np.random.default_rng(10).standard_normal(L.H)
+    D = [oracle.dequant_f32(mm).astype(np.float64) for mm in m]
+    np.testing.assert_allclose(oracle.expert(*m, x), _torch_expert(D[0], D[1], D[2], x), rtol=1e-9, atol=1e-12)
+    assert not np.allclose(_torch_expert(D[1], D[0], D[2], x), _torch_expert(D[0], D[1], D[2], x))
+
+
+# ------------------------------------------------------------------ layer ---
+
+def _brute_layer(L, mats, mu, protect):
+    """Every expert on every token (library matmuls), then Eq. 1 / Eq. 5 by hand."""
+    D = [[oracle.dequant_f32(mm).astype(np.float64) for mm in me] for me in mats]
+    lg = torch.tensor(oracle.gate_logits(L.x_f32(), L.gate_f32()))
+    p = torch.softmax(lg, dim=1).numpy()
+    y = np.zeros((L.T, L.H))
+    for t in range(L.T):
+        outs = [_torch_expert(*D[e], L.x_f32()[t]) for e in range(L.E)]
+        best = None
+        for a, b in itertools.permutations(range(L.E), 2):  # exhaustive pair search
+            key = (np.float32(lg[t, a]), np.float32(lg[t, b]), -a, -b)
+            if np.float32(lg[t, a]) < np.float32(lg[t, b]) or (
+                    np.float32(lg[t, a]) == np.float32(lg[t, b]) and a > b):
+                continue
+            if best is None or key > best[0]:
+                best = (key, a, b)
+        _, a, b = best
+        # routing weights are carried in fp32 between the gate and the combine
+        wa = float(np.float32(p[t, a] / (p[t, a] + p[t, b])))
+        wb = float(np.float32(p[t, b] / (p[t, a] + p[t, b])))
+        prot = protect is not None and protect[t]
+        if not prot and wb / wa < mu:
+            y[t] = outs[a]
+        else:
+            y[t] = wa * outs[a] + wb * outs[b]
+    return y
+
+
+@pytest.mark.parametrize("mu", [0.0, 0.8])
+def test_layer_brute_force_tiny(mu):
+    L = _rand_layer(T=10, H=16, F=24, E=4, group=8, bits=(1, 2, 3, 2), seed=11,
+                    gate_std=0.5, protect_frac=0.3)
+    mats = _mats(L)
+    y, idx, w, pr = oracle.moe_layer(L.x_f32(), L.gate_f32(), mats, mu, L.protect)
+    if mu > 0:
+        assert 0 < pr.sum() < L.T  # the case exercises both branches
+    np.testing.assert_allclose(y, _brute_layer(L, mats, mu, L.protect), rtol=1e-9, atol=1e-12)
+
+
+def test_layer_token_subset_matches_full():
+    L = _rand_layer(T=10, H=16, F=24, E=4, group=8, seed=12, gate_std=0.5)
+    mats = _mats(L)
+    y, *_ = oracle.moe_layer(L.x_f32(), L.gate_f32(), mats, 0.5)
+    ys, *_ = oracle.moe_layer(L.x_f32(), L.gate_f32(), mats, 0.5, tokens=[7, 2])
+    np.testing.assert_array_equal(ys, y[[7, 2]])
+
+
+def test_layer_all_16bit_equals_unquantised_moe():
+    """All experts at 16 bits reproduce the unquantised Mixtral block (torch)."""
+    T, H, F, E = 6, 16, 32, 4
+    L = _rand_layer(T=T, H=H, F=F, E=E, experts=False, gate_std=0.5, seed=13)
+    W = [[synth.bf16_bits_to_f32(w) for w in synth.dense_expert_weights(13, e, H, F, std=0.2)]
+         for e in range(E)]
+    mats = [[oracle.QMat(*w.shape, 8, 16, dense=w) for w in We] for We in W]
+    y, idx, w, pr = oracle.moe_layer(L.x_f32(), L.gate_f32(), mats, 0.0)
+    xt = torch.tensor(L.x_f32(), dtype=torch.float64)
+    logits = xt @ torch.tensor(L.gate_f32(), dtype=torch.float64).T
+    top = torch.topk(torch.softmax(logits, 1), 2, dim=1)
+    ww = (top.values / top.values.sum(1, keepdim=True)).float().double()
+    want = np.zeros((T, H))
+    for t in range(T):
+        for s in range(2):
+            e = int(top.indices[t, s])
+            want[t] += float(ww[t, s]) * _torch_expert(*W[e], L.x_f32()[t])
+    np.testing.assert_allclose(y, want, rtol=1e-9, atol=1e-12)
+
+
+def test_rmsnorm_textbook():
+    x = np.random.default_rng(14).standard_normal(64)
+    g = np.random.default_rng(15).uniform(0.5, 1.5, 64).astype(np.float32)
+    xt = torch.tensor(x)
+    want = (xt * torch.rsqrt((xt * xt).mean() + 1e-5) * torch.tensor(g, dtype=torch.float64)).numpy()
+    np.testing.assert_allclose(oracle.rmsnorm(x, g), want, rtol=1e-12)
