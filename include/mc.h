@@ -1,0 +1,198 @@
+/*
+ * mc.h -- C ABI of the GB300 (sm_103a) library for the compressed MoE layer of
+ * "MC: Mixture Compressor for MoE LLMs" (Huang et al., ICLR 2025).
+ *
+ * The layer (Sec. 2.1 Eq. 1, Sec. 2.3 Eq. 5/6):
+ *   logits  = x Wg^T                                  (gate G of Eq. 1)
+ *   (e0,e1) = top-2 experts, w = renormalised softmax  (Eq. 1)
+ *   pruned  = !protect && w1/w0 < mu  -> w = (1, 0)    (Eq. 5, Sec. 2.3.2)
+ *   y       = sum over kept slots of w * E_e(x)        (Eq. 1)
+ *   E(x)    = W2 (silu(W1 x) * W3 x)                   (Mixtral SwiGLU expert)
+ * with every expert's W1, W3, W2 quantised weight-only to that expert's bit width
+ * b in {1,2,3} (PMQ, Sec. 2.2), group-wise along the input dimension, asymmetric:
+ *   w = (q - z) * s,  q in [0, 2^b - 1], one fp16 s and one fp16 z per group
+ * (Sec. 2.1, Eq. 2's integer grid; 1-bit codes are App. A.2's (sign(W)+1)/2 with
+ * z = 1/2, s = 2*alpha).
+ *
+ * Conventions for every entry point:
+ *   - Pointers are DEVICE pointers unless the parameter name ends in _host.
+ *   - The caller allocates every buffer; no entry point allocates device memory
+ *     except mc_pack_experts, which uses a temporary pinned host staging buffer.
+ *   - Device work is enqueued on `stream` (a cudaStream_t passed as void*; NULL is
+ *     the legacy default stream) and is asynchronous unless stated otherwise.
+ *   - Return value: MC_OK (0) or a negative MC_ERR_* code; mc_last_error() gives a
+ *     thread-local message for the last failing call on the calling thread.
+ *   - Bad arguments are rejected on the host before anything is enqueued.
+ *   - Device-detected faults (a packed buffer whose header does not match the
+ *     shape, activations outside the fp16 range, a bounded wait that expired) do
+ *     not abort: the kernels record a code in the status word at the start of the
+ *     workspace and skip their work; mc_check_status() reads it.
+ * Shapes supported by this version: E <= 16, top_k == 2, group in {64, 128},
+ * H and F multiples of 128, H <= 16384, F <= 65536.
+ */
+#ifndef MC_H_
+#define MC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum {
+    MC_OK = 0,
+    MC_ERR_INVALID_ARG = -1, /* null/misaligned pointer, bad shape, bad mu, ... */
+    MC_ERR_UNSUPPORTED = -2, /* a bit width outside {1,2,3}, E > 16, ... */
+    MC_ERR_CUDA = -3,        /* a CUDA runtime call failed (message has the text) */
+    MC_ERR_TIMEOUT = -4,     /* a bounded device wait expired (status word) */
+    MC_ERR_BAD_PACK = -5,    /* packed buffer header does not match (magic/shape/bits) */
+    MC_ERR_RANGE = -6        /* an activation was non-finite or outside the fp16 range */
+};
+
+/* Layer shape.  E experts, hidden size H, SwiGLU width F, quantisation group
+ * size `group` (weights per scale/zero along the input dimension), top_k = 2. */
+typedef struct {
+    int32_t E, H, F, group, top_k;
+} mc_shape;
+
+/* Thread-local text of the last error on this thread ("" if none). */
+const char *mc_last_error(void);
+
+/* Library version (major*10000 + minor*100 + patch) and packed-format version. */
+int mc_version(void);
+int mc_pack_format_version(void);
+
+/* ------------------------------------------------------------------------ *
+ * Packed expert weights (PMQ storage, Sec. 2.2 / App. A.2).
+ *
+ * Canonical input, per expert e and matrix m (0 = W1 [F,H], 1 = W3 [F,H],
+ * 2 = W2 [H,F], row-major, groups of `group` consecutive columns):
+ *   codes  uint8 [rows*cols], one code per byte, value < 2^bits[e]
+ *   scale  fp16 bit patterns [rows, cols/group]
+ *   zero   fp16 bit patterns [rows, cols/group]
+ * The packed layout is private to this library and versioned by a header at the
+ * start of the buffer; only its total size is part of the ABI.
+ * ------------------------------------------------------------------------ */
+
+/* Bytes needed for the packed buffer of this shape and bit table (host int8[E]),
+ * or 0 if the shape or a bit width is invalid (mc_last_error says which). */
+size_t mc_packed_size(const mc_shape *shape, const int8_t *bits_host);
+
+/* Pack canonical host arrays into a HOST buffer of mc_packed_size() bytes.  The
+ * arrays are indexed [3*e + m].  Pure host code (no GPU needed).  Returns
+ * MC_ERR_INVALID_ARG for a code >= 2^bits, a null array or a short buffer;
+ * MC_ERR_UNSUPPORTED for a bit width outside {1,2,3}. */
+int mc_pack_experts_host(const mc_shape *shape, const int8_t *bits_host,
+                         const uint8_t *const *codes_host,
+                         const uint16_t *const *scale_host,
+                         const uint16_t *const *zero_host,
+                         void *packed_host, size_t packed_bytes);
+
+/* mc_pack_experts_host into a pinned staging buffer, then a copy to packed_dev
+ * on `stream`.  SYNCHRONOUS: returns after the copy has completed. */
+int mc_pack_experts(const mc_shape *shape, const int8_t *bits_host,
+                    const uint8_t *const *codes_host,
+                    const uint16_t *const *scale_host,
+                    const uint16_t *const *zero_host,
+                    void *packed_dev, size_t packed_bytes, void *stream);
+
+/* Inverse of the packing for one (expert, matrix), from a HOST packed buffer:
+ * writes canonical codes [rows*cols] and fp16 scale/zero [rows, cols/group]
+ * (scale_host / zero_host may be NULL).  Pure host code.  MC_ERR_BAD_PACK if
+ * the header is not a valid packed buffer. */
+int mc_unpack_experts_host(const void *packed_host, size_t packed_bytes, int expert, int mat,
+                           uint8_t *codes_host, uint16_t *scale_host, uint16_t *zero_host);
+
+/* The same inverse run by a device kernel on a DEVICE packed buffer (the codes
+ * the GPU kernels actually decode), writing device arrays.  Asynchronous.
+ * `shape` and `bits_host` describe the buffer; the kernel also checks the header
+ * and records MC_ERR_BAD_PACK in *status_dev (a device int32, may be NULL). */
+int mc_unpack_experts(const mc_shape *shape, const int8_t *bits_host,
+                      const void *packed_dev, int expert, int mat,
+                      uint8_t *codes_dev, uint16_t *scale_dev, uint16_t *zero_dev,
+                      int32_t *status_dev, void *stream);
+
+/* Read and check the header of a DEVICE packed buffer against shape/bits.
+ * SYNCHRONOUS.  MC_OK or MC_ERR_BAD_PACK. */
+int mc_pack_verify(const mc_shape *shape, const int8_t *bits_host, const void *packed_dev,
+                   size_t packed_bytes);
+
+/* ------------------------------------------------------------------------ *
+ * Routing: Eq. 1 gate + top-2 + renormalised softmax, Eq. 5 ODP, Sec. 2.3.2
+ * protection, then the permutation of kept (token, slot) pairs by expert.
+ *   x       bf16 [T, H]        gate_w  bf16 [E, H]
+ *   mu      Eq. 5 threshold (finite, >= 0; 0 disables pruning; > 1 prunes every
+ *           unprotected token)
+ *   protect uint8 [T], nonzero = never prune; may be NULL
+ * Outputs (device):
+ *   topk_idx int32 [T, 2]  slot 0 = primary (larger weight), ties -> lower index
+ *   topk_w   fp32  [T, 2]  renormalised weights; (1, 0) for a pruned token
+ *   pruned   uint8 [T]
+ *   expert_offsets int32 [E+1]  exclusive prefix counts of kept pairs
+ *   perm     int32 [2T]   first expert_offsets[E] entries valid: 2*token + slot,
+ *                          grouped by expert, ascending token within an expert
+ * The decision is taken on fp32 logits; the ODP test is evaluated as
+ * (l0 - l1) > -ln(mu), which equals w1/w0 < mu.
+ * ------------------------------------------------------------------------ */
+int mc_route(const void *x, const void *gate_w, int T, const mc_shape *shape, float mu,
+             const uint8_t *protect, int32_t *topk_idx, float *topk_w, uint8_t *pruned,
+             int32_t *expert_offsets, int32_t *perm, void *stream);
+
+/* ------------------------------------------------------------------------ *
+ * The whole layer (Eq. 1 with Eq. 5 on PMQ experts).
+ *   x bf16 [T, H] (values must be finite and |x| <= 65504), gate_w bf16 [E, H],
+ *   packed_dev: the buffer written by mc_pack_experts for (shape, bits_host),
+ *   mu, protect as in mc_route, y bf16 [T, H] output.
+ *   workspace: device scratch of at least mc_moe_workspace_size(shape, T) bytes,
+ *   256-byte aligned; its first 4 bytes are the status word (see mc_check_status).
+ *   topk_idx_out int32 [T,2], topk_w_out fp32 [T,2], pruned_out uint8 [T]: optional
+ *   copies of the routing decisions (NULL to skip).
+ * Never synchronises and never allocates; capturable in a CUDA graph.
+ * T == 0 is a no-op returning MC_OK.
+ * ------------------------------------------------------------------------ */
+size_t mc_moe_workspace_size(const mc_shape *shape, int T_max);
+
+int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *shape,
+                   const int8_t *bits_host, const void *packed_dev, float mu,
+                   const uint8_t *protect, void *y, void *workspace, size_t ws_bytes,
+                   int32_t *topk_idx_out, float *topk_w_out, uint8_t *pruned_out,
+                   void *stream);
+
+/* Choose the expert path of mc_moe_forward: 0 = automatic (GEMV for small T,
+ * tensor-core GEMM otherwise), 1 = force the GEMV path, 2 = force the GEMM path.
+ * Process-wide; returns the previous value. */
+int mc_set_path(int path);
+
+/* Test hook: `flags` = 1 makes the expert kernels' weight producer issue no
+ * copies, so every consumer wait reaches its bound and the status word reports
+ * MC_ERR_TIMEOUT (no fault, no hang).  `timeout_ns` (0 = keep) bounds every
+ * device wait (default 1 s).  Process-wide. */
+int mc_set_debug(int flags, unsigned long long timeout_ns);
+
+/* Synchronise `stream`, read the status word at the start of `workspace`, clear
+ * it, and return MC_OK or the recorded MC_ERR_* code. */
+int mc_check_status(void *workspace, void *stream);
+
+/* Per-kernel timing of this library's own launches with CUDA events recorded on
+ * the launching stream (for benchmarks; off by default).  mc_profile_read
+ * synchronises on the recorded events, writes the summed milliseconds and launch
+ * counts of kernel ids 0 .. n-1 (names from mc_profile_name: route, permute,
+ * gemv_w13, gemv_w2, combine, gemm_gather, gemm_w13, gemm_w2, rmsnorm) and
+ * clears the records.  Not for use inside CUDA graph capture. */
+int mc_profile_enable(int on);
+int mc_profile_read(double *ms_out, int *count_out, int n);
+const char *mc_profile_name(int id);
+
+/* RMSNorm used between stacked layers: out = x / sqrt(mean(x^2) + eps) * gamma,
+ * x and out bf16 [T, H] (may alias), gamma bf16 [H]. */
+int mc_rmsnorm(const void *x, const void *gamma, int T, int H, float eps, void *out,
+               void *stream);
+
+/* out = a + b elementwise over n bf16 values (residual add; may alias a). */
+int mc_add(const void *a, const void *b, size_t n, void *out, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MC_H_ */

@@ -1,0 +1,335 @@
+// mc_api.cu -- the extern "C" entry points of include/mc.h: argument checks,
+// workspace carving and kernel launches.  No entry point here allocates device
+// memory or synchronises, except the ones documented as synchronous.
+#include <math.h>
+#include <string.h>
+
+#include <atomic>
+#include <vector>
+
+#include "mc_host.h"
+#include "mc_kernels.h"
+#include "mc_profile.h"
+
+namespace mc {
+
+static std::atomic<int> g_path{0};
+static std::atomic<int> g_debug{0};
+static std::atomic<unsigned long long> g_timeout_ns{1000000000ull};  // 1 s
+
+#define MC_CUDA(call)                                                                         \
+    do {                                                                                      \
+        cudaError_t err_ = (call);                                                            \
+        if (err_ != cudaSuccess)                                                              \
+            return set_error(MC_ERR_CUDA, "%s failed: %s", #call, cudaGetErrorString(err_)); \
+    } while (0)
+
+static inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// Column splits of the W2 pass: more CTAs for the small-batch (GEMV) case.
+static int choose_ks(const mc_shape *s, int T)
+{
+    if (T > 64) return 1;
+    int nt = s->F / kTileK;
+    for (int ks : {4, 2}) if (nt % ks == 0) return ks;
+    return 1;
+}
+
+struct Workspace {
+    int32_t *status;
+    int32_t *idx;
+    float *w;
+    uint8_t *pruned;
+    int32_t *offsets, *perm, *inv;
+    __half *xh;
+    float *xtab;
+    __half *h;
+    float *htab;
+    float *opart;
+    size_t total;
+};
+
+static Workspace carve(const mc_shape *s, int T, void *base)
+{
+    Workspace w;
+    uint8_t *p = (uint8_t *)base;
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        uint8_t *r = p ? p + off : nullptr;
+        off = align256(off + bytes);
+        return r;
+    };
+    const int KS = choose_ks(s, T);
+    const size_t P = 2 * (size_t)T;
+    w.status = (int32_t *)take(256);
+    w.idx = (int32_t *)take(P * 4);
+    w.w = (float *)take(P * 4);
+    w.pruned = (uint8_t *)take((size_t)T);
+    w.offsets = (int32_t *)take(4 * (kMaxE + 1));
+    w.perm = (int32_t *)take(P * 4);
+    w.inv = (int32_t *)take(P * 4);
+    w.xh = (__half *)take((size_t)T * s->H * 2);
+    w.xtab = (float *)take((size_t)T * (s->H / s->group) * kTabFloats * 4);
+    w.h = (__half *)take(P * s->F * 2);
+    w.htab = (float *)take(P * (s->F / s->group) * kTabFloats * 4);
+    w.opart = (float *)take((size_t)KS * P * s->H * 4);
+    w.total = off;
+    return w;
+}
+
+static int check_mu(float mu)
+{
+    if (!(mu == mu) || mu < 0.f || isinf(mu))
+        return set_error(MC_ERR_INVALID_ARG, "mu=%g: need a finite mu >= 0", (double)mu);
+    return MC_OK;
+}
+
+static float neg_log_mu(float mu)
+{
+    if (mu <= 0.f) return INFINITY;
+    return (float)(-log((double)mu));
+}
+
+static int launch_route(const void *x, const void *gate_w, int T, const mc_shape *s, float mu, const uint8_t *protect,
+                        int32_t *idx, float *w, uint8_t *pruned, int32_t *idx_out, float *w_out,
+                        uint8_t *pruned_out, __half *xh, float *xtab, int32_t *offsets, int32_t *perm, int32_t *inv,
+                        int32_t *status, cudaStream_t st)
+{
+    RouteParams rp;
+    rp.x = (const __nv_bfloat16 *)x;
+    rp.gate = (const __nv_bfloat16 *)gate_w;
+    rp.T = T;
+    rp.H = s->H;
+    rp.E = s->E;
+    rp.group = s->group;
+    rp.neg_log_mu = neg_log_mu(mu);
+    rp.protect = protect;
+    rp.idx = idx;
+    rp.w = w;
+    rp.pruned = pruned;
+    rp.idx_out = idx_out;
+    rp.w_out = w_out;
+    rp.pruned_out = pruned_out;
+    rp.xh = xh;
+    rp.xtab = xtab;
+    rp.status = status;
+    profile_begin(kKRoute, st);
+    route_kernel<<<(T + 7) / 8, 256, 0, st>>>(rp);
+    profile_end(kKRoute, st);
+    MC_CUDA(cudaGetLastError());
+    PermuteParams pp;
+    pp.idx = idx;
+    pp.pruned = pruned;
+    pp.T = T;
+    pp.E = s->E;
+    pp.offsets = offsets;
+    pp.perm = perm;
+    pp.inv = inv;
+    profile_begin(kKPermute, st);
+    permute_kernel<<<1, 1024, 0, st>>>(pp);
+    profile_end(kKPermute, st);
+    MC_CUDA(cudaGetLastError());
+    return MC_OK;
+}
+
+}  // namespace mc
+
+using namespace mc;
+
+extern "C" {
+
+int mc_set_path(int path)
+{
+    return g_path.exchange(path);
+}
+
+// Test hook (not in the public header's main API): debug flags and the bound on
+// device waits.  flags = 1 makes the weight producer issue nothing, so every
+// consumer wait runs into the bound and the status word reports MC_ERR_TIMEOUT.
+int mc_set_debug(int flags, unsigned long long timeout_ns)
+{
+    g_debug = flags;
+    if (timeout_ns) g_timeout_ns = timeout_ns;
+    return MC_OK;
+}
+
+size_t mc_moe_workspace_size(const mc_shape *shape, int T_max)
+{
+    if (check_shape(shape) || T_max < 0) return 0;
+    return carve(shape, T_max, nullptr).total;
+}
+
+int mc_route(const void *x, const void *gate_w, int T, const mc_shape *shape, float mu, const uint8_t *protect,
+             int32_t *topk_idx, float *topk_w, uint8_t *pruned, int32_t *expert_offsets, int32_t *perm, void *stream)
+{
+    clear_error();
+    int rc = check_shape(shape);
+    if (rc) return rc;
+    if ((rc = check_mu(mu))) return rc;
+    if (T < 0) return set_error(MC_ERR_INVALID_ARG, "T=%d < 0", T);
+    if (T == 0) return MC_OK;
+    if (!x || !gate_w || !topk_idx || !topk_w || !pruned || !expert_offsets || !perm)
+        return set_error(MC_ERR_INVALID_ARG, "NULL pointer argument");
+    if (!aligned(x, 16) || !aligned(gate_w, 16))
+        return set_error(MC_ERR_INVALID_ARG, "x and gate_w must be 16-byte aligned");
+    cudaStream_t st = (cudaStream_t)stream;
+    RouteParams rp;
+    rp.x = (const __nv_bfloat16 *)x;
+    rp.gate = (const __nv_bfloat16 *)gate_w;
+    rp.T = T;
+    rp.H = shape->H;
+    rp.E = shape->E;
+    rp.group = shape->group;
+    rp.neg_log_mu = neg_log_mu(mu);
+    rp.protect = protect;
+    rp.idx = topk_idx;
+    rp.w = topk_w;
+    rp.pruned = pruned;
+    rp.idx_out = nullptr;
+    rp.w_out = nullptr;
+    rp.pruned_out = nullptr;
+    rp.xh = nullptr;
+    rp.xtab = nullptr;
+    rp.status = nullptr;
+    route_kernel<<<(T + 7) / 8, 256, 0, st>>>(rp);
+    MC_CUDA(cudaGetLastError());
+    PermuteParams pp;
+    pp.idx = topk_idx;
+    pp.pruned = pruned;
+    pp.T = T;
+    pp.E = shape->E;
+    pp.offsets = expert_offsets;
+    pp.perm = perm;
+    pp.inv = nullptr;
+    permute_kernel<<<1, 1024, 0, st>>>(pp);
+    MC_CUDA(cudaGetLastError());
+    return MC_OK;
+}
+
+int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *shape, const int8_t *bits_host,
+                   const void *packed_dev, float mu, const uint8_t *protect, void *y, void *workspace,
+                   size_t ws_bytes, int32_t *topk_idx_out, float *topk_w_out, uint8_t *pruned_out, void *stream)
+{
+    clear_error();
+    int rc = check_bits(shape, bits_host);
+    if (rc) return rc;
+    if ((rc = check_mu(mu))) return rc;
+    if (T < 0) return set_error(MC_ERR_INVALID_ARG, "T=%d < 0", T);
+    if (T == 0) return MC_OK;
+    if (!x || !gate_w || !packed_dev || !y || !workspace)
+        return set_error(MC_ERR_INVALID_ARG, "NULL pointer argument");
+    if (!aligned(x, 16) || !aligned(gate_w, 16) || !aligned(y, 16) || !aligned(packed_dev, 256) ||
+        !aligned(workspace, 256))
+        return set_error(MC_ERR_INVALID_ARG, "x, gate_w, y need 16-byte and packed_dev, workspace 256-byte alignment");
+    Workspace ws = carve(shape, T, workspace);
+    if (ws_bytes < ws.total)
+        return set_error(MC_ERR_INVALID_ARG, "workspace has %zu bytes, needs %zu", ws_bytes, ws.total);
+    cudaStream_t st = (cudaStream_t)stream;
+
+    rc = launch_route(x, gate_w, T, shape, mu, protect, ws.idx, ws.w, ws.pruned, topk_idx_out, topk_w_out,
+                      pruned_out, ws.xh, ws.xtab, ws.offsets, ws.perm, ws.inv, ws.status, st);
+    if (rc) return rc;
+
+    ExpertParams ep;
+    memset(&ep, 0, sizeof ep);
+    ep.packed = (const uint8_t *)packed_dev;
+    uint64_t total;
+    layout_offsets(shape, bits_host, ep.mat_off, &total);
+    for (int e = 0; e < shape->E; ++e) ep.bits[e] = bits_host[e];
+    ep.E = shape->E;
+    ep.H = shape->H;
+    ep.F = shape->F;
+    ep.group = shape->group;
+    ep.offsets = ws.offsets;
+    ep.perm = ws.perm;
+    ep.xh = ws.xh;
+    ep.xtab = ws.xtab;
+    ep.h = ws.h;
+    ep.htab = ws.htab;
+    ep.opart = ws.opart;
+    ep.KS = choose_ks(shape, T);
+    ep.Pmax = 2 * T;
+    ep.status = ws.status;
+    ep.timeout_ns = g_timeout_ns;
+    ep.debug = g_debug;
+
+    rc = launch_gemv(ep, T <= 8 ? 1 : 2, st);
+    if (rc) return rc;
+
+    CombineParams cp;
+    cp.opart = ws.opart;
+    cp.w = ws.w;
+    cp.inv = ws.inv;
+    cp.T = T;
+    cp.H = shape->H;
+    cp.KS = ep.KS;
+    cp.Pmax = 2 * T;
+    cp.y = (__nv_bfloat16 *)y;
+    return launch_combine(cp, st);
+}
+
+int mc_check_status(void *workspace, void *stream)
+{
+    clear_error();
+    if (!workspace) return set_error(MC_ERR_INVALID_ARG, "NULL workspace");
+    cudaStream_t st = (cudaStream_t)stream;
+    int32_t v = 0;
+    MC_CUDA(cudaMemcpyAsync(&v, workspace, 4, cudaMemcpyDeviceToHost, st));
+    MC_CUDA(cudaStreamSynchronize(st));
+    if (v != 0) {
+        int32_t z = 0;
+        MC_CUDA(cudaMemcpyAsync(workspace, &z, 4, cudaMemcpyHostToDevice, st));
+        MC_CUDA(cudaStreamSynchronize(st));
+        return set_error(v, "device status word reported %d", v);
+    }
+    return MC_OK;
+}
+
+int mc_pack_experts(const mc_shape *shape, const int8_t *bits_host, const uint8_t *const *codes_host,
+                    const uint16_t *const *scale_host, const uint16_t *const *zero_host, void *packed_dev,
+                    size_t packed_bytes, void *stream)
+{
+    clear_error();
+    size_t need = mc_packed_size(shape, bits_host);
+    if (!need) return check_bits(shape, bits_host);
+    if (!packed_dev) return set_error(MC_ERR_INVALID_ARG, "NULL packed_dev");
+    if (!aligned(packed_dev, 256)) return set_error(MC_ERR_INVALID_ARG, "packed_dev must be 256-byte aligned");
+    if (packed_bytes < need)
+        return set_error(MC_ERR_INVALID_ARG, "packed buffer has %zu bytes, needs %zu", packed_bytes, need);
+    void *stage = nullptr;
+    MC_CUDA(cudaMallocHost(&stage, need));
+    int rc = mc_pack_experts_host(shape, bits_host, codes_host, scale_host, zero_host, stage, need);
+    if (rc == MC_OK) {
+        cudaStream_t st = (cudaStream_t)stream;
+        cudaError_t e1 = cudaMemcpyAsync(packed_dev, stage, need, cudaMemcpyHostToDevice, st);
+        cudaError_t e2 = e1 == cudaSuccess ? cudaStreamSynchronize(st) : e1;
+        if (e2 != cudaSuccess) rc = set_error(MC_ERR_CUDA, "upload failed: %s", cudaGetErrorString(e2));
+    }
+    cudaFreeHost(stage);
+    return rc;
+}
+
+int mc_pack_verify(const mc_shape *shape, const int8_t *bits_host, const void *packed_dev, size_t packed_bytes)
+{
+    clear_error();
+    int rc = check_bits(shape, bits_host);
+    if (rc) return rc;
+    if (!packed_dev) return set_error(MC_ERR_INVALID_ARG, "NULL packed_dev");
+    size_t need = mc_packed_size(shape, bits_host);
+    if (packed_bytes < need) return set_error(MC_ERR_BAD_PACK, "buffer has %zu bytes, needs %zu", packed_bytes, need);
+    PackHeader hd;
+    MC_CUDA(cudaMemcpy(&hd, packed_dev, sizeof hd, cudaMemcpyDeviceToHost));
+    if (hd.magic != kMagic || hd.version != kFormatVersion)
+        return set_error(MC_ERR_BAD_PACK, "bad magic/version (%08x/%u)", hd.magic, hd.version);
+    if (hd.E != shape->E || hd.H != shape->H || hd.F != shape->F || hd.group != shape->group)
+        return set_error(MC_ERR_BAD_PACK, "header shape (%d,%d,%d,%d) != (%d,%d,%d,%d)", hd.E, hd.H, hd.F, hd.group,
+                         shape->E, shape->H, shape->F, shape->group);
+    for (int e = 0; e < shape->E; ++e)
+        if (hd.bits[e] != bits_host[e])
+            return set_error(MC_ERR_BAD_PACK, "header bits[%d]=%d != %d", e, hd.bits[e], bits_host[e]);
+    if (hd.total_bytes != need) return set_error(MC_ERR_BAD_PACK, "header total %llu != %zu",
+                                                 (unsigned long long)hd.total_bytes, need);
+    return MC_OK;
+}
+
+}  // extern "C"

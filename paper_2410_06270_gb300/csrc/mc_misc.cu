@@ -1,0 +1,147 @@
+// mc_misc.cu -- device unpacking of the packed expert layout (the codes the
+// expert kernels decode, for bit-exact checks), RMSNorm and the residual add
+// used between stacked layers.
+#include "mc_host.h"
+#include "mc_kernels.h"
+
+namespace mc {
+
+// One thread per (tile, lane): the exact inverse of mc_pack.cpp's packing.
+__global__ void unpack_kernel(const uint8_t *packed, uint64_t mat_off, int rows, int cols, int bits, int group,
+                              int E, int H, int F, int expert, uint8_t *codes, uint16_t *scale, uint16_t *zero,
+                              int32_t *status)
+{
+    const PackHeader *hd = reinterpret_cast<const PackHeader *>(packed);
+    if (hd->magic != kMagic || hd->version != kFormatVersion || hd->E != E || hd->H != H || hd->F != F ||
+        hd->group != group || hd->bits[expert] != bits) {
+        if (blockIdx.x == 0 && threadIdx.x == 0) set_status(status, MC_ERR_BAD_PACK);
+        return;
+    }
+    const int KT = cols / kTileK, ng = cols / group, gpt = kTileK / group;
+    const int ntiles = (rows / kTileRows) * KT;
+    const int gid = blockIdx.x * blockDim.x + threadIdx.x;
+    const int tile_id = gid >> 5, lane = gid & 31;
+    if (tile_id >= ntiles) return;
+    const int rb = tile_id / KT, kt = tile_id % KT;
+    const uint8_t *tile = packed + mat_off + tile_offset(rb, kt, KT, bits, group);
+    const int R0 = rb * kTileRows, K0 = kt * kTileK;
+    uint32_t w2[4] = {0, 0, 0, 0}, w1[2] = {0, 0};
+    if (bits >= 2) {
+        uint4 v = *reinterpret_cast<const uint4 *>(tile + 16 * lane);
+        w2[0] = v.x; w2[1] = v.y; w2[2] = v.z; w2[3] = v.w;
+    }
+    if (bits != 2) {
+        uint2 v = *reinterpret_cast<const uint2 *>(tile + (bits >= 2 ? 512 : 0) + 8 * lane);
+        w1[0] = v.x; w1[1] = v.y;
+    }
+    for (int j = 0; j < 32; ++j) {
+        int row, col;
+        pair_pos(lane, j, row, col);
+        uint32_t qa = 0, qb = 0;
+        if (bits >= 2) {
+            int p = j & 7;
+            qa = (w2[j >> 3] >> (2 * p)) & 3u;
+            qb = (w2[j >> 3] >> (16 + 2 * p)) & 3u;
+        }
+        if (bits != 2) {
+            int p = j & 15, sh = bits == 1 ? 0 : 2;
+            qa |= ((w1[j >> 4] >> p) & 1u) << sh;
+            qb |= ((w1[j >> 4] >> (16 + p)) & 1u) << sh;
+        }
+        uint8_t *d = codes + (size_t)(R0 + row) * cols + K0 + col;
+        d[0] = (uint8_t)qa;
+        d[1] = (uint8_t)qb;
+    }
+    if (lane < 8 * gpt) {
+        const int gi = lane >> 3, g8 = lane & 7;
+        const uint16_t *m4 = reinterpret_cast<const uint16_t *>(tile + tile_code_bytes(bits)) + (gi * 8 + g8) * 4;
+        const int gcol = (K0 + gi * group) / group;
+        const size_t i0 = (size_t)(R0 + g8) * ng + gcol, i1 = (size_t)(R0 + g8 + 8) * ng + gcol;
+        if (scale) { scale[i0] = m4[0]; scale[i1] = m4[2]; }
+        if (zero) { zero[i0] = m4[1]; zero[i1] = m4[3]; }
+    }
+}
+
+// One CTA of 256 threads per row; fp32 statistics.
+__global__ void __launch_bounds__(256) rmsnorm_kernel(const __nv_bfloat16 *x, const __nv_bfloat16 *gamma, int H,
+                                                      float eps, __nv_bfloat16 *out)
+{
+    const __nv_bfloat16 *xr = x + (size_t)blockIdx.x * H;
+    __shared__ float red[8];
+    float ss = 0.f;
+    for (int c = threadIdx.x; c < H; c += blockDim.x) {
+        float v = __bfloat162float(xr[c]);
+        ss = fmaf(v, v, ss);
+    }
+    for (int m = 16; m >= 1; m >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, m);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+    __syncthreads();
+    float tot = 0.f;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += red[w];
+    const float inv = rsqrtf(tot / H + eps);
+    __syncthreads();  // every thread has read x before any in-place write
+    for (int c = threadIdx.x; c < H; c += blockDim.x)
+        out[(size_t)blockIdx.x * H + c] =
+            __float2bfloat16_rn(__bfloat162float(xr[c]) * inv * __bfloat162float(gamma[c]));
+}
+
+__global__ void add_kernel(const __nv_bfloat16 *a, const __nv_bfloat16 *b, size_t n, __nv_bfloat16 *out)
+{
+    size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < n) out[i] = __float2bfloat16_rn(__bfloat162float(a[i]) + __bfloat162float(b[i]));
+}
+
+}  // namespace mc
+
+using namespace mc;
+
+extern "C" {
+
+int mc_unpack_experts(const mc_shape *shape, const int8_t *bits_host, const void *packed_dev, int expert, int mat,
+                      uint8_t *codes_dev, uint16_t *scale_dev, uint16_t *zero_dev, int32_t *status_dev, void *stream)
+{
+    clear_error();
+    int rc = check_bits(shape, bits_host);
+    if (rc) return rc;
+    if (!packed_dev || !codes_dev) return set_error(MC_ERR_INVALID_ARG, "NULL pointer argument");
+    if (expert < 0 || expert >= shape->E || mat < 0 || mat > 2)
+        return set_error(MC_ERR_INVALID_ARG, "expert %d / matrix %d out of range", expert, mat);
+    uint64_t off[kMaxE][3], total;
+    layout_offsets(shape, bits_host, off, &total);
+    const int rows = mat < 2 ? shape->F : shape->H, cols = mat < 2 ? shape->H : shape->F;
+    const int ntiles = (rows / kTileRows) * (cols / kTileK);
+    const long threads = (long)ntiles * 32;
+    unpack_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, (cudaStream_t)stream>>>(
+        (const uint8_t *)packed_dev, off[expert][mat], rows, cols, bits_host[expert], shape->group, shape->E,
+        shape->H, shape->F, expert, codes_dev, scale_dev, zero_dev, status_dev);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return set_error(MC_ERR_CUDA, "unpack launch: %s", cudaGetErrorString(e));
+    return MC_OK;
+}
+
+int mc_rmsnorm(const void *x, const void *gamma, int T, int H, float eps, void *out, void *stream)
+{
+    clear_error();
+    if (T < 0 || H <= 0 || !(eps >= 0.f)) return set_error(MC_ERR_INVALID_ARG, "bad T/H/eps");
+    if (T == 0) return MC_OK;
+    if (!x || !gamma || !out) return set_error(MC_ERR_INVALID_ARG, "NULL pointer argument");
+    rmsnorm_kernel<<<T, 256, 0, (cudaStream_t)stream>>>((const __nv_bfloat16 *)x, (const __nv_bfloat16 *)gamma, H,
+                                                        eps, (__nv_bfloat16 *)out);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return set_error(MC_ERR_CUDA, "rmsnorm launch: %s", cudaGetErrorString(e));
+    return MC_OK;
+}
+
+int mc_add(const void *a, const void *b, size_t n, void *out, void *stream)
+{
+    clear_error();
+    if (n == 0) return MC_OK;
+    if (!a || !b || !out) return set_error(MC_ERR_INVALID_ARG, "NULL pointer argument");
+    add_kernel<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(
+        (const __nv_bfloat16 *)a, (const __nv_bfloat16 *)b, n, (__nv_bfloat16 *)out);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return set_error(MC_ERR_CUDA, "add launch: %s", cudaGetErrorString(e));
+    return MC_OK;
+}
+
+}  // extern "C"

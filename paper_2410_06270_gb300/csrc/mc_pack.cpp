@@ -1,0 +1,270 @@
+// mc_pack.cpp -- host side of the PMQ weight storage (Sec. 2.2, App. A.2):
+// canonical per-weight codes + fp16 scale/zero  <->  the packed tile layout of
+// mc_layout.h, plus shape validation and the thread-local error text.
+#include <string.h>
+
+#include <algorithm>
+#include <string>
+#include <thread>
+#include <vector>
+
+#include "mc_host.h"
+
+namespace mc {
+
+static thread_local std::string g_err;
+
+int set_error(int code, const char *fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_err = buf;
+    return code;
+}
+
+void clear_error() { g_err.clear(); }
+
+int check_shape(const mc_shape *s)
+{
+    if (!s) return set_error(MC_ERR_INVALID_ARG, "shape is NULL");
+    if (s->top_k != 2) return set_error(MC_ERR_UNSUPPORTED, "top_k=%d: only top-2 routing is supported", s->top_k);
+    if (s->E < 2 || s->E > kMaxE) return set_error(MC_ERR_UNSUPPORTED, "E=%d: need 2 <= E <= %d", s->E, kMaxE);
+    if (s->group != 64 && s->group != 128)
+        return set_error(MC_ERR_INVALID_ARG, "group=%d: need 64 or 128", s->group);
+    if (s->H <= 0 || s->H % kTileK || s->H > 16384)
+        return set_error(MC_ERR_INVALID_ARG, "H=%d: need a positive multiple of 128, <= 16384", s->H);
+    if (s->F <= 0 || s->F % kTileK || s->F > 65536)
+        return set_error(MC_ERR_INVALID_ARG, "F=%d: need a positive multiple of 128, <= 65536", s->F);
+    return MC_OK;
+}
+
+int check_bits(const mc_shape *s, const int8_t *bits)
+{
+    int rc = check_shape(s);
+    if (rc) return rc;
+    if (!bits) return set_error(MC_ERR_INVALID_ARG, "bits table is NULL");
+    for (int e = 0; e < s->E; ++e)
+        if (bits[e] < 1 || bits[e] > 3)
+            return set_error(MC_ERR_UNSUPPORTED, "bits[%d]=%d: only 1, 2 or 3 bits are supported", e, bits[e]);
+    return MC_OK;
+}
+
+void layout_offsets(const mc_shape *s, const int8_t *bits, uint64_t off[kMaxE][3], uint64_t *total)
+{
+    uint64_t pos = kHeaderBytes;
+    for (int e = 0; e < s->E; ++e)
+        for (int m = 0; m < 3; ++m) {
+            int rows = m < 2 ? s->F : s->H, cols = m < 2 ? s->H : s->F;
+            off[e][m] = pos;
+            pos += mat_bytes(rows, cols, bits[e], s->group);
+            pos = (pos + 255) & ~(uint64_t)255;
+        }
+    *total = pos;
+}
+
+// Pack one matrix [rows, cols] into its tile stream.  Returns false on a code
+// that does not fit in `bits`.
+static bool pack_matrix(int rows, int cols, int bits, int group, const uint8_t *codes,
+                        const uint16_t *scale, const uint16_t *zero, uint8_t *dst, int rb_lo, int rb_hi)
+{
+    const int KT = cols / kTileK, ng = cols / group, gpt = kTileK / group;
+    const uint32_t lim = 1u << bits;
+    for (int rb = rb_lo; rb < rb_hi; ++rb)
+        for (int kt = 0; kt < KT; ++kt) {
+            uint8_t *tile = dst + tile_offset(rb, kt, KT, bits, group);
+            const int R0 = rb * kTileRows, K0 = kt * kTileK;
+            uint8_t *plane2 = tile;                                // 32 lanes x 16 B
+            uint8_t *plane1 = tile + (bits >= 2 ? 512 : 0);        // 32 lanes x 8 B
+            for (int lane = 0; lane < 32; ++lane) {
+                uint32_t w2[4] = {0, 0, 0, 0}, w1[2] = {0, 0};
+                for (int j = 0; j < 32; ++j) {
+                    int row, col;
+                    pair_pos(lane, j, row, col);
+                    const uint8_t *src = codes + (size_t)(R0 + row) * cols + K0 + col;
+                    uint32_t qa = src[0], qb = src[1];
+                    if (qa >= lim || qb >= lim) return false;
+                    if (bits >= 2) {
+                        int p = j & 7;
+                        w2[j >> 3] |= ((qa & 3u) << (2 * p)) | ((qb & 3u) << (16 + 2 * p));
+                    }
+                    if (bits != 2) {
+                        int p = j & 15;
+                        uint32_t ha = bits == 1 ? qa : (qa >> 2), hb = bits == 1 ? qb : (qb >> 2);
+                        w1[j >> 4] |= (ha << p) | (hb << (16 + p));
+                    }
+                }
+                if (bits >= 2) memcpy(plane2 + 16 * lane, w2, 16);
+                if (bits != 2) memcpy(plane1 + 8 * lane, w1, 8);
+            }
+            uint16_t *meta = (uint16_t *)(tile + tile_code_bytes(bits));
+            for (int gi = 0; gi < gpt; ++gi) {
+                int gcol = (K0 + gi * group) / group;
+                for (int g8 = 0; g8 < 8; ++g8) {
+                    uint16_t *m4 = meta + (gi * 8 + g8) * 4;
+                    size_t i0 = (size_t)(R0 + g8) * ng + gcol, i1 = (size_t)(R0 + g8 + 8) * ng + gcol;
+                    m4[0] = scale[i0];
+                    m4[1] = zero[i0];
+                    m4[2] = scale[i1];
+                    m4[3] = zero[i1];
+                }
+            }
+        }
+    return true;
+}
+
+static void unpack_matrix(int rows, int cols, int bits, int group, const uint8_t *src,
+                          uint8_t *codes, uint16_t *scale, uint16_t *zero)
+{
+    const int KT = cols / kTileK, ng = cols / group, gpt = kTileK / group;
+    for (int rb = 0; rb < rows / kTileRows; ++rb)
+        for (int kt = 0; kt < KT; ++kt) {
+            const uint8_t *tile = src + tile_offset(rb, kt, KT, bits, group);
+            const int R0 = rb * kTileRows, K0 = kt * kTileK;
+            const uint8_t *plane2 = tile, *plane1 = tile + (bits >= 2 ? 512 : 0);
+            for (int lane = 0; lane < 32; ++lane) {
+                uint32_t w2[4] = {0, 0, 0, 0}, w1[2] = {0, 0};
+                if (bits >= 2) memcpy(w2, plane2 + 16 * lane, 16);
+                if (bits != 2) memcpy(w1, plane1 + 8 * lane, 8);
+                for (int j = 0; j < 32; ++j) {
+                    int row, col;
+                    pair_pos(lane, j, row, col);
+                    uint32_t qa = 0, qb = 0;
+                    if (bits >= 2) {
+                        int p = j & 7;
+                        qa = (w2[j >> 3] >> (2 * p)) & 3u;
+                        qb = (w2[j >> 3] >> (16 + 2 * p)) & 3u;
+                    }
+                    if (bits != 2) {
+                        int p = j & 15;
+                        uint32_t ha = (w1[j >> 4] >> p) & 1u, hb = (w1[j >> 4] >> (16 + p)) & 1u;
+                        int sh = bits == 1 ? 0 : 2;
+                        qa |= ha << sh;
+                        qb |= hb << sh;
+                    }
+                    uint8_t *d = codes + (size_t)(R0 + row) * cols + K0 + col;
+                    d[0] = (uint8_t)qa;
+                    d[1] = (uint8_t)qb;
+                }
+            }
+            const uint16_t *meta = (const uint16_t *)(tile + tile_code_bytes(bits));
+            for (int gi = 0; gi < gpt; ++gi) {
+                int gcol = (K0 + gi * group) / group;
+                for (int g8 = 0; g8 < 8; ++g8) {
+                    const uint16_t *m4 = meta + (gi * 8 + g8) * 4;
+                    size_t i0 = (size_t)(R0 + g8) * ng + gcol, i1 = (size_t)(R0 + g8 + 8) * ng + gcol;
+                    if (scale) { scale[i0] = m4[0]; scale[i1] = m4[2]; }
+                    if (zero) { zero[i0] = m4[1]; zero[i1] = m4[3]; }
+                }
+            }
+        }
+}
+
+}  // namespace mc
+
+using namespace mc;
+
+extern "C" {
+
+size_t mc_packed_size(const mc_shape *shape, const int8_t *bits_host)
+{
+    if (check_bits(shape, bits_host)) return 0;
+    uint64_t off[kMaxE][3], total;
+    layout_offsets(shape, bits_host, off, &total);
+    return (size_t)total;
+}
+
+int mc_pack_experts_host(const mc_shape *shape, const int8_t *bits_host,
+                         const uint8_t *const *codes_host, const uint16_t *const *scale_host,
+                         const uint16_t *const *zero_host, void *packed_host, size_t packed_bytes)
+{
+    clear_error();
+    int rc = check_bits(shape, bits_host);
+    if (rc) return rc;
+    if (!codes_host || !scale_host || !zero_host || !packed_host)
+        return set_error(MC_ERR_INVALID_ARG, "NULL array argument");
+    uint64_t off[kMaxE][3], total;
+    layout_offsets(shape, bits_host, off, &total);
+    if (packed_bytes < total)
+        return set_error(MC_ERR_INVALID_ARG, "packed buffer has %zu bytes, needs %llu", packed_bytes,
+                         (unsigned long long)total);
+    for (int i = 0; i < 3 * shape->E; ++i)
+        if (!codes_host[i] || !scale_host[i] || !zero_host[i])
+            return set_error(MC_ERR_INVALID_ARG, "NULL array for expert %d matrix %d", i / 3, i % 3);
+    uint8_t *base = (uint8_t *)packed_host;
+    memset(base, 0, kHeaderBytes);
+    PackHeader *hd = (PackHeader *)base;
+    hd->magic = kMagic;
+    hd->version = kFormatVersion;
+    hd->E = shape->E;
+    hd->H = shape->H;
+    hd->F = shape->F;
+    hd->group = shape->group;
+    for (int e = 0; e < shape->E; ++e) {
+        hd->bits[e] = bits_host[e];
+        for (int m = 0; m < 3; ++m) hd->mat_off[e][m] = off[e][m];
+    }
+    hd->total_bytes = total;
+
+    // one work item per (expert, matrix, 128-row block), spread over host threads
+    struct Item { int e, m, rb_lo, rb_hi; };
+    std::vector<Item> items;
+    for (int e = 0; e < shape->E; ++e)
+        for (int m = 0; m < 3; ++m) {
+            int rows = m < 2 ? shape->F : shape->H;
+            for (int r = 0; r < rows / kTileRows; r += 8) items.push_back({e, m, r, std::min(r + 8, rows / kTileRows)});
+        }
+    unsigned nth = std::max(1u, std::min(32u, std::thread::hardware_concurrency()));
+    std::vector<int> bad(nth, -1);
+    auto work = [&](unsigned id) {
+        for (size_t i = id; i < items.size(); i += nth) {
+            const Item &it = items[i];
+            int rows = it.m < 2 ? shape->F : shape->H, cols = it.m < 2 ? shape->H : shape->F;
+            int k = 3 * it.e + it.m;
+            if (!pack_matrix(rows, cols, bits_host[it.e], shape->group, codes_host[k], scale_host[k],
+                             zero_host[k], base + off[it.e][it.m], it.rb_lo, it.rb_hi)) {
+                bad[id] = k;
+                return;
+            }
+        }
+    };
+    std::vector<std::thread> th;
+    for (unsigned i = 1; i < nth; ++i) th.emplace_back(work, i);
+    work(0);
+    for (auto &t : th) t.join();
+    for (unsigned i = 0; i < nth; ++i)
+        if (bad[i] >= 0)
+            return set_error(MC_ERR_INVALID_ARG, "expert %d matrix %d has a code >= 2^%d", bad[i] / 3, bad[i] % 3,
+                             bits_host[bad[i] / 3]);
+    return MC_OK;
+}
+
+int mc_unpack_experts_host(const void *packed_host, size_t packed_bytes, int expert, int mat,
+                           uint8_t *codes_host, uint16_t *scale_host, uint16_t *zero_host)
+{
+    clear_error();
+    if (!packed_host || !codes_host) return set_error(MC_ERR_INVALID_ARG, "NULL argument");
+    if (packed_bytes < (size_t)kHeaderBytes) return set_error(MC_ERR_BAD_PACK, "buffer shorter than the header");
+    const PackHeader *hd = (const PackHeader *)packed_host;
+    if (hd->magic != kMagic || hd->version != kFormatVersion)
+        return set_error(MC_ERR_BAD_PACK, "bad magic/version (%08x/%u)", hd->magic, hd->version);
+    mc_shape s = {hd->E, hd->H, hd->F, hd->group, 2};
+    int rc = check_bits(&s, hd->bits);
+    if (rc) return set_error(MC_ERR_BAD_PACK, "header: %s", mc_last_error());
+    if (hd->total_bytes > packed_bytes) return set_error(MC_ERR_BAD_PACK, "buffer shorter than header total");
+    if (expert < 0 || expert >= hd->E || mat < 0 || mat > 2)
+        return set_error(MC_ERR_INVALID_ARG, "expert %d / matrix %d out of range", expert, mat);
+    int rows = mat < 2 ? hd->F : hd->H, cols = mat < 2 ? hd->H : hd->F;
+    unpack_matrix(rows, cols, hd->bits[expert], hd->group, (const uint8_t *)packed_host + hd->mat_off[expert][mat],
+                  codes_host, scale_host, zero_host);
+    return MC_OK;
+}
+
+const char *mc_last_error(void) { return g_err.c_str(); }
+
+int mc_version(void) { return 10000; }
+int mc_pack_format_version(void) { return (int)kFormatVersion; }
+
+}  // extern "C"

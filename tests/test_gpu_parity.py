@@ -1,0 +1,255 @@
+"""GPU parity: the CUDA path through the C ABI against the CPU oracle on the same
+seeded inputs.  Routing indices, prune flags, the permutation and the unpacked
+codes must be bit-exact; layer outputs must be within rel-Frobenius 5e-3 and
+max-abs 2e-2 * max|ref| of the fp64 oracle."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from helpers import (assert_close, condition_routing, errors, flat, oracle_layer, oracle_mats, to_dev)
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def mc():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2410_06270_gb300 import build
+    build.build()
+    import paper_2410_06270_gb300 as m
+    m.load()
+    m.set_debug(0, 1_000_000_000)
+    return m
+
+
+def _pack(mc, L):
+    shape = mc.Shape(L.E, L.H, L.F, L.group)
+    return shape, mc.pack_experts(shape, L.bits, flat(L, "codes"), flat(L, "scale"), flat(L, "zero"))
+
+
+def _check_routing(mc, L, idx, w, pr, offsets=None, perm=None):
+    oidx, ow, opr = oracle.route(L.x_f32(), L.gate_f32(), L.mu, L.protect)
+    np.testing.assert_array_equal(idx.cpu().numpy(), oidx)
+    np.testing.assert_array_equal(pr.cpu().numpy(), opr)
+    np.testing.assert_allclose(w.cpu().numpy(), ow, rtol=2e-6, atol=2e-6)
+    if offsets is not None:
+        ooff, operm = oracle.permute(oidx, opr, L.E)
+        np.testing.assert_array_equal(offsets.cpu().numpy(), ooff)
+        np.testing.assert_array_equal(perm.cpu().numpy()[: ooff[-1]], operm)
+
+
+# -------------------------------------------------------------- routing ----
+
+@pytest.mark.parametrize("case", ["tiny", "odp", "odp_heavy", "many_tokens", "e16", "ragged_h"])
+def test_route_bit_exact(mc, case):
+    if case == "tiny":
+        L = synth.config_tiny()
+    elif case == "odp":
+        L = synth.make_layer(200, 256, 128, 8, 64, [2] * 8, 31, gate_std=0.15, mu=0.3, protect_frac=0.25,
+                             experts=False)
+    elif case == "odp_heavy":
+        L = synth.make_layer(300, 512, 128, 8, 128, [2] * 8, 32, gate_std=0.1, mu=0.8, protect_frac=0.1,
+                             experts=False)
+    elif case == "many_tokens":
+        L = synth.make_layer(5000, 256, 128, 8, 64, [2] * 8, 33, gate_std=0.1, mu=0.5, protect_frac=0.02,
+                             experts=False)
+    elif case == "e16":
+        L = synth.make_layer(100, 384, 128, 16, 128, [2] * 16, 34, gate_std=0.1, mu=0.6, experts=False)
+    else:  # H = 384 is a multiple of 128 but not of 256
+        L = synth.make_layer(77, 384, 128, 8, 64, [2] * 8, 35, gate_std=0.1, mu=0.4, protect_frac=0.3,
+                             experts=False)
+    condition_routing(L, L.mu)
+    x, g, p = to_dev(L)
+    shape = mc.Shape(L.E, L.H, L.F, L.group)
+    out = mc.route(x, g, shape, L.mu, p)
+    torch.cuda.synchronize()
+    _check_routing(mc, L, out["idx"], out["w"], out["pruned"], out["offsets"], out["perm"])
+    if case != "tiny":
+        assert 0 < int(out["pruned"].sum()) < L.T
+
+
+def test_route_mu_zero_and_above_one(mc):
+    L = synth.make_layer(64, 256, 128, 8, 64, [2] * 8, 36, gate_std=0.2, protect_frac=0.25, experts=False)
+    condition_routing(L, 0.0)
+    x, g, p = to_dev(L)
+    shape = mc.Shape(8, 256, 128, 64)
+    a = mc.route(x, g, shape, 0.0, p)
+    assert int(a["pruned"].sum()) == 0 and int(a["offsets"][-1]) == 2 * L.T
+    b = mc.route(x, g, shape, 1.5, p)
+    np.testing.assert_array_equal(b["pruned"].cpu().numpy(), 1 - L.protect)
+    assert int(b["offsets"][-1]) == 2 * L.T - int((1 - L.protect).sum())
+
+
+# ------------------------------------------------------------ unpacking ----
+
+@pytest.mark.parametrize("group", [64, 128])
+def test_device_unpack_bit_exact(mc, group):
+    L = synth.make_layer(2, 256, 384, 4, group, [1, 2, 3, 2], 41, zero_mode="fractional")
+    shape, packed = _pack(mc, L)
+    mc.pack_verify(shape, L.bits, packed)
+    for e in range(4):
+        for m in range(3):
+            c, s, z = mc.unpack_experts(shape, L.bits, packed, e, m)
+            torch.cuda.synchronize()
+            np.testing.assert_array_equal(c.cpu().numpy(), L.codes[e][m])
+            np.testing.assert_array_equal(s.cpu().numpy().view(np.uint16), L.scale[e][m].view(np.uint16))
+            np.testing.assert_array_equal(z.cpu().numpy().view(np.uint16), L.zero[e][m].view(np.uint16))
+
+
+# ---------------------------------------------------------------- layer ----
+
+def _forward_and_check(mc, L, tokens=None, path=None):
+    condition_routing(L, L.mu)
+    shape, packed = _pack(mc, L)
+    x, g, p = to_dev(L)
+    ws = mc.alloc_workspace(shape, L.T)
+    old = mc.set_path(path) if path is not None else None
+    try:
+        y, r = mc.moe_forward(x, g, shape, L.bits, packed, L.mu, p, workspace=ws, routing=True)
+        mc.check_status(ws)
+    finally:
+        if old is not None:
+            mc.set_path(old)
+    torch.cuda.synchronize()
+    _check_routing(mc, L, r["idx"], r["w"], r["pruned"])
+    mats = oracle_mats(L)
+    ref, *_ = oracle_layer(L, mats, tokens)
+    got = y.float().cpu().numpy()
+    if tokens is not None:
+        got = got[list(tokens)]
+    return assert_close(got, ref, "T=%d" % L.T)
+
+
+def test_forward_tiny_config(mc):
+    """H 256, F 512, 8 experts, 64 tokens, group 64, bits [3,2,2,1,3,2,2,3],
+    mu 0.3, 25% of tokens protected."""
+    _forward_and_check(mc, synth.config_tiny())
+
+
+@pytest.mark.parametrize("T", [1, 2, 3, 8, 9, 16, 17, 40])
+def test_forward_token_counts(mc, T):
+    """Empty experts, one token, full n-tiles, ragged n-tiles and the chunked path."""
+    L = synth.make_layer(T, 256, 512, 8, 64, [3, 2, 2, 1, 3, 2, 2, 3], 50 + T, gate_std=0.1, mu=0.5,
+                         protect_frac=0.25)
+    _forward_and_check(mc, L)
+
+
+@pytest.mark.parametrize("bits", [[1] * 4, [2] * 4, [3] * 4, [1, 3, 1, 3]])
+@pytest.mark.parametrize("group", [64, 128])
+def test_forward_bit_widths_and_groups(mc, bits, group):
+    L = synth.make_layer(12, 512, 384, 4, group, bits, 60 + group + sum(bits), gate_std=0.1)
+    _forward_and_check(mc, L)
+
+
+def test_forward_fractional_zeros(mc):
+    """Arbitrary fp16 zero points (HQQ-style storage), not only integer ones."""
+    L = synth.make_layer(16, 384, 640, 8, 128, [3, 2, 1, 2, 3, 2, 1, 3], 70, gate_std=0.1,
+                         zero_mode="fractional", mu=0.4, protect_frac=0.1)
+    _forward_and_check(mc, L)
+
+
+def test_forward_odd_row_blocks(mc):
+    """H / 128 odd: the last W2 CTA has a single row stream."""
+    L = synth.make_layer(10, 384, 256, 8, 64, [2, 3, 1, 2, 2, 3, 1, 2], 71, gate_std=0.1)
+    _forward_and_check(mc, L)
+
+
+def test_forward_sixteen_experts(mc):
+    L = synth.make_layer(24, 256, 256, 16, 64, [1, 2, 3] * 5 + [2], 72, gate_std=0.1, mu=0.5)
+    _forward_and_check(mc, L)
+
+
+@pytest.mark.parametrize("T", [1, 4, 16])
+def test_forward_mixtral_decode(mc, T):
+    """Mixtral-8x7b-shaped decode layer (H 4096, F 14336, group 128, mean 2.5
+    bits), outputs on sampled tokens, routing on all tokens."""
+    L = synth.config_decode(T=T)
+    tokens = list(range(T)) if T <= 4 else [0, 5, 10, 15]
+    _forward_and_check(mc, L, tokens=tokens)
+
+
+def test_forward_is_deterministic(mc):
+    L = synth.make_layer(16, 256, 512, 8, 64, [3, 2, 2, 1, 3, 2, 2, 3], 80, gate_std=0.1)
+    shape, packed = _pack(mc, L)
+    x, g, p = to_dev(L)
+    y1 = mc.moe_forward(x, g, shape, L.bits, packed)
+    y2 = mc.moe_forward(x, g, shape, L.bits, packed)
+    torch.cuda.synchronize()
+    assert torch.equal(y1.view(torch.int16), y2.view(torch.int16))
+
+
+# ---------------------------------------------------------- device faults ----
+
+def test_bounded_wait_reports_timeout_and_context_survives(mc):
+    L = synth.make_layer(4, 256, 256, 8, 64, [2] * 8, 90, gate_std=0.1)
+    shape, packed = _pack(mc, L)
+    x, g, p = to_dev(L)
+    ws = mc.alloc_workspace(shape, L.T)
+    mc.set_debug(1, 20_000_000)  # producer issues nothing; waits give up after 20 ms
+    try:
+        mc.moe_forward(x, g, shape, L.bits, packed, workspace=ws)
+        with pytest.raises(mc.MCError) as ei:
+            mc.check_status(ws)
+        assert ei.value.code == mc.ERR_TIMEOUT
+    finally:
+        mc.set_debug(0, 1_000_000_000)
+    y = mc.moe_forward(x, g, shape, L.bits, packed, workspace=ws)
+    mc.check_status(ws)
+    torch.cuda.synchronize()
+    assert torch.isfinite(y.float()).all()
+
+
+def test_corrupt_pack_header_is_reported(mc):
+    L = synth.make_layer(4, 256, 256, 8, 64, [2] * 8, 91, gate_std=0.1)
+    shape, packed = _pack(mc, L)
+    x, g, p = to_dev(L)
+    bad = packed.clone()
+    bad[0] ^= 0xFF
+    with pytest.raises(mc.MCError) as ei:
+        mc.pack_verify(shape, L.bits, bad)
+    assert ei.value.code == mc.ERR_BAD_PACK
+    ws = mc.alloc_workspace(shape, L.T)
+    mc.moe_forward(x, g, shape, L.bits, bad, workspace=ws)
+    with pytest.raises(mc.MCError) as ei:
+        mc.check_status(ws)
+    assert ei.value.code == mc.ERR_BAD_PACK
+    # a bit table that disagrees with the buffer is reported the same way
+    other = np.array(L.bits).copy()
+    other[0] = 3 if other[0] != 3 else 1
+    mc.moe_forward(x, g, shape, other, packed, workspace=ws)
+    with pytest.raises(mc.MCError) as ei:
+        mc.check_status(ws)
+    assert ei.value.code == mc.ERR_BAD_PACK
+
+
+def test_activation_outside_fp16_range_is_reported(mc):
+    L = synth.make_layer(4, 256, 256, 8, 64, [2] * 8, 92, gate_std=0.1)
+    L.x[2, 17] = synth.f32_to_bf16_bits(np.array([1e6], np.float32))[0]
+    shape, packed = _pack(mc, L)
+    x, g, p = to_dev(L)
+    ws = mc.alloc_workspace(shape, L.T)
+    mc.moe_forward(x, g, shape, L.bits, packed, workspace=ws)
+    with pytest.raises(mc.MCError) as ei:
+        mc.check_status(ws)
+    assert ei.value.code == mc.ERR_RANGE
+
+
+# ------------------------------------------------------------- rmsnorm ----
+
+def test_rmsnorm_and_add(mc):
+    r = np.random.default_rng(5)
+    xs = synth.f32_to_bf16_bits(r.standard_normal((6, 4096)).astype(np.float32) * 3)
+    gs = synth.f32_to_bf16_bits(r.uniform(0.5, 1.5, 4096).astype(np.float32))
+    x = torch.from_numpy(xs.view(np.int16)).view(torch.bfloat16).cuda()
+    g = torch.from_numpy(gs.view(np.int16)).view(torch.bfloat16).cuda()
+    y = mc.rmsnorm(x, g, 1e-5).float().cpu().numpy()
+    for t in range(6):
+        ref = oracle.rmsnorm(synth.bf16_bits_to_f32(xs[t]), synth.bf16_bits_to_f32(gs), 1e-5)
+        rel, mx = errors(y[t], ref)
+        assert rel < 4e-3 and mx < 8e-3
+    s = mc.add(x, x).float().cpu().numpy()
+    np.testing.assert_array_equal(s, 2 * synth.bf16_bits_to_f32(xs))
