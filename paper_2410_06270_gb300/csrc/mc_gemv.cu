@@ -333,12 +333,17 @@ __device__ __forceinline__ void gemv_body(const ExpertParams &p, uint8_t *smem, 
     }
 }
 
-// The packed buffer must carry the header written for this shape and bit table.
+// The packed buffer must carry the header written for this shape and bit table:
+// the expert's bit width and the byte offsets of its matrices (which depend on
+// every earlier expert's width) must match what the host computed, so a CTA never
+// reads outside the region the buffer was packed with.
 __device__ __forceinline__ bool header_ok(const ExpertParams &p, int e)
 {
     const PackHeader *hd = reinterpret_cast<const PackHeader *>(p.packed);
     const bool ok = hd->magic == kMagic && hd->version == kFormatVersion && hd->E == p.E && hd->H == p.H &&
-                    hd->F == p.F && hd->group == p.group && hd->bits[e] == p.bits[e];
+                    hd->F == p.F && hd->group == p.group && hd->bits[e] == p.bits[e] &&
+                    hd->mat_off[e][0] == p.mat_off[e][0] && hd->mat_off[e][1] == p.mat_off[e][1] &&
+                    hd->mat_off[e][2] == p.mat_off[e][2];
     if (!ok && threadIdx.x == 0) set_status(p.status, MC_ERR_BAD_PACK);
     return ok;
 }

@@ -77,5 +77,6 @@ def errors(got, ref):
 
 def assert_close(got, ref, what=""):
     rel, mx = errors(got, ref)
+    print("[parity] %s rel_fro=%.3e max_abs/max=%.3e" % (what, rel, mx))
     assert rel <= REL_FRO and mx <= MAX_ABS, "%s rel_fro=%.3e max_abs/max=%.3e" % (what, rel, mx)
     return rel, mx

@@ -121,7 +121,8 @@ def _forward_and_check(mc, L, tokens=None, path=None):
     got = y.float().cpu().numpy()
     if tokens is not None:
         got = got[list(tokens)]
-    return assert_close(got, ref, "T=%d" % L.T)
+    return assert_close(got, ref, "T=%d H=%d F=%d E=%d g=%d bits=%s mu=%g" % (
+        L.T, L.H, L.F, L.E, L.group, list(map(int, L.bits)), L.mu))
 
 
 def test_forward_tiny_config(mc):
@@ -217,13 +218,19 @@ def test_corrupt_pack_header_is_reported(mc):
     with pytest.raises(mc.MCError) as ei:
         mc.check_status(ws)
     assert ei.value.code == mc.ERR_BAD_PACK
-    # a bit table that disagrees with the buffer is reported the same way
-    other = np.array(L.bits).copy()
-    other[0] = 3 if other[0] != 3 else 1
-    mc.moe_forward(x, g, shape, other, packed, workspace=ws)
-    with pytest.raises(mc.MCError) as ei:
-        mc.check_status(ws)
-    assert ei.value.code == mc.ERR_BAD_PACK
+    # a bit table that disagrees with the buffer is reported the same way, both
+    # when the wrong entry is a routed expert's and when it only shifts the
+    # offsets of the experts after it (expert 0 untouched by these tokens)
+    idx, _, _ = oracle.route(L.x_f32(), L.gate_f32(), 0.0)
+    touched = sorted(set(idx.reshape(-1).tolist()))
+    untouched = [e for e in range(L.E) if e not in touched]
+    for e in [touched[0]] + untouched[:1]:
+        other = np.array(L.bits).copy()
+        other[e] = 3 if other[e] != 3 else 1
+        mc.moe_forward(x, g, shape, other, packed, workspace=ws)
+        with pytest.raises(mc.MCError) as ei:
+            mc.check_status(ws)
+        assert ei.value.code == mc.ERR_BAD_PACK
 
 
 def test_activation_outside_fp16_range_is_reported(mc):
