@@ -41,11 +41,14 @@ struct Workspace {
     float *w;
     uint8_t *pruned;
     int32_t *offsets, *perm, *inv;
-    __half *xh;
+    ChunkInfo *chunks;
+    int32_t *nchunks, *counters;
+    uint8_t *xfrag;
     float *xtab;
-    __half *h;
+    uint8_t *hfrag;
     float *htab;
     float *opart;
+    int max_chunks, KS;
     size_t total;
 };
 
@@ -59,8 +62,10 @@ static Workspace carve(const mc_shape *s, int T, void *base)
         off = align256(off + bytes);
         return r;
     };
-    const int KS = choose_ks(s, T);
-    const size_t P = 2 * (size_t)T;
+    w.KS = choose_ks(s, T);
+    w.max_chunks = max_chunks_for(T, s->E);
+    const size_t P = 2 * (size_t)T, MC = (size_t)w.max_chunks;
+    const size_t tb = (size_t)tab_bytes(s->group);
     w.status = (int32_t *)take(256);
     w.idx = (int32_t *)take(P * 4);
     w.w = (float *)take(P * 4);
@@ -68,11 +73,14 @@ static Workspace carve(const mc_shape *s, int T, void *base)
     w.offsets = (int32_t *)take(4 * (kMaxE + 1));
     w.perm = (int32_t *)take(P * 4);
     w.inv = (int32_t *)take(P * 4);
-    w.xh = (__half *)take((size_t)T * s->H * 2);
-    w.xtab = (float *)take((size_t)T * (s->H / s->group) * kTabFloats * 4);
-    w.h = (__half *)take(P * s->F * 2);
-    w.htab = (float *)take(P * (s->F / s->group) * kTabFloats * 4);
-    w.opart = (float *)take((size_t)KS * P * s->H * 4);
+    w.chunks = (ChunkInfo *)take(MC * sizeof(ChunkInfo));
+    w.nchunks = (int32_t *)take(4);
+    w.counters = (int32_t *)take(16);
+    w.xfrag = (uint8_t *)take(MC * (s->H / kTileK) * kFragBytes);
+    w.xtab = (float *)take(MC * (s->H / kTileK) * tb);
+    w.hfrag = (uint8_t *)take(MC * (s->F / kTileK) * kFragBytes);
+    w.htab = (float *)take(MC * (s->F / kTileK) * tb);
+    w.opart = (float *)take((size_t)w.KS * P * s->H * 4);
     w.total = off;
     return w;
 }
@@ -88,48 +96,6 @@ static float neg_log_mu(float mu)
 {
     if (mu <= 0.f) return INFINITY;
     return (float)(-log((double)mu));
-}
-
-static int launch_route(const void *x, const void *gate_w, int T, const mc_shape *s, float mu, const uint8_t *protect,
-                        int32_t *idx, float *w, uint8_t *pruned, int32_t *idx_out, float *w_out,
-                        uint8_t *pruned_out, __half *xh, float *xtab, int32_t *offsets, int32_t *perm, int32_t *inv,
-                        int32_t *status, cudaStream_t st)
-{
-    RouteParams rp;
-    rp.x = (const __nv_bfloat16 *)x;
-    rp.gate = (const __nv_bfloat16 *)gate_w;
-    rp.T = T;
-    rp.H = s->H;
-    rp.E = s->E;
-    rp.group = s->group;
-    rp.neg_log_mu = neg_log_mu(mu);
-    rp.protect = protect;
-    rp.idx = idx;
-    rp.w = w;
-    rp.pruned = pruned;
-    rp.idx_out = idx_out;
-    rp.w_out = w_out;
-    rp.pruned_out = pruned_out;
-    rp.xh = xh;
-    rp.xtab = xtab;
-    rp.status = status;
-    profile_begin(kKRoute, st);
-    route_kernel<<<(T + 7) / 8, 256, 0, st>>>(rp);
-    profile_end(kKRoute, st);
-    MC_CUDA(cudaGetLastError());
-    PermuteParams pp;
-    pp.idx = idx;
-    pp.pruned = pruned;
-    pp.T = T;
-    pp.E = s->E;
-    pp.offsets = offsets;
-    pp.perm = perm;
-    pp.inv = inv;
-    profile_begin(kKPermute, st);
-    permute_kernel<<<1, 1024, 0, st>>>(pp);
-    profile_end(kKPermute, st);
-    MC_CUDA(cudaGetLastError());
-    return MC_OK;
 }
 
 }  // namespace mc
@@ -172,38 +138,27 @@ int mc_route(const void *x, const void *gate_w, int T, const mc_shape *shape, fl
         return set_error(MC_ERR_INVALID_ARG, "NULL pointer argument");
     if (!aligned(x, 16) || !aligned(gate_w, 16))
         return set_error(MC_ERR_INVALID_ARG, "x and gate_w must be 16-byte aligned");
-    cudaStream_t st = (cudaStream_t)stream;
     RouteParams rp;
+    memset(&rp, 0, sizeof rp);
     rp.x = (const __nv_bfloat16 *)x;
     rp.gate = (const __nv_bfloat16 *)gate_w;
     rp.T = T;
     rp.H = shape->H;
     rp.E = shape->E;
-    rp.group = shape->group;
     rp.neg_log_mu = neg_log_mu(mu);
     rp.protect = protect;
     rp.idx = topk_idx;
     rp.w = topk_w;
     rp.pruned = pruned;
-    rp.idx_out = nullptr;
-    rp.w_out = nullptr;
-    rp.pruned_out = nullptr;
-    rp.xh = nullptr;
-    rp.xtab = nullptr;
-    rp.status = nullptr;
-    route_kernel<<<(T + 7) / 8, 256, 0, st>>>(rp);
-    MC_CUDA(cudaGetLastError());
     PermuteParams pp;
+    memset(&pp, 0, sizeof pp);
     pp.idx = topk_idx;
     pp.pruned = pruned;
     pp.T = T;
     pp.E = shape->E;
     pp.offsets = expert_offsets;
     pp.perm = perm;
-    pp.inv = nullptr;
-    permute_kernel<<<1, 1024, 0, st>>>(pp);
-    MC_CUDA(cudaGetLastError());
-    return MC_OK;
+    return launch_route(rp, pp, (cudaStream_t)stream);
 }
 
 int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *shape, const int8_t *bits_host,
@@ -226,8 +181,35 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
         return set_error(MC_ERR_INVALID_ARG, "workspace has %zu bytes, needs %zu", ws_bytes, ws.total);
     cudaStream_t st = (cudaStream_t)stream;
 
-    rc = launch_route(x, gate_w, T, shape, mu, protect, ws.idx, ws.w, ws.pruned, topk_idx_out, topk_w_out,
-                      pruned_out, ws.xh, ws.xtab, ws.offsets, ws.perm, ws.inv, ws.status, st);
+    RouteParams rp;
+    memset(&rp, 0, sizeof rp);
+    rp.x = (const __nv_bfloat16 *)x;
+    rp.gate = (const __nv_bfloat16 *)gate_w;
+    rp.T = T;
+    rp.H = shape->H;
+    rp.E = shape->E;
+    rp.neg_log_mu = neg_log_mu(mu);
+    rp.protect = protect;
+    rp.idx = ws.idx;
+    rp.w = ws.w;
+    rp.pruned = ws.pruned;
+    rp.idx_out = topk_idx_out;
+    rp.w_out = topk_w_out;
+    rp.pruned_out = pruned_out;
+    PermuteParams pp;
+    memset(&pp, 0, sizeof pp);
+    pp.idx = ws.idx;
+    pp.pruned = ws.pruned;
+    pp.T = T;
+    pp.E = shape->E;
+    for (int e = 0; e < shape->E; ++e) pp.bits[e] = bits_host[e];
+    pp.offsets = ws.offsets;
+    pp.perm = ws.perm;
+    pp.inv = ws.inv;
+    pp.chunks = ws.chunks;
+    pp.nchunks = ws.nchunks;
+    pp.counters = ws.counters;
+    rc = launch_route(rp, pp, st);
     if (rc) return rc;
 
     ExpertParams ep;
@@ -240,20 +222,23 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     ep.H = shape->H;
     ep.F = shape->F;
     ep.group = shape->group;
-    ep.offsets = ws.offsets;
+    ep.chunks = ws.chunks;
+    ep.nchunks = ws.nchunks;
+    ep.counters = ws.counters;
+    ep.x = (const __nv_bfloat16 *)x;
     ep.perm = ws.perm;
-    ep.xh = ws.xh;
+    ep.xfrag = ws.xfrag;
     ep.xtab = ws.xtab;
-    ep.h = ws.h;
+    ep.hfrag = ws.hfrag;
     ep.htab = ws.htab;
     ep.opart = ws.opart;
-    ep.KS = choose_ks(shape, T);
+    ep.KS = ws.KS;
     ep.Pmax = 2 * T;
+    ep.max_chunks = ws.max_chunks;
     ep.status = ws.status;
     ep.timeout_ns = g_timeout_ns;
     ep.debug = g_debug;
-
-    rc = launch_gemv(ep, T <= 8 ? 1 : 2, st);
+    rc = launch_gemv(ep, st);
     if (rc) return rc;
 
     CombineParams cp;
@@ -262,7 +247,7 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     cp.inv = ws.inv;
     cp.T = T;
     cp.H = shape->H;
-    cp.KS = ep.KS;
+    cp.KS = ws.KS;
     cp.Pmax = 2 * T;
     cp.y = (__nv_bfloat16 *)y;
     return launch_combine(cp, st);

@@ -1,4 +1,4 @@
-// mc_kernels.h -- kernel parameter blocks and launch declarations shared by the
+// mc_kernels.h -- kernel parameter blocks and host launchers shared by the
 // translation units of the library (host side: mc_api.cu).
 #pragma once
 #include <cuda_runtime.h>
@@ -7,10 +7,30 @@
 
 namespace mc {
 
+// Activations of up to 16 pairs of one expert ("chunk") are processed together:
+// two mma n-tiles of 8.  NT = 1 when the chunk has at most 8 pairs.
+constexpr int kChunk = 16;
+
+// One chunk of one expert, written by permute_kernel in the order the expert
+// kernels schedule them (experts with more bits first).
+struct ChunkInfo {
+    int32_t e;          // expert
+    int32_t pair_base;  // first pair (position in perm) of the chunk
+    int32_t nv;         // valid pairs, 1..16
+    int32_t bits;
+};
+
+// Fragment-ordered activations of one chunk and one 128-column tile:
+//   frag [j (2)][s (8)][lane (32)] x 8 bytes = 4 fp16 (B operand of mma k-step s,
+//   n-tile j); j-major so that an NT = 1 chunk copies only the first 2 KB.
+constexpr int kFragBytes = 2 * 8 * 32 * 8;
+// Offset tables of one chunk and one tile: [n (16)][group-in-tile][8 floats].
+__host__ __device__ inline int tab_bytes(int group) { return kChunk * (kTileK / group) * kTabFloats * 4; }
+
 struct RouteParams {
     const __nv_bfloat16 *x;     // [T, H]
     const __nv_bfloat16 *gate;  // [E, H]
-    int T, H, E, group;
+    int T, H, E;
     float neg_log_mu;           // prune iff (l0 - l1) > neg_log_mu  (+inf: never)
     const uint8_t *protect;     // [T] or null
     int32_t *idx;               // [T, 2]
@@ -19,35 +39,41 @@ struct RouteParams {
     int32_t *idx_out;           // optional copies
     float *w_out;
     uint8_t *pruned_out;
-    __half *xh;                 // [T, H] fp16 copy, or null (routing only)
-    float *xtab;                // [T, H/group, 8]
-    int32_t *status;
 };
 
 struct PermuteParams {
     const int32_t *idx;
     const uint8_t *pruned;
     int T, E;
-    int32_t *offsets;  // [E+1]
-    int32_t *perm;     // [2T]
-    int32_t *inv;      // [2T]
+    int8_t bits[kMaxE];
+    int32_t *offsets;     // [E+1]
+    int32_t *perm;        // [2T]
+    int32_t *inv;         // [2T] or null
+    ChunkInfo *chunks;    // [max_chunks] or null
+    int32_t *nchunks;     // [1]
+    int32_t *counters;    // [4] work counters of the expert kernels, reset here
 };
 
-// Expert GEMV/GEMM work description shared by the decode and prefill kernels.
+// Decode-path expert kernels (persistent, mma.sync).
 struct ExpertParams {
     const uint8_t *packed;
     uint64_t mat_off[kMaxE][3];
     int8_t bits[kMaxE];
     int E, H, F, group;
-    const int32_t *offsets;  // [E+1]
+    const ChunkInfo *chunks;
+    const int32_t *nchunks;
+    int32_t *counters;
+    const __nv_bfloat16 *x;  // [T, H]
     const int32_t *perm;     // [P]
-    const __half *xh;        // [T, H]
-    const float *xtab;       // [T, H/g, 8]
-    __half *h;               // [Pmax, F]   SwiGLU output, pair order
-    float *htab;             // [Pmax, F/g, 8]
+    uint8_t *xfrag;          // [max_chunks][H/128] kFragBytes
+    float *xtab;             // [max_chunks][H/128] tab_bytes
+    uint8_t *hfrag;          // [max_chunks][F/128] kFragBytes
+    float *htab;             // [max_chunks][F/128] tab_bytes
     float *opart;            // [KS, Pmax, H]  expert outputs (fp32), pair order
     int KS;                  // column splits of the W2 pass
     int Pmax;                // 2 * T
+    int max_chunks;
+    int nslots;              // stages of the shared-memory ring
     int32_t *status;
     uint64_t timeout_ns;
     int debug;               // test hooks (kDebugNoProducer)
@@ -63,14 +89,10 @@ struct CombineParams {
     __nv_bfloat16 *y;     // [T, H]
 };
 
-__global__ void route_kernel(RouteParams p);
-__global__ void permute_kernel(PermuteParams p);
-__global__ void combine_kernel(CombineParams p);
-
-// decode (mma.sync) expert kernels; NT = n-tiles of 8 pairs per expert.
-// Host launchers return MC_OK or an MC_ERR_* code with the message set.
-int launch_gemv(const ExpertParams &ep, int NT, cudaStream_t st);
+// Host launchers: MC_OK or an MC_ERR_* code with the message set.
+int launch_route(const RouteParams &rp, const PermuteParams &pp, cudaStream_t st);
+int launch_gemv(ExpertParams ep, cudaStream_t st);
 int launch_combine(const CombineParams &cp, cudaStream_t st);
-size_t gemv_smem_bytes(int NT, bool w13, const ExpertParams &p);
+int max_chunks_for(int T, int E);
 
 }  // namespace mc

@@ -2,33 +2,33 @@
 // weights, the ODP test of Eq. 5 with the token protection of Sec. 2.3.2, and the
 // permutation of kept (token, slot) pairs by expert.
 //
-// route_kernel: one warp per token.  The warp streams the token's bf16 row once
-// (16-byte loads) and, in the same pass, writes the fp16 copy the expert kernels
-// consume plus the per-group offset tables of mc_layout.h.
+// route_kernel: one CTA of 4 warps per token; each warp takes a quarter of the
+//   row (16-byte loads of x and of the gate rows), the partial logits meet in
+//   shared memory and thread 0 takes the decision in fp32.
 // permute_kernel: one CTA; histogram, exclusive scan and a stable placement with
-// __match_any_sync ranks, so the permutation is unique (ascending token within an
-// expert) and identical run to run.
+//   __match_any_sync ranks, so the permutation is unique (ascending token within
+//   an expert) and identical run to run.  It also lists the work chunks of the
+//   expert kernels and resets their work counters.
+#include "mc_host.h"
 #include "mc_kernels.h"
+#include "mc_profile.h"
 
 namespace mc {
 
-__global__ void __launch_bounds__(256) route_kernel(RouteParams p)
+constexpr int kRouteWarps = 4;
+
+__global__ void __launch_bounds__(kRouteWarps * 32) route_kernel(RouteParams p)
 {
-    const int lane = threadIdx.x & 31;
-    const int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    if (t >= p.T) return;
+    __shared__ float part[kRouteWarps][kMaxE];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int t = blockIdx.x;
     const int H = p.H, E = p.E;
     const __nv_bfloat16 *xr = p.x + (size_t)t * H;
     float acc[kMaxE];
 #pragma unroll
     for (int e = 0; e < kMaxE; ++e) acc[e] = 0.f;
-    bool bad = false;
-    // lanes of one half-warp cover 128 consecutive columns per iteration; every
-    // lane runs every iteration (H is a multiple of 128, not always of 256)
-    for (int it = 0; it < (H + 255) / 256; ++it) {
-        const int c0 = it * 256 + 8 * lane;
-        const bool act = c0 < H;
-        uint4 raw = act ? *reinterpret_cast<const uint4 *>(xr + c0) : make_uint4(0, 0, 0, 0);
+    for (int c0 = 8 * (threadIdx.x); c0 < H; c0 += 8 * 32 * kRouteWarps) {
+        uint4 raw = *reinterpret_cast<const uint4 *>(xr + c0);
         const __nv_bfloat162 *x2 = reinterpret_cast<const __nv_bfloat162 *>(&raw);
         float xf[8];
 #pragma unroll
@@ -39,7 +39,7 @@ __global__ void __launch_bounds__(256) route_kernel(RouteParams p)
         }
 #pragma unroll
         for (int e = 0; e < kMaxE; ++e) {
-            if (e < E && act) {
+            if (e < E) {
                 uint4 gr = *reinterpret_cast<const uint4 *>(p.gate + (size_t)e * H + c0);
                 const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gr);
 #pragma unroll
@@ -50,54 +50,32 @@ __global__ void __launch_bounds__(256) route_kernel(RouteParams p)
                 }
             }
         }
-        if (p.xh) {
-            // fp16 copy for the tensor-core expert kernels + offset tables
-            __half hv[8];
-            float tab[7] = {0, 0, 0, 0, 0, 0, 0};
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                if (!(fabsf(xf[i]) <= 65504.f)) bad = true;
-                hv[i] = __float2half_rn(xf[i]);
-                float v = __half2float(hv[i]);
-                int col = (c0 + i) & (kTileK - 1);
-                int j0 = pair_of_col(col, 0), j1 = pair_of_col(col, 1);
-                tab[0] += v;
-                tab[1] = fmaf(off1(j0), v, tab[1]);
-                tab[2] = fmaf(off1(j1), v, tab[2]);
-                tab[3] = fmaf(off2(j0), v, tab[3]);
-                tab[4] = fmaf(off2(j1), v, tab[4]);
-            }
-            if (act) *reinterpret_cast<uint4 *>(p.xh + (size_t)t * H + c0) = *reinterpret_cast<uint4 *>(hv);
-            // reduce over the lanes sharing a quantisation group (8 cols per lane)
-            const int lanes_per_group = p.group / 8;  // 8 or 16
-#pragma unroll
-            for (int k = 0; k < 5; ++k)
-                for (int m = 1; m < lanes_per_group; m <<= 1) tab[k] += __shfl_xor_sync(0xffffffffu, tab[k], m);
-            if (act && (lane & (lanes_per_group - 1)) == 0) {
-                int G = c0 / p.group, ng = H / p.group;
-                float4 *dst = reinterpret_cast<float4 *>(p.xtab + ((size_t)t * ng + G) * kTabFloats);
-                dst[0] = make_float4(tab[0], tab[1], tab[2], tab[3]);
-                dst[1] = make_float4(tab[4], tab[3] + 4.f * tab[1], tab[4] + 4.f * tab[2], 0.f);
-            }
-        }
     }
 #pragma unroll
-    for (int e = 0; e < kMaxE; ++e)
+    for (int e = 0; e < kMaxE; ++e) {
         for (int m = 16; m >= 1; m >>= 1) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], m);
-    if (p.xh && __any_sync(0xffffffffu, bad) && lane == 0) set_status(p.status, MC_ERR_RANGE);
-    if (lane != 0) return;
+        if (lane == 0) part[warp][e] = acc[e];
+    }
+    __syncthreads();
+    if (threadIdx.x != 0) return;
+    float l[kMaxE];
+    for (int e = 0; e < E; ++e) {
+        float s = 0.f;
+        for (int w = 0; w < kRouteWarps; ++w) s += part[w][e];
+        l[e] = s;
+    }
     // top-2 on fp32 logits, lower index wins ties
     int e0 = 0;
     for (int e = 1; e < E; ++e)
-        if (acc[e] > acc[e0]) e0 = e;
+        if (l[e] > l[e0]) e0 = e;
     int e1 = e0 == 0 ? 1 : 0;
     for (int e = 0; e < E; ++e)
-        if (e != e0 && acc[e] > acc[e1]) e1 = e;
-    float d = acc[e0] - acc[e1];  // >= 0
-    float r = __expf(-d);         // = p1 / p0
+        if (e != e0 && l[e] > l[e1]) e1 = e;
+    const float d = l[e0] - l[e1];  // >= 0
+    const float r = __expf(-d);     // = p1 / p0
     float w0 = 1.f / (1.f + r), w1 = r / (1.f + r);
-    bool prot = p.protect != nullptr && p.protect[t] != 0;
-    bool prune = !prot && (d > p.neg_log_mu);
+    const bool prot = p.protect != nullptr && p.protect[t] != 0;
+    const bool prune = !prot && (d > p.neg_log_mu);
     if (prune) {
         w0 = 1.f;
         w1 = 0.f;
@@ -143,6 +121,24 @@ __global__ void __launch_bounds__(1024) permute_kernel(PermuteParams p)
             s += cnt[e];
         }
         p.offsets[p.E] = s;
+        if (p.chunks) {
+            // work chunks of <= 16 pairs, experts with more bits first
+            int k = 0;
+            for (int b = 3; b >= 1; --b)
+                for (int e = 0; e < p.E; ++e) {
+                    if (p.bits[e] != b) continue;
+                    for (int c = 0; c < cnt[e]; c += kChunk) {
+                        ChunkInfo ci;
+                        ci.e = e;
+                        ci.pair_base = run[e] + c;
+                        ci.nv = min(kChunk, cnt[e] - c);
+                        ci.bits = b;
+                        p.chunks[k++] = ci;
+                    }
+                }
+            *p.nchunks = k;
+            for (int i = 0; i < 4; ++i) p.counters[i] = 0;
+        }
     }
     __syncthreads();
     for (int base = 0; base < NP; base += blockDim.x) {
@@ -175,6 +171,23 @@ __global__ void __launch_bounds__(1024) permute_kernel(PermuteParams p)
         }
         __syncthreads();
     }
+}
+
+int max_chunks_for(int T, int E) { return (2 * T + kChunk - 1) / kChunk + E; }
+
+int launch_route(const RouteParams &rp, const PermuteParams &pp, cudaStream_t st)
+{
+    profile_begin(kKRoute, st);
+    route_kernel<<<rp.T, kRouteWarps * 32, 0, st>>>(rp);
+    profile_end(kKRoute, st);
+    cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "route launch: %s", cudaGetErrorString(err));
+    profile_begin(kKPermute, st);
+    permute_kernel<<<1, 1024, 0, st>>>(pp);
+    profile_end(kKPermute, st);
+    err = cudaGetLastError();
+    if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "permute launch: %s", cudaGetErrorString(err));
+    return MC_OK;
 }
 
 }  // namespace mc

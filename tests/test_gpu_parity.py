@@ -223,8 +223,8 @@ def test_corrupt_pack_header_is_reported(mc):
     # offsets of the experts after it (expert 0 untouched by these tokens)
     idx, _, _ = oracle.route(L.x_f32(), L.gate_f32(), 0.0)
     touched = sorted(set(idx.reshape(-1).tolist()))
-    untouched = [e for e in range(L.E) if e not in touched]
-    for e in [touched[0]] + untouched[:1]:
+    shifting = [e for e in range(L.E) if e not in touched and any(t > e for t in touched)]
+    for e in [touched[0]] + shifting[:1]:
         other = np.array(L.bits).copy()
         other[e] = 3 if other[e] != 3 else 1
         mc.moe_forward(x, g, shape, other, packed, workspace=ws)
