@@ -108,17 +108,19 @@ __device__ __forceinline__ void write_tables(const __half *rows, int ntok, int g
             for (int m = 16; m >= 1; m >>= 1) tb[k] += __shfl_xor_sync(0xffffffffu, tb[k], m);
         if (lane == 0) {
             float4 *d = reinterpret_cast<float4 *>(dst + (size_t)item * kTabFloats);
-            d[0] = make_float4(tb[0], tb[1], tb[2], tb[3]);
-            d[1] = make_float4(tb[4], tb[3] + 4.f * tb[1], tb[4] + 4.f * tb[2], 0.f);
+            d[0] = make_float4(tb[0], 0.f, tb[1], tb[2]);
+            d[1] = make_float4(tb[3], tb[4], tb[3] + 4.f * tb[1], tb[4] + 4.f * tb[2]);
         }
     }
 }
 
-// Fragment entries (j < NT) of a [16][128] fp16 tile held in shared memory.
+// Fragment entries (j < NT) of a [16][128] fp16 tile held in shared memory,
+// 8 bytes each, ordered [j][s/2][lane][s%2] so that one 16-byte load gives a
+// lane its B fragments of k-steps 2q and 2q+1.
 __device__ __forceinline__ void write_frags(const __half *rows, int NT, uint8_t *dst, int tid, int nthreads)
 {
     for (int idx = tid; idx < NT * 256; idx += nthreads) {
-        const int j = idx >> 8, s = (idx >> 5) & 7, ln = idx & 31;
+        const int j = idx >> 8, s = 2 * ((idx >> 6) & 3) + (idx & 1), ln = (idx >> 1) & 31;
         const int n = 8 * j + (ln >> 2), t = ln & 3;
         const int col = 64 * (s >> 2) + 16 * t + 4 * (s & 3);
         reinterpret_cast<uint2 *>(dst)[idx] = *reinterpret_cast<const uint2 *>(rows + n * kTileK + col);
@@ -164,7 +166,7 @@ __global__ void __launch_bounds__(256) frag_x_kernel(ExpertParams p)
 // fold.  Accumulates into y[j][c] (C-fragment layout, rows g8 / g8+8, pairs
 // 8j + 2t + {0,1}).
 template <int NT, int BITS>
-__device__ __forceinline__ void stage_compute(const uint8_t *tile, const uint2 *frag, const float *tab, int group,
+__device__ __forceinline__ void stage_compute(const uint8_t *tile, const uint4 *frag, const float *tab, int group,
                                               int lane, float (&y)[2][4])
 {
     const int gpt = kTileK / group;
@@ -181,30 +183,41 @@ __device__ __forceinline__ void stage_compute(const uint8_t *tile, const uint2 *
     uint2 meta[2];
     meta[0] = *reinterpret_cast<const uint2 *>(mt + (lane >> 2) * 8);
     meta[1] = gpt == 2 ? *reinterpret_cast<const uint2 *>(mt + 64 + (lane >> 2) * 8) : meta[0];
-    constexpr int oa = 2 * BITS - 1;  // table index of O for row half 0 (half 1: oa + 1)
-    float acc[NT][4];
+    // two independent accumulators halve the dependent mma chain: 1/2-bit by
+    // k-step parity, 3-bit low plane / high plane
+    float acc[2][NT][4];
 #pragma unroll
-    for (int j = 0; j < NT; ++j)
+    for (int a = 0; a < 2; ++a)
 #pragma unroll
-        for (int c = 0; c < 4; ++c) acc[j][c] = 0.f;
+        for (int j = 0; j < NT; ++j)
+#pragma unroll
+            for (int c = 0; c < 4; ++c) acc[a][j][c] = 0.f;
 #pragma unroll
     for (int qd = 0; qd < 4; ++qd) {
         uint32_t r[8], rh[8];
         if (BITS == 1) cvt1_half<false>(c1[qd >> 1], 8 * (qd & 1), r);
         if (BITS >= 2) cvt2(c2[qd], r);
         if (BITS == 3) cvt1_half<true>(c1[qd >> 1], 8 * (qd & 1), rh);
+        uint4 bq[NT];
+#pragma unroll
+        for (int j = 0; j < NT; ++j) bq[j] = frag[(j * 4 + qd) * 32 + lane];
 #pragma unroll
         for (int kk = 0; kk < 2; ++kk) {
             const int s = 2 * qd + kk;
 #pragma unroll
             for (int j = 0; j < NT; ++j) {
-                const uint2 b = frag[(j * 8 + s) * 32 + lane];
-                mma16816(acc[j], r[4 * kk], r[4 * kk + 1], r[4 * kk + 2], r[4 * kk + 3], b.x, b.y);
-                if (BITS == 3) mma16816(acc[j], rh[4 * kk], rh[4 * kk + 1], rh[4 * kk + 2], rh[4 * kk + 3], b.x, b.y);
+                const uint32_t b0 = kk ? bq[j].z : bq[j].x, b1 = kk ? bq[j].w : bq[j].y;
+                if (BITS == 3) {
+                    mma16816(acc[0][j], r[4 * kk], r[4 * kk + 1], r[4 * kk + 2], r[4 * kk + 3], b0, b1);
+                    mma16816(acc[1][j], rh[4 * kk], rh[4 * kk + 1], rh[4 * kk + 2], rh[4 * kk + 3], b0, b1);
+                } else {
+                    mma16816(acc[kk][j], r[4 * kk], r[4 * kk + 1], r[4 * kk + 2], r[4 * kk + 3], b0, b1);
+                }
             }
             if ((s == 3 && gpt == 2) || s == 7) {
                 const int gi = s == 3 ? 0 : gpt - 1;
-                const __half2 *m2 = reinterpret_cast<const __half2 *>(&meta[gi]);
+                const uint2 mg = gi == 0 ? meta[0] : meta[1];  // no dynamic index: keeps meta in registers
+                const __half2 *m2 = reinterpret_cast<const __half2 *>(&mg);
                 const float2 sz0 = __half22float2(m2[0]), sz1 = __half22float2(m2[1]);
 #pragma unroll
                 for (int j = 0; j < NT; ++j) {
@@ -212,12 +225,16 @@ __device__ __forceinline__ void stage_compute(const uint8_t *tile, const uint2 *
                     const float *T0 = tab + (size_t)(n0 * gpt + gi) * kTabFloats;
                     const float *T1 = T0 + gpt * kTabFloats;
                     const float X0 = T0[0], X1 = T1[0];
-                    y[j][0] += sz0.x * (acc[j][0] - T0[oa] - sz0.y * X0);
-                    y[j][1] += sz0.x * (acc[j][1] - T1[oa] - sz0.y * X1);
-                    y[j][2] += sz1.x * (acc[j][2] - T0[oa + 1] - sz1.y * X0);
-                    y[j][3] += sz1.x * (acc[j][3] - T1[oa + 1] - sz1.y * X1);
+                    const float2 O0 = *reinterpret_cast<const float2 *>(T0 + 2 * BITS);
+                    const float2 O1 = *reinterpret_cast<const float2 *>(T1 + 2 * BITS);
+                    y[j][0] += sz0.x * (acc[0][j][0] + acc[1][j][0] - O0.x - sz0.y * X0);
+                    y[j][1] += sz0.x * (acc[0][j][1] + acc[1][j][1] - O1.x - sz0.y * X1);
+                    y[j][2] += sz1.x * (acc[0][j][2] + acc[1][j][2] - O0.y - sz1.y * X0);
+                    y[j][3] += sz1.x * (acc[0][j][3] + acc[1][j][3] - O1.y - sz1.y * X1);
 #pragma unroll
-                    for (int c = 0; c < 4; ++c) acc[j][c] = 0.f;
+                    for (int a = 0; a < 2; ++a)
+#pragma unroll
+                        for (int c = 0; c < 4; ++c) acc[a][j][c] = 0.f;
                 }
             }
         }
@@ -225,7 +242,7 @@ __device__ __forceinline__ void stage_compute(const uint8_t *tile, const uint2 *
 }
 
 template <int NT>
-__device__ __forceinline__ void stage_dispatch(int bits, const uint8_t *tile, const uint2 *frag, const float *tab,
+__device__ __forceinline__ void stage_dispatch(int bits, const uint8_t *tile, const uint4 *frag, const float *tab,
                                                int group, int lane, float (&y)[2][4])
 {
     if (bits == 1) stage_compute<NT, 1>(tile, frag, tab, group, lane, y);
@@ -262,6 +279,64 @@ __device__ __forceinline__ Item decode_item(const ExpertParams &p, int item, int
         it.kt0 = it.ks * it.nkt;
     }
     return it;
+}
+
+// All consumer warps meet at the CTA's consumer barrier; false once the CTA
+// aborted (bounded like every other wait).
+__device__ __forceinline__ bool consumer_sync(const ExpertParams &p, RingShared *sh, int lane, int &uses)
+{
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sh->cbar);
+    return wait_or_abort(&sh->cbar, (uses++) & 1, p, sh);
+}
+
+// End of an item.  W13: h = silu(W1 x) * (W3 x) for the item's 128 rows, written
+// in W2's fragment order with its tables.  W2: fp32 outputs of the split.
+template <bool W13>
+__device__ __forceinline__ void epilogue(const ExpertParams &p, const Item &J, const float (&y)[2][4], int x, int tl,
+                                         int lane, int warp, float *xbuf, __half *hs, RingShared *sh, int &cbar_uses)
+{
+    const int NT = J.ci.nv > 8 ? 2 : 1;
+    const int g8 = lane >> 2, t2 = 2 * (lane & 3);
+    if (W13) {
+        if (x == 1) {
+            float4 *d = reinterpret_cast<float4 *>(xbuf + (tl * 32 + lane) * 8);
+            d[0] = make_float4(y[0][0], y[0][1], y[0][2], y[0][3]);
+            d[1] = make_float4(y[1][0], y[1][1], y[1][2], y[1][3]);
+        }
+        if (!consumer_sync(p, sh, lane, cbar_uses)) return;
+        if (x == 0) {
+            const float4 *u4 = reinterpret_cast<const float4 *>(xbuf + (tl * 32 + lane) * 8);
+            const float4 ua = u4[0], ub = u4[1];
+            const float u[2][4] = {{ua.x, ua.y, ua.z, ua.w}, {ub.x, ub.y, ub.z, ub.w}};
+#pragma unroll
+            for (int j = 0; j < 2; ++j)
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    const int n = 8 * j + t2 + (c & 1);
+                    const int r = tl * 16 + g8 + 8 * (c >> 1);
+                    const float hv = (j < NT && n < J.ci.nv) ? silu(y[j][c]) * u[j][c] : 0.f;
+                    hs[n * kTileK + r] = __float2half_rn(hv);
+                }
+        }
+        if (!consumer_sync(p, sh, lane, cbar_uses)) return;
+        const int tabf = tab_bytes(p.group) / 4;
+        const size_t vt = (size_t)J.k * (p.F / kTileK) + J.u;  // W2 column tile = this row block
+        write_frags(hs, NT, p.hfrag + vt * kFragBytes, threadIdx.x, kCW * 32);
+        write_tables(hs, 8 * NT, p.group, p.htab + vt * tabf, warp, kCW, lane);
+    } else {
+        if (x == 1 && J.blkB < 0) return;
+        const int blk = x ? J.blkB : J.blkA;
+        float *out = p.opart + (size_t)J.ks * p.Pmax * p.H;
+#pragma unroll
+        for (int j = 0; j < 2; ++j)
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                const int n = 8 * j + t2 + (c & 1);
+                const int r = blk * kBlockRows + tl * 16 + g8 + 8 * (c >> 1);
+                if (j < NT && n < J.ci.nv) out[(size_t)(J.ci.pair_base + n) * p.H + r] = y[j][c];
+            }
+    }
 }
 
 template <bool W13>
@@ -350,65 +425,17 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
     } else {
         // --------------------------------------------------------- consumers --
         const int x = warp >> 3, tl = warp & 7;
-        const int ctid = threadIdx.x;
-        const int g8 = lane >> 2, t2 = 2 * (lane & 3);
         float y[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-        int cur = -1;
+        int cur = -1, cbar_uses = 0;
         Item I;
         I.k = 0;
-        int cbar_uses = 0;
-        // all consumer warps meet; gives up (false) once the CTA aborted
-        auto consumer_sync = [&]() -> bool {
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&sh->cbar);
-            return wait_or_abort(&sh->cbar, (cbar_uses++) & 1, p, sh);
-        };
-        auto epilogue = [&](const Item &J) {
-            const int NT = J.ci.nv > 8 ? 2 : 1;
-            if (W13) {
-                if (x == 1) {
-                    float4 *d = reinterpret_cast<float4 *>(xbuf + (tl * 32 + lane) * 8);
-                    d[0] = make_float4(y[0][0], y[0][1], y[0][2], y[0][3]);
-                    d[1] = make_float4(y[1][0], y[1][1], y[1][2], y[1][3]);
-                }
-                if (!consumer_sync()) return;
-                if (x == 0) {
-                    const float *u = xbuf + (tl * 32 + lane) * 8;
-#pragma unroll
-                    for (int j = 0; j < 2; ++j)
-#pragma unroll
-                        for (int c = 0; c < 4; ++c) {
-                            const int n = 8 * j + t2 + (c & 1);
-                            const int r = tl * 16 + g8 + 8 * (c >> 1);
-                            const float hv = (j < NT && n < J.ci.nv) ? silu(y[j][c]) * u[4 * j + c] : 0.f;
-                            hs[n * kTileK + r] = __float2half_rn(hv);
-                        }
-                }
-                if (!consumer_sync()) return;
-                const size_t vt = (size_t)J.k * (p.F / kTileK) + J.u;  // W2 column tile = this row block
-                write_frags(hs, NT, p.hfrag + vt * kFragBytes, ctid, kCW * 32);
-                write_tables(hs, 8 * NT, group, p.htab + vt * tabf, warp, kCW, lane);
-            } else {
-                if (x == 1 && J.blkB < 0) return;
-                const int blk = x ? J.blkB : J.blkA;
-                float *out = p.opart + (size_t)J.ks * p.Pmax * p.H;
-#pragma unroll
-                for (int j = 0; j < 2; ++j)
-#pragma unroll
-                    for (int c = 0; c < 4; ++c) {
-                        const int n = 8 * j + t2 + (c & 1);
-                        const int r = blk * kBlockRows + tl * 16 + g8 + 8 * (c >> 1);
-                        if (j < NT && n < J.ci.nv) out[(size_t)(J.ci.pair_base + n) * p.H + r] = y[j][c];
-                    }
-            }
-        };
         for (int it = 0;; ++it) {
             const int slot = it % S;
             if (!wait_or_abort(&full[slot], (it / S) & 1, p, sh)) break;
             const int item = sh->slot_item[slot];
             if (item < 0) break;
             if (item != cur) {
-                if (cur >= 0) epilogue(I);
+                if (cur >= 0) epilogue<W13>(p, I, y, x, tl, lane, warp, xbuf, hs, sh, cbar_uses);
                 cur = item;
                 I = decode_item<W13>(p, item, U);
 #pragma unroll
@@ -420,7 +447,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
             if (!(x == 1 && I.blkB < 0)) {
                 const int TB = tile_bytes(I.ci.bits, group);
                 const uint8_t *tile = base + x * stmax + tl * TB;
-                const uint2 *frag = reinterpret_cast<const uint2 *>(base + 2 * stmax);
+                const uint4 *frag = reinterpret_cast<const uint4 *>(base + 2 * stmax);
                 const float *tab = reinterpret_cast<const float *>(base + 2 * stmax + kFragBytes);
                 if (I.ci.nv > 8) stage_dispatch<2>(I.ci.bits, tile, frag, tab, group, lane, y);
                 else stage_dispatch<1>(I.ci.bits, tile, frag, tab, group, lane, y);
@@ -428,7 +455,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
             __syncwarp();
             if (lane == 0) mbar_arrive(&empty[slot]);
         }
-        if (cur >= 0 && !sh->abort) epilogue(I);
+        if (cur >= 0 && !sh->abort) epilogue<W13>(p, I, y, x, tl, lane, warp, xbuf, hs, sh, cbar_uses);
     }
     __syncthreads();
     // On an abort, let copies that were issued but never consumed land before the
