@@ -170,6 +170,13 @@ int mc_set_path(int path);
  * device wait (default 1 s).  Process-wide. */
 int mc_set_debug(int flags, unsigned long long timeout_ns);
 
+/* Self-test of the tensor-core (tcgen05) building blocks used by the expert
+ * kernels: D = A * B^T for one 128-row tile, A fp16 [128, K], B fp16 [N, K]
+ * (row-major, 16-byte aligned), D fp32 [128, N]; 16 <= N <= 256 (multiple of 16),
+ * 64 <= K <= 256 (multiple of 64).  A bounded wait records MC_ERR_TIMEOUT in
+ * *status (device int32, may be NULL).  For the test suite; not on the layer path. */
+int mc_selftest_umma(const void *A, const void *B, float *D, int N, int K, int32_t *status, void *stream);
+
 /* Synchronise `stream`, read the status word at the start of `workspace`, clear
  * it, and return MC_OK or the recorded MC_ERR_* code. */
 int mc_check_status(void *workspace, void *stream);

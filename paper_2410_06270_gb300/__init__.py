@@ -67,6 +67,7 @@ def load():
         "mc_check_status": (I, [P, P]),
         "mc_rmsnorm": (I, [P, P, I, I, F32, P, P]),
         "mc_add": (I, [P, P, Z, P, P]),
+        "mc_selftest_umma": (I, [P, P, P, I, I, P, P]),
         "mc_profile_enable": (I, [I]),
         "mc_profile_read": (I, [P, P, I]),
         "mc_profile_name": (ctypes.c_char_p, [I]),
@@ -303,3 +304,11 @@ def profile_read() -> dict:
     _check(load().mc_profile_read(ms.ctypes.data, cnt.ctypes.data, N_KERNELS))
     lib = load()
     return {lib.mc_profile_name(i).decode(): (float(ms[i]), int(cnt[i])) for i in range(N_KERNELS) if cnt[i]}
+
+
+def selftest_umma(A, B, status=None):
+    """D = A @ B.T through the tcgen05 path (A fp16 [128, K], B fp16 [N, K])."""
+    import torch
+    D = torch.empty((A.shape[0], B.shape[0]), dtype=torch.float32, device=A.device)
+    _check(load().mc_selftest_umma(_ptr(A), _ptr(B), _ptr(D), B.shape[0], A.shape[1], _ptr(status), _stream()))
+    return D
