@@ -185,7 +185,7 @@ int mc_check_status(void *workspace, void *stream);
  * the launching stream (for benchmarks; off by default).  mc_profile_read
  * synchronises on the recorded events, writes the summed milliseconds and launch
  * counts of kernel ids 0 .. n-1 (names from mc_profile_name: route, permute,
- * gemv_w13, gemv_w2, combine, gemm_gather, gemm_w13, gemm_w2, rmsnorm) and
+ * gemv_w13, gemv_w2, combine, gemm_gather, gemm_w13, gemm_w2, rmsnorm, glu) and
  * clears the records.  Not for use inside CUDA graph capture. */
 int mc_profile_enable(int on);
 int mc_profile_read(double *ms_out, int *count_out, int n);

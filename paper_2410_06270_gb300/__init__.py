@@ -290,7 +290,7 @@ def add(a, b, out=None):
 
 # -------------------------------------------------------------- profiling --
 
-N_KERNELS = 9
+N_KERNELS = 10
 
 
 def profile_enable(on: bool = True) -> bool:

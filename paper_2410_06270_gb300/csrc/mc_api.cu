@@ -47,6 +47,7 @@ struct Workspace {
     float *xtab;
     uint8_t *hfrag;
     float *htab;
+    float *gu;
     float *opart;
     int max_chunks, KS;
     size_t total;
@@ -80,6 +81,7 @@ static Workspace carve(const mc_shape *s, int T, void *base)
     w.xtab = (float *)take(MC * (s->H / kTileK) * tb);
     w.hfrag = (uint8_t *)take(MC * (s->F / kTileK) * kFragBytes);
     w.htab = (float *)take(MC * (s->F / kTileK) * tb);
+    w.gu = (float *)take(MC * 2 * (size_t)s->F * kChunk * 4);
     w.opart = (float *)take((size_t)w.KS * P * s->H * 4);
     w.total = off;
     return w;
@@ -231,6 +233,7 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     ep.xtab = ws.xtab;
     ep.hfrag = ws.hfrag;
     ep.htab = ws.htab;
+    ep.gu = ws.gu;
     ep.opart = ws.opart;
     ep.KS = ws.KS;
     ep.Pmax = 2 * T;
@@ -238,7 +241,7 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     ep.status = ws.status;
     ep.timeout_ns = g_timeout_ns;
     ep.debug = g_debug;
-    rc = launch_gemv(ep, st);
+    rc = g_path == 1 ? launch_gemv(ep, st) : launch_tc(ep, st);
     if (rc) return rc;
 
     CombineParams cp;

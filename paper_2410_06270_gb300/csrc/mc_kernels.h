@@ -69,6 +69,7 @@ struct ExpertParams {
     float *xtab;             // [max_chunks][H/128] tab_bytes
     uint8_t *hfrag;          // [max_chunks][F/128] kFragBytes
     float *htab;             // [max_chunks][F/128] tab_bytes
+    float *gu;               // [max_chunks][2][F][16] W1 / W3 results (tensor-core path)
     float *opart;            // [KS, Pmax, H]  expert outputs (fp32), pair order
     int KS;                  // column splits of the W2 pass
     int Pmax;                // 2 * T
@@ -91,7 +92,8 @@ struct CombineParams {
 
 // Host launchers: MC_OK or an MC_ERR_* code with the message set.
 int launch_route(const RouteParams &rp, const PermuteParams &pp, cudaStream_t st);
-int launch_gemv(ExpertParams ep, cudaStream_t st);
+int launch_gemv(ExpertParams ep, cudaStream_t st);   // mma.sync path
+int launch_tc(ExpertParams ep, cudaStream_t st);     // tcgen05 path
 int launch_combine(const CombineParams &cp, cudaStream_t st);
 int max_chunks_for(int T, int E);
 

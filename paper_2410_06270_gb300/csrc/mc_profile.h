@@ -15,6 +15,7 @@ enum KernelId {
     kKGemmW13,
     kKGemmW2,
     kKRmsnorm,
+    kKGlu,
     kKCount
 };
 
