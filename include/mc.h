@@ -159,8 +159,8 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
                    int32_t *topk_idx_out, float *topk_w_out, uint8_t *pruned_out,
                    void *stream);
 
-/* Choose the expert path of mc_moe_forward: 0 = automatic (GEMV for small T,
- * tensor-core GEMM otherwise), 1 = force the GEMV path, 2 = force the GEMM path.
+/* Choose the expert path of mc_moe_forward: 0 = automatic, 1 = the mma.sync
+ * grouped GEMV (small batches), 2 = the tcgen05 tensor-memory kernels.
  * Process-wide; returns the previous value. */
 int mc_set_path(int path);
 
@@ -173,9 +173,16 @@ int mc_set_debug(int flags, unsigned long long timeout_ns);
 /* Self-test of the tensor-core (tcgen05) building blocks used by the expert
  * kernels: D = A * B^T for one 128-row tile, A fp16 [128, K], B fp16 [N, K]
  * (row-major, 16-byte aligned), D fp32 [128, N]; 16 <= N <= 256 (multiple of 16),
- * 64 <= K <= 256 (multiple of 64).  A bounded wait records MC_ERR_TIMEOUT in
+ * 64 <= K <= 256 (multiple of 64).  A negative N selects the variant with A held
+ * in tensor memory (|N| <= 128).  A bounded wait records MC_ERR_TIMEOUT in
  * *status (device int32, may be NULL).  For the test suite; not on the layer path. */
 int mc_selftest_umma(const void *A, const void *B, float *D, int N, int K, int32_t *status, void *stream);
+
+/* Profiling hook: while set, CTA 0 of every expert-kernel launch writes a
+ * globaltimer timeline of its first `steps` pipeline steps into trace_dev
+ * (device uint64 [7][steps]; row 0 = producer issue, row 1/2 = consumer
+ * start/end of the step).  NULL turns it off.  Process-wide. */
+int mc_set_trace(unsigned long long *trace_dev, int steps);
 
 /* Synchronise `stream`, read the status word at the start of `workspace`, clear
  * it, and return MC_OK or the recorded MC_ERR_* code. */

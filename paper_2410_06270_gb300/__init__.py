@@ -68,6 +68,7 @@ def load():
         "mc_rmsnorm": (I, [P, P, I, I, F32, P, P]),
         "mc_add": (I, [P, P, Z, P, P]),
         "mc_selftest_umma": (I, [P, P, P, I, I, P, P]),
+        "mc_set_trace": (I, [P, I]),
         "mc_profile_enable": (I, [I]),
         "mc_profile_read": (I, [P, P, I]),
         "mc_profile_name": (ctypes.c_char_p, [I]),
@@ -306,9 +307,16 @@ def profile_read() -> dict:
     return {lib.mc_profile_name(i).decode(): (float(ms[i]), int(cnt[i])) for i in range(N_KERNELS) if cnt[i]}
 
 
-def selftest_umma(A, B, status=None):
-    """D = A @ B.T through the tcgen05 path (A fp16 [128, K], B fp16 [N, K])."""
+def selftest_umma(A, B, status=None, a_in_tmem=False):
+    """D = A @ B.T through the tcgen05 path (A fp16 [128, K], B fp16 [N, K]);
+    a_in_tmem: the A operand is staged in tensor memory instead of shared memory."""
     import torch
     D = torch.empty((A.shape[0], B.shape[0]), dtype=torch.float32, device=A.device)
-    _check(load().mc_selftest_umma(_ptr(A), _ptr(B), _ptr(D), B.shape[0], A.shape[1], _ptr(status), _stream()))
+    n = -B.shape[0] if a_in_tmem else B.shape[0]
+    _check(load().mc_selftest_umma(_ptr(A), _ptr(B), _ptr(D), n, A.shape[1], _ptr(status), _stream()))
     return D
+
+
+def set_trace(buf=None, steps=0):
+    """Record CTA 0's per-step pipeline timeline into buf (int64 [7, steps] on the device)."""
+    load().mc_set_trace(_ptr(buf), int(steps))

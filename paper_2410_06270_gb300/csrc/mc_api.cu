@@ -16,6 +16,8 @@ namespace mc {
 static std::atomic<int> g_path{0};
 static std::atomic<int> g_debug{0};
 static std::atomic<unsigned long long> g_timeout_ns{1000000000ull};  // 1 s
+static uint64_t *g_trace = nullptr;
+static int g_trace_steps = 0;
 
 #define MC_CUDA(call)                                                                         \
     do {                                                                                      \
@@ -118,6 +120,15 @@ int mc_set_debug(int flags, unsigned long long timeout_ns)
 {
     g_debug = flags;
     if (timeout_ns) g_timeout_ns = timeout_ns;
+    return MC_OK;
+}
+
+// Profiling hook: record the per-step event timeline of CTA 0 of the next expert
+// kernel launches into trace_dev (device uint64 [7][steps]); NULL turns it off.
+int mc_set_trace(unsigned long long *trace_dev, int steps)
+{
+    g_trace = (uint64_t *)trace_dev;
+    g_trace_steps = trace_dev ? steps : 0;
     return MC_OK;
 }
 
@@ -241,7 +252,10 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     ep.status = ws.status;
     ep.timeout_ns = g_timeout_ns;
     ep.debug = g_debug;
-    rc = g_path == 1 ? launch_gemv(ep, st) : launch_tc(ep, st);
+    ep.trace = g_trace;
+    ep.trace_steps = g_trace_steps;
+    // decode-sized work: mma.sync GEMV; path 2 forces the tcgen05 kernels
+    rc = g_path == 2 ? launch_tc(ep, st) : launch_gemv(ep, st);
     if (rc) return rc;
 
     CombineParams cp;

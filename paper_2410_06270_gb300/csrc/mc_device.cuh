@@ -173,6 +173,18 @@ __device__ __forceinline__ void cvt1_half(uint32_t w, int p0, uint32_t (&r)[8])
     }
 }
 
+// 1-bit plane word, all 16 positions -> 16 registers.
+template <bool HI4>
+__device__ __forceinline__ void cvt1(uint32_t w, uint32_t (&r)[16])
+{
+    constexpr int b = HI4 ? 27 : 25;
+    const uint32_t v = w >> 10;
+#pragma unroll
+    for (int p = 0; p < 10; ++p) r[p] = lop_and_or(w, 0x00010001u << p, MC_C(b - p));
+#pragma unroll
+    for (int p = 0; p < 6; ++p) r[10 + p] = lop_and_or(v, 0x00010001u << p, MC_C(b - p));
+}
+
 __device__ __forceinline__ float silu(float g) { return g / (1.0f + __expf(-g)); }
 
 }  // namespace mc

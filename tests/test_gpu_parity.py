@@ -260,3 +260,13 @@ def test_rmsnorm_and_add(mc):
         assert rel < 4e-3 and mx < 8e-3
     s = mc.add(x, x).float().cpu().numpy()
     np.testing.assert_array_equal(s, 2 * synth.bf16_bits_to_f32(xs))
+
+
+@pytest.mark.parametrize("path", [1, 2])
+@pytest.mark.parametrize("group", [64, 128])
+def test_forward_both_expert_paths(mc, path, group):
+    """The mma.sync GEMV kernels (path 1) and the tcgen05 tensor-memory kernels
+    (path 2) against the oracle on the same layer."""
+    L = synth.make_layer(20, 384, 512, 8, group, [3, 2, 1, 3, 2, 2, 1, 3], 95 + group, gate_std=0.1, mu=0.4,
+                         protect_frac=0.2, zero_mode="fractional")
+    _forward_and_check(mc, L, path=path)

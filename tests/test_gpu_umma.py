@@ -16,13 +16,14 @@ def mc():
     return m
 
 
+@pytest.mark.parametrize("a_in_tmem", [False, True])
 @pytest.mark.parametrize("N,K", [(16, 64), (16, 128), (32, 256), (64, 128), (128, 64)])
-def test_umma_tile_matches_matmul(mc, N, K):
+def test_umma_tile_matches_matmul(mc, N, K, a_in_tmem):
     g = torch.Generator().manual_seed(N * 1000 + K)
     A = torch.randn(128, K, generator=g).half().cuda()
     B = torch.randn(N, K, generator=g).half().cuda()
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
-    D = mc.selftest_umma(A, B, st)
+    D = mc.selftest_umma(A, B, st, a_in_tmem=a_in_tmem)
     torch.cuda.synchronize()
     assert int(st.item()) == 0
     ref = A.double() @ B.double().T
@@ -30,11 +31,12 @@ def test_umma_tile_matches_matmul(mc, N, K):
     assert err < 1e-5, err
 
 
-def test_umma_integer_operands_exact(mc):
+@pytest.mark.parametrize("a_in_tmem", [False, True])
+def test_umma_integer_operands_exact(mc, a_in_tmem):
     """Small integers are exact in fp16 and fp32: the product must be exact."""
     g = torch.Generator().manual_seed(7)
     A = torch.randint(0, 8, (128, 128), generator=g).half().cuda()
     B = torch.randint(-4, 5, (16, 128), generator=g).half().cuda()
-    D = mc.selftest_umma(A, B)
+    D = mc.selftest_umma(A, B, a_in_tmem=a_in_tmem)
     torch.cuda.synchronize()
     assert torch.equal(D.cpu(), (A.float() @ B.float().T).cpu())
