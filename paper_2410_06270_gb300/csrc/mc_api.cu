@@ -50,6 +50,7 @@ struct Workspace {
     uint8_t *hfrag;
     float *htab;
     float *gu;
+    uint8_t *xvec, *hvec;
     float *opart;
     int max_chunks, KS;
     size_t total;
@@ -84,6 +85,8 @@ static Workspace carve(const mc_shape *s, int T, void *base)
     w.hfrag = (uint8_t *)take(MC * (s->F / kTileK) * kFragBytes);
     w.htab = (float *)take(MC * (s->F / kTileK) * tb);
     w.gu = (float *)take(MC * 2 * (size_t)s->F * kChunk * 4);
+    w.xvec = (uint8_t *)take(MC * 2 * (s->H / kTileK) * (size_t)vec_bytes(s->group));
+    w.hvec = (uint8_t *)take(MC * 2 * (s->F / kTileK) * (size_t)vec_bytes(s->group));
     w.opart = (float *)take((size_t)w.KS * P * s->H * 4);
     w.total = off;
     return w;
@@ -245,6 +248,8 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     ep.hfrag = ws.hfrag;
     ep.htab = ws.htab;
     ep.gu = ws.gu;
+    ep.xvec = ws.xvec;
+    ep.hvec = ws.hvec;
     ep.opart = ws.opart;
     ep.KS = ws.KS;
     ep.Pmax = 2 * T;

@@ -3,56 +3,60 @@
 //
 // frag_x_kernel: gathers the routed tokens' activations per work chunk (<= 16
 //   pairs of one expert) into mma B-fragment order, fp16, with the per-group
-//   offset tables, one 128-column tile at a time.
+//   offset tables: one "vector block" per (chunk, n-tile, 128-column step).
 // gemv_kernel<W13>: persistent, one CTA per SM.  A producer warp claims work
-//   items from an atomic counter (chunks of experts with more bits first) and
-//   streams, for every 128-column step of an item, one ring stage holding
-//     [row stream A supertile][row stream B supertile][B fragments][tables]
-//   with cp.async.bulk (mbarrier transaction counts, L2 evict-first for the
-//   weights), never pausing between items.  Sixteen consumer warps each own one
-//   16-row tile of one stream: its code words become fp16 mma.sync A fragments
-//   with one LOP3 per register (mc_layout.h), and every quantisation group is
-//   folded as
+//   items (a chunk x a 128-row block of W1|W3, or a chunk x a 256-row block pair
+//   of W2 over one column split) from an atomic counter, experts with more bits
+//   first, and streams each item as ring stages of kKPS 128-column steps:
+//     [weights of both row streams, kKPS steps]   one cp.async.bulk copy
+//     [vector blocks of n-tile 0][of n-tile 1]      one copy each
+//   The packed layout interleaves the two streams step by step (mc_layout.h), so
+//   a stage is a few large copies: small copies cap the streaming bandwidth well
+//   below the HBM peak.  Eight consumer warps each own one 16-row tile of BOTH
+//   streams (the B fragments and tables are loaded once for the two).  Code
+//   words become fp16 mma.sync A fragments with one LOP3 per register
+//   (mc_layout.h), and every quantisation group is folded as
 //       y += s * (acc - O - z * X)
 //   where acc = sum_k (off_k + q_k) x_k, O = sum_k off_k x_k, X = sum_k x_k, i.e.
 //   y += s * sum_k (q_k - z) x_k, the group-wise dequantised product.
-//   W13: streams = W1 and W3 rows of a 128-row block; the epilogue forms
-//        h = silu(W1 x) * (W3 x) and writes it straight into W2's fragment order
-//        with its tables.
-//   W2:  streams = two 128-row blocks of W2 over one column split; the epilogue
-//        writes fp32 expert outputs.
-// The decode path is bound by HBM bandwidth on the packed weight bytes.
+//   W13: streams = W1 and W3 rows of a 128-row block; each warp forms
+//        h = silu(W1 x) * (W3 x) in registers and the CTA writes W2's vector
+//        blocks.
+//   W2:  streams = two 128-row blocks of W2; the epilogue writes fp32 outputs.
+// Decoding costs one ALU instruction per two weights of a bit plane, so the
+// consumers are kept lean: this path is bound by HBM bandwidth on the packed
+// weight bytes only while the decode keeps up with it.
 #include "mc_host.h"
 #include "mc_kernels.h"
 #include "mc_profile.h"
 
 namespace mc {
 
-constexpr int kCW = 16;                     // consumer warps
+constexpr int kCW = 8;                      // consumer warps (tile tl of both streams)
 constexpr int kGemvThreads = (kCW + 1) * 32;
 constexpr int kMaxSlots = 16;
 constexpr int kRingOff = 1024;
+constexpr int kKPS = 2;                     // 128-column steps per ring stage
 
 struct RingShared {
     uint64_t cbar;  // consumer-warp barrier of the W13 epilogue (bounded waits)
     volatile int abort;
     volatile int issued;
     int slot_item[kMaxSlots];
-    int slot_i[kMaxSlots];
+    int slot_kc[kMaxSlots];  // column steps held by the stage (1..kKPS)
 };
+
+constexpr int kVecMax = kVecFragBytes + 8 * 2 * kTabFloats * 4;  // vec_bytes(64), the largest
 
 __host__ __device__ inline int slot_bytes(int group)
 {
-    return 2 * supertile_bytes(3, group) + kFragBytes + tab_bytes(group);
+    return kKPS * 2 * supertile_bytes(3, group) + 2 * kKPS * kVecMax;
 }
-
-__host__ __device__ inline size_t epi_off(int nslots, int group) { return kRingOff + (size_t)nslots * slot_bytes(group); }
-constexpr int kXbufBytes = 8 * 32 * 8 * 4;   // stream-B results handed to stream A
-constexpr int kHsBytes = kChunk * kTileK * 2;  // h tile [16][128] fp16
+constexpr int kHsBytes = kChunk * kTileK * 2;  // h tile [16][128] fp16 (two of them)
 
 __host__ __device__ inline size_t gemv_smem(int nslots, int group)
 {
-    return epi_off(nslots, group) + kXbufBytes + kHsBytes;
+    return kRingOff + (size_t)nslots * slot_bytes(group) + 2 * kHsBytes;
 }
 
 // Bounded wait that gives up as soon as another thread of the CTA aborted.
@@ -84,14 +88,29 @@ __device__ __forceinline__ bool header_ok(const ExpertParams &p, int e)
            hd->mat_off[e][2] == p.mat_off[e][2];
 }
 
-// Offset tables (mc_layout.h) of `ntok` rows of 128 fp16 columns held in shared
-// memory; one warp per (row, group) item, written to dst[(n * gpt + gi) * 8].
-__device__ __forceinline__ void write_tables(const __half *rows, int ntok, int group, float *dst, int warp, int nwarps,
-                                             int lane)
+// Vector block of n-tile j built from a [16][128] fp16 tile in shared memory:
+//   fragments, 256 entries of 8 bytes ordered [s/2][lane][s%2] (one 16-byte load
+//     gives a lane its B fragments of k-steps 2q and 2q+1); an entry holds the
+//     4 fp16 values at columns 64(s/4) + 16t + 4(s%4) .. +3 of pair 8j + lane/4;
+//   then the offset tables of pairs 8j .. 8j+7, [n][group][8 floats]:
+//     [O2 half 0, O2 half 1, X, O1 half 0, O3 half 0, O3 half 1, X, O1 half 1]
+//   (X = sum of the group's inputs, O_b = sum of the b-bit plane offsets times
+//   the inputs for the rows of one half, O3 = O2 + 4 O1; mc_layout.h), so that a
+//   2- or 3-bit fold reads its O pair and X with one 16-byte load.
+// Threads share the fragment entries; one warp per table item.
+__device__ __forceinline__ void write_vec_block(const __half *rows, int j, int group, uint8_t *dst, int tid,
+                                                int nthreads, int warp, int nwarps, int lane)
 {
+    for (int idx = tid; idx < 256; idx += nthreads) {
+        const int s = 2 * ((idx >> 6) & 3) + (idx & 1), ln = (idx >> 1) & 31;
+        const int n = 8 * j + (ln >> 2), t = ln & 3;
+        const int col = 64 * (s >> 2) + 16 * t + 4 * (s & 3);
+        reinterpret_cast<uint2 *>(dst)[idx] = *reinterpret_cast<const uint2 *>(rows + n * kTileK + col);
+    }
     const int gpt = kTileK / group;
-    for (int item = warp; item < ntok * gpt; item += nwarps) {
-        const int n = item / gpt, gi = item % gpt;
+    float *tab = reinterpret_cast<float *>(dst + kVecFragBytes);
+    for (int item = warp; item < 8 * gpt; item += nwarps) {
+        const int nl = item / gpt, gi = item % gpt, n = 8 * j + nl;
         float tb[5] = {0, 0, 0, 0, 0};
         for (int c = gi * group + lane; c < (gi + 1) * group; c += 32) {
             const float v = __half2float(rows[n * kTileK + c]);
@@ -107,23 +126,10 @@ __device__ __forceinline__ void write_tables(const __half *rows, int ntok, int g
 #pragma unroll
             for (int m = 16; m >= 1; m >>= 1) tb[k] += __shfl_xor_sync(0xffffffffu, tb[k], m);
         if (lane == 0) {
-            float4 *d = reinterpret_cast<float4 *>(dst + (size_t)item * kTabFloats);
-            d[0] = make_float4(tb[0], 0.f, tb[1], tb[2]);
-            d[1] = make_float4(tb[3], tb[4], tb[3] + 4.f * tb[1], tb[4] + 4.f * tb[2]);
+            float4 *d = reinterpret_cast<float4 *>(tab + (size_t)item * kTabFloats);
+            d[0] = make_float4(tb[3], tb[4], tb[0], tb[1]);
+            d[1] = make_float4(tb[3] + 4.f * tb[1], tb[4] + 4.f * tb[2], tb[0], tb[2]);
         }
-    }
-}
-
-// Fragment entries (j < NT) of a [16][128] fp16 tile held in shared memory,
-// 8 bytes each, ordered [j][s/2][lane][s%2] so that one 16-byte load gives a
-// lane its B fragments of k-steps 2q and 2q+1.
-__device__ __forceinline__ void write_frags(const __half *rows, int NT, uint8_t *dst, int tid, int nthreads)
-{
-    for (int idx = tid; idx < NT * 256; idx += nthreads) {
-        const int j = idx >> 8, s = 2 * ((idx >> 6) & 3) + (idx & 1), ln = (idx >> 1) & 31;
-        const int n = 8 * j + (ln >> 2), t = ln & 3;
-        const int col = 64 * (s >> 2) + 16 * t + 4 * (s & 3);
-        reinterpret_cast<uint2 *>(dst)[idx] = *reinterpret_cast<const uint2 *>(rows + n * kTileK + col);
     }
 }
 
@@ -156,105 +162,158 @@ __global__ void __launch_bounds__(256) frag_x_kernel(ExpertParams p)
         *reinterpret_cast<uint4 *>(xs + n * kTileK + c8) = out;
     }
     __syncthreads();
-    const size_t tile = (size_t)k * KT + kt;
-    write_frags(xs, NT, p.xfrag + tile * kFragBytes, tid, 256);
-    write_tables(xs, 8 * NT, p.group, p.xtab + tile * (tab_bytes(p.group) / 4), tid >> 5, 8, tid & 31);
+    for (int j = 0; j < NT; ++j)
+        write_vec_block(xs, j, p.group, p.xvec + vec_off(k, j, kt, KT, p.group), tid, 256, tid >> 5, 8, tid & 31);
 }
 
-// -------------------------------------------------------------- one stage --
-// One consumer warp, one 128-column step of its 16-row tile: decode, mma and
-// fold.  Accumulates into y[j][c] (C-fragment layout, rows g8 / g8+8, pairs
-// 8j + 2t + {0,1}).
-template <int NT, int BITS>
-__device__ __forceinline__ void stage_compute(const uint8_t *tile, const uint4 *frag, const float *tab, int group,
-                                              int lane, float (&y)[2][4])
+// --------------------------------------------------------------- one step --
+
+// D = A * B (+ C), m16n8k16, fp16 inputs, fp32 accumulate; ZERO: C = 0.
+template <bool ZERO>
+__device__ __forceinline__ void mma_acc(float (&d)[4], const uint32_t *a, uint32_t b0, uint32_t b1)
 {
-    const int gpt = kTileK / group;
+    if (ZERO)
+        asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+            "{%10,%10,%10,%10};"
+            : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+            : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(0.f));
+    else
+        asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+            "{%0,%1,%2,%3};"
+            : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+            : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// The code words and fp16 (scale, zero) pairs one lane needs from a tile.
+template <int BITS, int GPT>
+struct TileRegs {
     uint32_t c2[4], c1[2];
+    uint2 meta[GPT];
+};
+
+template <int BITS, int GPT>
+__device__ __forceinline__ void load_tile(const uint8_t *tile, int lane, TileRegs<BITS, GPT> &t)
+{
     if (BITS >= 2) {
         const uint4 v = *reinterpret_cast<const uint4 *>(tile + 16 * lane);
-        c2[0] = v.x; c2[1] = v.y; c2[2] = v.z; c2[3] = v.w;
+        t.c2[0] = v.x; t.c2[1] = v.y; t.c2[2] = v.z; t.c2[3] = v.w;
     }
     if (BITS != 2) {
         const uint2 v = *reinterpret_cast<const uint2 *>(tile + (BITS == 3 ? 512 : 0) + 8 * lane);
-        c1[0] = v.x; c1[1] = v.y;
+        t.c1[0] = v.x; t.c1[1] = v.y;
     }
     const uint8_t *mt = tile + tile_code_bytes(BITS);
-    uint2 meta[2];
-    meta[0] = *reinterpret_cast<const uint2 *>(mt + (lane >> 2) * 8);
-    meta[1] = gpt == 2 ? *reinterpret_cast<const uint2 *>(mt + 64 + (lane >> 2) * 8) : meta[0];
-    // two independent accumulators halve the dependent mma chain: 1/2-bit by
-    // k-step parity, 3-bit low plane / high plane
-    float acc[2][NT][4];
 #pragma unroll
-    for (int a = 0; a < 2; ++a)
-#pragma unroll
-        for (int j = 0; j < NT; ++j)
-#pragma unroll
-            for (int c = 0; c < 4; ++c) acc[a][j][c] = 0.f;
+    for (int g = 0; g < GPT; ++g) t.meta[g] = *reinterpret_cast<const uint2 *>(mt + 64 * g + (lane >> 2) * 8);
+}
+
+// A-fragment registers of k-steps 2qd, 2qd+1: r (low / only plane), rh (3-bit
+// high plane, weighted x4 through its exponent).
+template <int BITS, int GPT>
+__device__ __forceinline__ void decode_qd(const TileRegs<BITS, GPT> &t, int qd, uint32_t (&r)[8], uint32_t (&rh)[8])
+{
+    if (BITS == 1) cvt1_half<false>(t.c1[qd >> 1], 8 * (qd & 1), r);
+    if (BITS >= 2) cvt2(t.c2[qd], r);
+    if (BITS == 3) cvt1_half<true>(t.c1[qd >> 1], 8 * (qd & 1), rh);
+}
+
+// y += s * (acc0 + acc1 - O - z X) for the lane's four C-fragment entries:
+// entries 0/1 are row g8 with pairs 2t / 2t+1, entries 2/3 row g8+8.
+__device__ __forceinline__ void fold(float (&y)[4], const float (&a0)[4], const float (&a1)[4], uint2 meta,
+                                     float2 O0, float2 O1, float X0, float X1)
+{
+    const __half2 *m2 = reinterpret_cast<const __half2 *>(&meta);
+    const float2 sz0 = __half22float2(m2[0]), sz1 = __half22float2(m2[1]);
+    y[0] = fmaf(sz0.x, a0[0] + a1[0] - O0.x - sz0.y * X0, y[0]);
+    y[1] = fmaf(sz0.x, a0[1] + a1[1] - O1.x - sz0.y * X1, y[1]);
+    y[2] = fmaf(sz1.x, a0[2] + a1[2] - O0.y - sz1.y * X0, y[2]);
+    y[3] = fmaf(sz1.x, a0[3] + a1[3] - O1.y - sz1.y * X1, y[3]);
+}
+
+// One consumer warp, one 128-column step of its 16-row tile in both streams:
+// decode, mma and fold.  y*[j][c]: C-fragment layout, rows g8 / g8+8 of the
+// tile, pairs 8j + 2t + {0,1}.  vec0 / vec1: the step's vector blocks of
+// n-tiles 0 / 1.  Two accumulators per tile and n-tile keep the dependent mma
+// chains short: 1/2-bit by k-step parity, 3-bit low plane / high plane.
+template <int NT, int BITS, int GPT>
+__device__ __forceinline__ void step2(const uint8_t *tA, const uint8_t *tB, const uint8_t *vec0, const uint8_t *vec1,
+                                      int lane, float (&yA)[NT][4], float (&yB)[NT][4])
+{
+    constexpr int SPG = 8 / GPT;  // k-steps per quantisation group
+    TileRegs<BITS, GPT> RA, RB;
+    load_tile<BITS, GPT>(tA, lane, RA);
+    load_tile<BITS, GPT>(tB, lane, RB);
+    float accA[2][NT][4], accB[2][NT][4];
 #pragma unroll
     for (int qd = 0; qd < 4; ++qd) {
-        uint32_t r[8], rh[8];
-        if (BITS == 1) cvt1_half<false>(c1[qd >> 1], 8 * (qd & 1), r);
-        if (BITS >= 2) cvt2(c2[qd], r);
-        if (BITS == 3) cvt1_half<true>(c1[qd >> 1], 8 * (qd & 1), rh);
+        uint32_t ra[8], rha[8], rb[8], rhb[8];
+        decode_qd<BITS, GPT>(RA, qd, ra, rha);
+        decode_qd<BITS, GPT>(RB, qd, rb, rhb);
         uint4 bq[NT];
 #pragma unroll
-        for (int j = 0; j < NT; ++j) bq[j] = frag[(j * 4 + qd) * 32 + lane];
+        for (int j = 0; j < NT; ++j) bq[j] = reinterpret_cast<const uint4 *>(j ? vec1 : vec0)[qd * 32 + lane];
 #pragma unroll
         for (int kk = 0; kk < 2; ++kk) {
             const int s = 2 * qd + kk;
+            // the first k-step of a group (of each parity chain) starts from zero
+            const bool first = BITS == 3 ? (s % SPG == 0) : (s % SPG < 2);
 #pragma unroll
             for (int j = 0; j < NT; ++j) {
                 const uint32_t b0 = kk ? bq[j].z : bq[j].x, b1 = kk ? bq[j].w : bq[j].y;
-                if (BITS == 3) {
-                    mma16816(acc[0][j], r[4 * kk], r[4 * kk + 1], r[4 * kk + 2], r[4 * kk + 3], b0, b1);
-                    mma16816(acc[1][j], rh[4 * kk], rh[4 * kk + 1], rh[4 * kk + 2], rh[4 * kk + 3], b0, b1);
+                const int ca = BITS == 3 ? 0 : kk;
+                if (first) {
+                    mma_acc<true>(accA[ca][j], ra + 4 * kk, b0, b1);
+                    mma_acc<true>(accB[ca][j], rb + 4 * kk, b0, b1);
+                    if (BITS == 3) {
+                        mma_acc<true>(accA[1][j], rha + 4 * kk, b0, b1);
+                        mma_acc<true>(accB[1][j], rhb + 4 * kk, b0, b1);
+                    }
                 } else {
-                    mma16816(acc[kk][j], r[4 * kk], r[4 * kk + 1], r[4 * kk + 2], r[4 * kk + 3], b0, b1);
+                    mma_acc<false>(accA[ca][j], ra + 4 * kk, b0, b1);
+                    mma_acc<false>(accB[ca][j], rb + 4 * kk, b0, b1);
+                    if (BITS == 3) {
+                        mma_acc<false>(accA[1][j], rha + 4 * kk, b0, b1);
+                        mma_acc<false>(accB[1][j], rhb + 4 * kk, b0, b1);
+                    }
                 }
             }
-            if ((s == 3 && gpt == 2) || s == 7) {
-                const int gi = s == 3 ? 0 : gpt - 1;
-                const uint2 mg = gi == 0 ? meta[0] : meta[1];  // no dynamic index: keeps meta in registers
-                const __half2 *m2 = reinterpret_cast<const __half2 *>(&mg);
-                const float2 sz0 = __half22float2(m2[0]), sz1 = __half22float2(m2[1]);
+            if (s % SPG == SPG - 1) {
+                const int gi = s / SPG;
 #pragma unroll
                 for (int j = 0; j < NT; ++j) {
-                    const int n0 = 8 * j + 2 * (lane & 3);
-                    const float *T0 = tab + (size_t)(n0 * gpt + gi) * kTabFloats;
-                    const float *T1 = T0 + gpt * kTabFloats;
-                    const float X0 = T0[0], X1 = T1[0];
-                    const float2 O0 = *reinterpret_cast<const float2 *>(T0 + 2 * BITS);
-                    const float2 O1 = *reinterpret_cast<const float2 *>(T1 + 2 * BITS);
-                    y[j][0] += sz0.x * (acc[0][j][0] + acc[1][j][0] - O0.x - sz0.y * X0);
-                    y[j][1] += sz0.x * (acc[0][j][1] + acc[1][j][1] - O1.x - sz0.y * X1);
-                    y[j][2] += sz1.x * (acc[0][j][2] + acc[1][j][2] - O0.y - sz1.y * X0);
-                    y[j][3] += sz1.x * (acc[0][j][3] + acc[1][j][3] - O1.y - sz1.y * X1);
-#pragma unroll
-                    for (int a = 0; a < 2; ++a)
-#pragma unroll
-                        for (int c = 0; c < 4; ++c) acc[a][j][c] = 0.f;
+                    const float *T0 = reinterpret_cast<const float *>((j ? vec1 : vec0) + kVecFragBytes) +
+                                      (size_t)((2 * (lane & 3)) * GPT + gi) * kTabFloats;
+                    const float *T1 = T0 + GPT * kTabFloats;
+                    float2 O0, O1;
+                    float X0, X1;
+                    if (BITS == 1) {
+                        const float4 u0 = *reinterpret_cast<const float4 *>(T0);
+                        const float4 u1 = *reinterpret_cast<const float4 *>(T1);
+                        O0 = make_float2(u0.w, T0[7]);
+                        O1 = make_float2(u1.w, T1[7]);
+                        X0 = u0.z;
+                        X1 = u1.z;
+                    } else {
+                        const float4 u0 = *reinterpret_cast<const float4 *>(T0 + (BITS == 3 ? 4 : 0));
+                        const float4 u1 = *reinterpret_cast<const float4 *>(T1 + (BITS == 3 ? 4 : 0));
+                        O0 = make_float2(u0.x, u0.y);
+                        O1 = make_float2(u1.x, u1.y);
+                        X0 = u0.z;
+                        X1 = u1.z;
+                    }
+                    fold(yA[j], accA[0][j], accA[1][j], RA.meta[gi], O0, O1, X0, X1);
+                    fold(yB[j], accB[0][j], accB[1][j], RB.meta[gi], O0, O1, X0, X1);
                 }
             }
         }
     }
 }
 
-template <int NT>
-__device__ __forceinline__ void stage_dispatch(int bits, const uint8_t *tile, const uint4 *frag, const float *tab,
-                                               int group, int lane, float (&y)[2][4])
-{
-    if (bits == 1) stage_compute<NT, 1>(tile, frag, tab, group, lane, y);
-    else if (bits == 2) stage_compute<NT, 2>(tile, frag, tab, group, lane, y);
-    else stage_compute<NT, 3>(tile, frag, tab, group, lane, y);
-}
-
 struct Item {
     int k, u;          // chunk, unit
     ChunkInfo ci;
     int blkA, blkB;    // 128-row blocks of the two streams (blkB < 0: none)
-    int kt0, nkt, ks;
+    int kt0, nkt, ks;  // column steps [kt0, kt0 + nkt) of split ks
 };
 
 template <bool W13>
@@ -281,65 +340,93 @@ __device__ __forceinline__ Item decode_item(const ExpertParams &p, int item, int
     return it;
 }
 
-// All consumer warps meet at the CTA's consumer barrier; false once the CTA
-// aborted (bounded like every other wait).
-__device__ __forceinline__ bool consumer_sync(const ExpertParams &p, RingShared *sh, int lane, int &uses)
-{
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&sh->cbar);
-    return wait_or_abort(&sh->cbar, (uses++) & 1, p, sh);
-}
+// Ring geometry shared by the consumer warps.
+struct Ring {
+    uint64_t *full, *empty;
+    const uint8_t *base;
+    int S, SB, vec_off0, VB;
+};
 
-// End of an item.  W13: h = silu(W1 x) * (W3 x) for the item's 128 rows, written
-// in W2's fragment order with its tables.  W2: fp32 outputs of the split.
-template <bool W13>
-__device__ __forceinline__ void epilogue(const ExpertParams &p, const Item &J, const float (&y)[2][4], int x, int tl,
-                                         int lane, int warp, float *xbuf, __half *hs, RingShared *sh, int &cbar_uses)
+// One work item for one consumer warp (tile tl of both streams): all its
+// stages, then the epilogue.  The first stage's full barrier has already been
+// waited for; the ring position (slot, phase) advances by one per stage.
+//   W13: h = silu(W1 x) * (W3 x) for the warp's 16 rows goes to the h tile
+//        (double-buffered by item parity), the consumer warps meet once, and
+//        together write W2's vector blocks of this 128-row block.
+//   W2:  fp32 outputs of the split, rows of both blocks.
+template <bool W13, int NT, int BITS, int GPT>
+__device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, const Ring &R, const Item &I, int nrb,
+                                      int tl, int lane, int &slot, uint32_t &phase, __half *hs2, int &items)
 {
-    const int NT = J.ci.nv > 8 ? 2 : 1;
+    constexpr int group = kTileK / GPT;
+    const int STB = supertile_bytes(BITS, group), TB = tile_bytes(BITS, group);
+    const int pw = W13 ? 2 : w2_pair_width(I.blkA >> 1, nrb);
+    const int step_bytes = pw * STB;
+    const int offA = tl * TB, offB = (pw == 2 ? STB : 0) + tl * TB;  // lone W2 block: stream B repeats A
+    float yA[NT][4], yB[NT][4];
+#pragma unroll
+    for (int j = 0; j < NT; ++j)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) yA[j][c] = yB[j][c] = 0.f;
+    for (int i = 0; i < I.nkt; i += kKPS) {
+        if (i > 0 && !wait_or_abort(&R.full[slot], phase, p, sh)) return false;
+        const uint8_t *base = R.base + (size_t)slot * R.SB;
+        const int kc = sh->slot_kc[slot];
+        const uint8_t *v0 = base + R.vec_off0, *v1 = v0 + kKPS * R.VB;
+#pragma unroll
+        for (int kk = 0; kk < kKPS; ++kk)
+            if (kk < kc)
+                step2<NT, BITS, GPT>(base + kk * step_bytes + offA, base + kk * step_bytes + offB, v0 + kk * R.VB,
+                                     v1 + kk * R.VB, lane, yA, yB);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&R.empty[slot]);
+        if (++slot == R.S) {
+            slot = 0;
+            phase ^= 1u;
+        }
+    }
     const int g8 = lane >> 2, t2 = 2 * (lane & 3);
     if (W13) {
-        if (x == 1) {
-            float4 *d = reinterpret_cast<float4 *>(xbuf + (tl * 32 + lane) * 8);
-            d[0] = make_float4(y[0][0], y[0][1], y[0][2], y[0][3]);
-            d[1] = make_float4(y[1][0], y[1][1], y[1][2], y[1][3]);
-        }
-        if (!consumer_sync(p, sh, lane, cbar_uses)) return;
-        if (x == 0) {
-            const float4 *u4 = reinterpret_cast<const float4 *>(xbuf + (tl * 32 + lane) * 8);
-            const float4 ua = u4[0], ub = u4[1];
-            const float u[2][4] = {{ua.x, ua.y, ua.z, ua.w}, {ub.x, ub.y, ub.z, ub.w}};
+        __half *hs = hs2 + (items & 1) * (kChunk * kTileK);
 #pragma unroll
-            for (int j = 0; j < 2; ++j)
-#pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    const int n = 8 * j + t2 + (c & 1);
-                    const int r = tl * 16 + g8 + 8 * (c >> 1);
-                    const float hv = (j < NT && n < J.ci.nv) ? silu(y[j][c]) * u[j][c] : 0.f;
-                    hs[n * kTileK + r] = __float2half_rn(hv);
-                }
-        }
-        if (!consumer_sync(p, sh, lane, cbar_uses)) return;
-        const int tabf = tab_bytes(p.group) / 4;
-        const size_t vt = (size_t)J.k * (p.F / kTileK) + J.u;  // W2 column tile = this row block
-        write_frags(hs, NT, p.hfrag + vt * kFragBytes, threadIdx.x, kCW * 32);
-        write_tables(hs, 8 * NT, p.group, p.htab + vt * tabf, warp, kCW, lane);
-    } else {
-        if (x == 1 && J.blkB < 0) return;
-        const int blk = x ? J.blkB : J.blkA;
-        float *out = p.opart + (size_t)J.ks * p.Pmax * p.H;
-#pragma unroll
-        for (int j = 0; j < 2; ++j)
+        for (int j = 0; j < NT; ++j)
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 const int n = 8 * j + t2 + (c & 1);
-                const int r = blk * kBlockRows + tl * 16 + g8 + 8 * (c >> 1);
-                if (j < NT && n < J.ci.nv) out[(size_t)(J.ci.pair_base + n) * p.H + r] = y[j][c];
+                const int r = tl * 16 + g8 + 8 * (c >> 1);
+                const float hv = n < I.ci.nv ? silu(yA[j][c]) * yB[j][c] : 0.f;
+                hs[n * kTileK + r] = __float2half_rn(hv);
+            }
+        // every warp finished the previous item's vector blocks before it got here,
+        // so after this barrier the other h buffer is free again
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sh->cbar);
+        if (!wait_or_abort(&sh->cbar, items & 1, p, sh)) return false;
+        ++items;
+        // the item's 128 rows are W2's column step I.u
+        const int KT2 = p.F / kTileK;
+        for (int j = 0; j < NT; ++j)
+            write_vec_block(hs, j, group, p.hvec + vec_off(I.k, j, I.u, KT2, group), threadIdx.x, kCW * 32, tl,
+                            kCW, lane);
+    } else {
+        float *out = p.opart + (size_t)I.ks * p.Pmax * p.H;
+#pragma unroll
+        for (int j = 0; j < NT; ++j)
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                const int n = 8 * j + t2 + (c & 1);
+                const int r = tl * 16 + g8 + 8 * (c >> 1);
+                if (n < I.ci.nv) {
+                    float *o = out + (size_t)(I.ci.pair_base + n) * p.H;
+                    o[I.blkA * kBlockRows + r] = yA[j][c];
+                    if (I.blkB >= 0) o[I.blkB * kBlockRows + r] = yB[j][c];
+                }
             }
     }
+    return true;
 }
 
-template <bool W13>
+template <bool W13, int GPT>
 __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
 {
     extern __shared__ __align__(1024) uint8_t smem[];
@@ -348,15 +435,14 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
     RingShared *sh = reinterpret_cast<RingShared *>(smem + 256);
     uint8_t *ring = smem + kRingOff;
     const int S = p.nslots, group = p.group;
-    const int SB = slot_bytes(group), stmax = supertile_bytes(3, group);
-    float *xbuf = reinterpret_cast<float *>(smem + epi_off(S, group));
-    __half *hs = reinterpret_cast<__half *>(smem + epi_off(S, group) + kXbufBytes);
+    const int SB = slot_bytes(group), VB = vec_bytes(group);
+    const int vec_off0 = kKPS * 2 * supertile_bytes(3, group);
+    __half *hs2 = reinterpret_cast<__half *>(smem + kRingOff + (size_t)S * SB);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int U = W13 ? p.F / kBlockRows : ((p.H / kBlockRows + 1) / 2) * p.KS;
-    const int KTv = W13 ? p.H / kTileK : p.F / kTileK;  // column tiles of the activation vectors
-    const uint8_t *vfrag = W13 ? p.xfrag : p.hfrag;
-    const float *vtab = W13 ? p.xtab : p.htab;
-    const int tabf = tab_bytes(group) / 4;
+    const int nrb = W13 ? p.F / kBlockRows : p.H / kBlockRows;  // 128-row blocks of the matrix
+    const int U = W13 ? nrb : ((nrb + 1) / 2) * p.KS;
+    const int KTm = W13 ? p.H / kTileK : p.F / kTileK;  // column steps of the matrix and its vectors
+    const uint8_t *vbase = W13 ? p.xvec : p.hvec;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kMaxSlots; ++s) {
@@ -375,48 +461,56 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
         if (lane == 0 && !(p.debug & kDebugNoProducer)) {
             const uint64_t pol = policy_evict_first();
             const int total = *p.nchunks * U;
-            int it = 0;
+            int it = 0, pslot = 0;
+            uint32_t pphase = 0;  // phase of the ring round being filled
             bool ok = true;
+            uint32_t verified = 0;  // experts whose packed header has been checked
             while (ok) {
                 const int item = atomicAdd(&p.counters[W13 ? 0 : 1], 1);
                 if (item >= total) break;
                 const Item I = decode_item<W13>(p, item, U);
                 const int e = I.ci.e, bits = I.ci.bits, NT = I.ci.nv > 8 ? 2 : 1;
-                if (!header_ok(p, e)) {
-                    set_status(p.status, MC_ERR_BAD_PACK);
-                    sh->abort = 1;
-                    ok = false;
-                    break;
-                }
-                const int TB = tile_bytes(bits, group), STB = kTilesPerBlock * TB;
-                const int KTm = W13 ? p.H / kTileK : p.F / kTileK;
-                const uint8_t *matA = p.packed + p.mat_off[e][W13 ? 0 : 2];
-                const uint8_t *matB = p.packed + p.mat_off[e][W13 ? 1 : 2];
-                const uint32_t fbytes = NT * (kFragBytes / 2), tbytes = NT * (tabf * 4 / 2);
-                for (int i = 0; i < I.nkt; ++i, ++it) {
-                    const int slot = it % S;
-                    if (it >= S && !wait_or_abort(&empty[slot], ((it / S) - 1) & 1, p, sh)) {
+                if (!((verified >> e) & 1u)) {
+                    if (!header_ok(p, e)) {
+                        set_status(p.status, MC_ERR_BAD_PACK);
+                        sh->abort = 1;
                         ok = false;
                         break;
                     }
-                    const int kt = I.kt0 + i;
+                    verified |= 1u << e;
+                }
+                const int STB = supertile_bytes(bits, group);
+                // one column step of both streams is pw contiguous supertiles
+                const int pw = W13 ? 2 : w2_pair_width(I.blkA >> 1, nrb);
+                const uint8_t *wsrc =
+                    p.packed + p.mat_off[e][W13 ? 0 : 2] + supertile_off(W13 ? 0 : 2, I.blkA, I.kt0, KTm, nrb, STB);
+                for (int i = 0; i < I.nkt; i += kKPS, ++it) {
+                    const int slot = pslot;
+                    if (it >= S && !wait_or_abort(&empty[slot], pphase ^ 1u, p, sh)) {
+                        ok = false;
+                        break;
+                    }
+                    if (++pslot == S) {
+                        pslot = 0;
+                        pphase ^= 1u;
+                    }
+                    const int kc = min(kKPS, I.nkt - i);
                     sh->slot_item[slot] = item;
-                    sh->slot_i[slot] = i;
+                    sh->slot_kc[slot] = kc;
                     uint8_t *dst = ring + (size_t)slot * SB;
-                    const size_t vt = (size_t)I.k * KTv + kt;
-                    mbar_arrive_expect_tx(&full[slot], (I.blkB >= 0 ? 2 * STB : STB) + fbytes + tbytes);
-                    bulk_g2s_stream(dst, matA + ((size_t)I.blkA * KTm + kt) * STB, STB, &full[slot], pol);
-                    if (I.blkB >= 0)
-                        bulk_g2s_stream(dst + stmax, matB + ((size_t)I.blkB * KTm + kt) * STB, STB, &full[slot], pol);
-                    bulk_g2s(dst + 2 * stmax, vfrag + vt * kFragBytes, fbytes, &full[slot]);
-                    bulk_g2s(dst + 2 * stmax + kFragBytes, vtab + vt * tabf, tbytes, &full[slot]);
+                    const uint32_t wb = (uint32_t)(kc * pw * STB), vb = (uint32_t)(kc * VB);
+                    mbar_arrive_expect_tx(&full[slot], wb + NT * vb);
+                    bulk_g2s_stream(dst, wsrc + (size_t)i * pw * STB, wb, &full[slot], pol);
+                    for (int j = 0; j < NT; ++j)
+                        bulk_g2s(dst + vec_off0 + j * kKPS * VB, vbase + vec_off(I.k, j, I.kt0 + i, KTm, group), vb,
+                                 &full[slot]);
                     sh->issued = it + 1;
                 }
             }
             if (ok) {
                 // end marker: one more stage with item -1 and no data
-                const int slot = it % S;
-                if (it < S || wait_or_abort(&empty[slot], ((it / S) - 1) & 1, p, sh)) {
+                const int slot = pslot;
+                if (it < S || wait_or_abort(&empty[slot], pphase ^ 1u, p, sh)) {
                     sh->slot_item[slot] = -1;
                     mbar_arrive(&full[slot]);
                 }
@@ -424,38 +518,28 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
         }
     } else {
         // --------------------------------------------------------- consumers --
-        const int x = warp >> 3, tl = warp & 7;
-        float y[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-        int cur = -1, cbar_uses = 0;
-        Item I;
-        I.k = 0;
-        for (int it = 0;; ++it) {
-            const int slot = it % S;
-            if (!wait_or_abort(&full[slot], (it / S) & 1, p, sh)) break;
+        const Ring R{full, empty, ring, S, SB, vec_off0, VB};
+        int slot = 0, items = 0;
+        uint32_t phase = 0;
+        while (true) {
+            if (!wait_or_abort(&full[slot], phase, p, sh)) break;
             const int item = sh->slot_item[slot];
             if (item < 0) break;
-            if (item != cur) {
-                if (cur >= 0) epilogue<W13>(p, I, y, x, tl, lane, warp, xbuf, hs, sh, cbar_uses);
-                cur = item;
-                I = decode_item<W13>(p, item, U);
-#pragma unroll
-                for (int j = 0; j < 2; ++j)
-#pragma unroll
-                    for (int c = 0; c < 4; ++c) y[j][c] = 0.f;
+            const Item I = decode_item<W13>(p, item, U);
+            const int sel = (I.ci.bits - 1) * 2 + (I.ci.nv > 8 ? 1 : 0);
+            bool ok;
+#define MC_RUN(NT_, B_) run_item<W13, NT_, B_, GPT>(p, sh, R, I, nrb, warp, lane, slot, phase, hs2, items)
+            switch (sel) {
+            case 0: ok = MC_RUN(1, 1); break;
+            case 1: ok = MC_RUN(2, 1); break;
+            case 2: ok = MC_RUN(1, 2); break;
+            case 3: ok = MC_RUN(2, 2); break;
+            case 4: ok = MC_RUN(1, 3); break;
+            default: ok = MC_RUN(2, 3); break;
             }
-            const uint8_t *base = ring + (size_t)slot * SB;
-            if (!(x == 1 && I.blkB < 0)) {
-                const int TB = tile_bytes(I.ci.bits, group);
-                const uint8_t *tile = base + x * stmax + tl * TB;
-                const uint4 *frag = reinterpret_cast<const uint4 *>(base + 2 * stmax);
-                const float *tab = reinterpret_cast<const float *>(base + 2 * stmax + kFragBytes);
-                if (I.ci.nv > 8) stage_dispatch<2>(I.ci.bits, tile, frag, tab, group, lane, y);
-                else stage_dispatch<1>(I.ci.bits, tile, frag, tab, group, lane, y);
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&empty[slot]);
+#undef MC_RUN
+            if (!ok) break;
         }
-        if (cur >= 0 && !sh->abort) epilogue<W13>(p, I, y, x, tl, lane, warp, xbuf, hs, sh, cbar_uses);
     }
     __syncthreads();
     // On an abort, let copies that were issued but never consumed land before the
@@ -513,9 +597,10 @@ int launch_gemv(ExpertParams ep, cudaStream_t st)
     if (nslots < 2) return set_error(MC_ERR_UNSUPPORTED, "not enough shared memory for the GEMV ring");
     ep.nslots = nslots;
     const size_t sm = gemv_smem(nslots, ep.group);
-    err = cudaFuncSetAttribute(gemv_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-    if (err == cudaSuccess)
-        err = cudaFuncSetAttribute(gemv_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    auto k13 = ep.group == 64 ? gemv_kernel<true, 2> : gemv_kernel<true, 1>;
+    auto k2 = ep.group == 64 ? gemv_kernel<false, 2> : gemv_kernel<false, 1>;
+    err = cudaFuncSetAttribute(k13, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (err == cudaSuccess) err = cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(err));
 
     profile_begin(kKGemmGather, st);
@@ -524,13 +609,13 @@ int launch_gemv(ExpertParams ep, cudaStream_t st)
     err = cudaGetLastError();
     if (err == cudaSuccess) {
         profile_begin(kKGemvW13, st);
-        gemv_kernel<true><<<nsm, kGemvThreads, sm, st>>>(ep);
+        k13<<<nsm, kGemvThreads, sm, st>>>(ep);
         profile_end(kKGemvW13, st);
         err = cudaGetLastError();
     }
     if (err == cudaSuccess) {
         profile_begin(kKGemvW2, st);
-        gemv_kernel<false><<<nsm, kGemvThreads, sm, st>>>(ep);
+        k2<<<nsm, kGemvThreads, sm, st>>>(ep);
         profile_end(kKGemvW2, st);
         err = cudaGetLastError();
     }

@@ -27,6 +27,16 @@ constexpr int kFragBytes = 2 * 8 * 32 * 8;
 // Offset tables of one chunk and one tile: [n (16)][group-in-tile][8 floats].
 __host__ __device__ inline int tab_bytes(int group) { return kChunk * (kTileK / group) * kTabFloats * 4; }
 
+// Vector block of the mma.sync path: one (chunk, n-tile j, 128-column step),
+//   [fragments of pairs 8j..8j+7: 256 x 8 bytes][their offset tables [8][g][8]]
+// stored [chunk][j (2)][column step] so that consecutive steps are contiguous.
+constexpr int kVecFragBytes = 2048;
+__host__ __device__ inline int vec_bytes(int group) { return kVecFragBytes + 8 * (kTileK / group) * kTabFloats * 4; }
+__host__ __device__ inline size_t vec_off(int k, int j, int kt, int KT, int group)
+{
+    return (((size_t)k * 2 + j) * KT + kt) * (size_t)vec_bytes(group);
+}
+
 struct RouteParams {
     const __nv_bfloat16 *x;     // [T, H]
     const __nv_bfloat16 *gate;  // [E, H]
@@ -70,6 +80,8 @@ struct ExpertParams {
     uint8_t *hfrag;          // [max_chunks][F/128] kFragBytes
     float *htab;             // [max_chunks][F/128] tab_bytes
     float *gu;               // [max_chunks][2][F][16] W1 / W3 results (tensor-core path)
+    uint8_t *xvec;           // [max_chunks][2][H/128] vector blocks of x (mma.sync path)
+    uint8_t *hvec;           // [max_chunks][2][F/128] vector blocks of h (mma.sync path)
     float *opart;            // [KS, Pmax, H]  expert outputs (fp32), pair order
     int KS;                  // column splits of the W2 pass
     int Pmax;                // 2 * T

@@ -3,9 +3,14 @@
 //
 // Storage of one quantised matrix W [R, K] (groups of g along K, b bits):
 //   tile      = 16 rows x 128 columns; bytes = 256*b (codes) + 64*(128/g) (meta)
-//   supertile = the 8 tiles of a 128-row block at one 128-column step
-//   order     = [R/128][K/128][8 tiles]  -> one supertile is contiguous
-//
+//   supertile = the 8 tiles of a 128-row block at one 128-column step (STB bytes)
+// Supertiles are stored so that the expert kernels stream one large contiguous
+// block per step:
+//   W1 / W3 of an expert share one region, interleaved per supertile:
+//       [F/128 row blocks][H/128 column steps][W1 supertile][W3 supertile]
+//   W2 pairs its row blocks:
+//       [H/256 row-block pairs][F/128 column steps][block 2p][block 2p+1]
+//       (when H/128 is odd the last pair holds one block)
 // Inside a tile every one of the 32 lanes of a warp owns 64 codes: rows r0 = g8
 // and r1 = g8 + 8 (g8 = lane / 4), and for each row two runs of 16 consecutive
 // columns, so that an mma.sync.m16n8k16 A-fragment register (two consecutive
@@ -49,7 +54,7 @@ constexpr int kTileK = 128;
 constexpr int kBlockRows = 128;   // rows of a supertile
 constexpr int kTilesPerBlock = 8;
 constexpr uint32_t kMagic = 0x4B50434Du;  // "MCPK"
-constexpr uint32_t kFormatVersion = 1;
+constexpr uint32_t kFormatVersion = 3;
 constexpr int kMaxE = 16;
 constexpr int kHeaderBytes = 4096;
 
@@ -72,11 +77,22 @@ MC_HD uint64_t mat_bytes(int rows, int cols, int bits, int group)
 {
     return (uint64_t)(rows / kTileRows) * (uint64_t)(cols / kTileK) * (uint64_t)tile_bytes(bits, group);
 }
-// byte offset of tile (row block rb16 of 16 rows, column tile kt) inside a matrix
-MC_HD uint64_t tile_offset(int rb16, int kt, int KT, int bits, int group)
+// Byte offset of supertile (128-row block rb, column step kt) of matrix m
+// (0 = W1, 1 = W3: offsets inside the shared W1/W3 region; 2 = W2: inside the
+// W2 region).  KT = column steps of the matrix, nrb = its 128-row blocks.
+MC_HD uint64_t supertile_off(int m, int rb, int kt, int KT, int nrb, int STB)
 {
-    uint64_t st = (uint64_t)(rb16 >> 3) * (uint64_t)KT + (uint64_t)kt;
-    return (st * kTilesPerBlock + (uint64_t)(rb16 & 7)) * (uint64_t)tile_bytes(bits, group);
+    if (m < 2) return (((uint64_t)rb * KT + kt) * 2 + m) * (uint64_t)STB;
+    const int pr = rb >> 1, pw = (2 * pr + 1 < nrb) ? 2 : 1;
+    return ((uint64_t)pr * KT * 2 + (uint64_t)kt * pw + (rb & 1)) * (uint64_t)STB;
+}
+// supertiles per column step of W2 row-block pair pr
+MC_HD int w2_pair_width(int pr, int nrb) { return (2 * pr + 1 < nrb) ? 2 : 1; }
+// byte offset of tile (16-row block rb16, column step kt) of matrix m
+MC_HD uint64_t tile_off(int m, int rb16, int kt, int KT, int nrb, int bits, int group)
+{
+    const int TB = tile_bytes(bits, group);
+    return supertile_off(m, rb16 >> 3, kt, KT, nrb, kTilesPerBlock * TB) + (uint64_t)(rb16 & 7) * TB;
 }
 
 // row (0..15) and first column (0..127) of pair j of lane `lane` in a tile

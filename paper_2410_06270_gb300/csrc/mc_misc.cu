@@ -7,13 +7,13 @@
 namespace mc {
 
 // One thread per (tile, lane): the exact inverse of mc_pack.cpp's packing.
-__global__ void unpack_kernel(const uint8_t *packed, uint64_t mat_off, int rows, int cols, int bits, int group,
-                              int E, int H, int F, int expert, uint8_t *codes, uint16_t *scale, uint16_t *zero,
-                              int32_t *status)
+__global__ void unpack_kernel(const uint8_t *packed, uint64_t mat_off, int mat, int rows, int cols, int bits,
+                              int group, int E, int H, int F, int expert, uint8_t *codes, uint16_t *scale,
+                              uint16_t *zero, int32_t *status)
 {
     const PackHeader *hd = reinterpret_cast<const PackHeader *>(packed);
     if (hd->magic != kMagic || hd->version != kFormatVersion || hd->E != E || hd->H != H || hd->F != F ||
-        hd->group != group || hd->bits[expert] != bits) {
+        hd->group != group || hd->bits[expert] != bits || hd->mat_off[expert][mat] != mat_off) {
         if (blockIdx.x == 0 && threadIdx.x == 0) set_status(status, MC_ERR_BAD_PACK);
         return;
     }
@@ -23,7 +23,7 @@ __global__ void unpack_kernel(const uint8_t *packed, uint64_t mat_off, int rows,
     const int tile_id = gid >> 5, lane = gid & 31;
     if (tile_id >= ntiles) return;
     const int rb = tile_id / KT, kt = tile_id % KT;
-    const uint8_t *tile = packed + mat_off + tile_offset(rb, kt, KT, bits, group);
+    const uint8_t *tile = packed + mat_off + tile_off(mat, rb, kt, KT, rows / kBlockRows, bits, group);
     const int R0 = rb * kTileRows, K0 = kt * kTileK;
     uint32_t w2[4] = {0, 0, 0, 0}, w1[2] = {0, 0};
     if (bits >= 2) {
@@ -112,7 +112,7 @@ int mc_unpack_experts(const mc_shape *shape, const int8_t *bits_host, const void
     const int ntiles = (rows / kTileRows) * (cols / kTileK);
     const long threads = (long)ntiles * 32;
     unpack_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, (cudaStream_t)stream>>>(
-        (const uint8_t *)packed_dev, off[expert][mat], rows, cols, bits_host[expert], shape->group, shape->E,
+        (const uint8_t *)packed_dev, off[expert][mat], mat, rows, cols, bits_host[expert], shape->group, shape->E,
         shape->H, shape->F, expert, codes_dev, scale_dev, zero_dev, status_dev);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return set_error(MC_ERR_CUDA, "unpack launch: %s", cudaGetErrorString(e));

@@ -55,26 +55,28 @@ int check_bits(const mc_shape *s, const int8_t *bits)
 void layout_offsets(const mc_shape *s, const int8_t *bits, uint64_t off[kMaxE][3], uint64_t *total)
 {
     uint64_t pos = kHeaderBytes;
-    for (int e = 0; e < s->E; ++e)
-        for (int m = 0; m < 3; ++m) {
-            int rows = m < 2 ? s->F : s->H, cols = m < 2 ? s->H : s->F;
-            off[e][m] = pos;
-            pos += mat_bytes(rows, cols, bits[e], s->group);
-            pos = (pos + 255) & ~(uint64_t)255;
-        }
+    for (int e = 0; e < s->E; ++e) {
+        // W1 and W3 share one interleaved region; W2 follows
+        off[e][0] = off[e][1] = pos;
+        pos += 2 * mat_bytes(s->F, s->H, bits[e], s->group);
+        pos = (pos + 255) & ~(uint64_t)255;
+        off[e][2] = pos;
+        pos += mat_bytes(s->H, s->F, bits[e], s->group);
+        pos = (pos + 255) & ~(uint64_t)255;
+    }
     *total = pos;
 }
 
 // Pack one matrix [rows, cols] into its tile stream.  Returns false on a code
 // that does not fit in `bits`.
-static bool pack_matrix(int rows, int cols, int bits, int group, const uint8_t *codes,
+static bool pack_matrix(int m, int rows, int cols, int bits, int group, const uint8_t *codes,
                         const uint16_t *scale, const uint16_t *zero, uint8_t *dst, int rb_lo, int rb_hi)
 {
-    const int KT = cols / kTileK, ng = cols / group, gpt = kTileK / group;
+    const int KT = cols / kTileK, ng = cols / group, gpt = kTileK / group, nrb = rows / kBlockRows;
     const uint32_t lim = 1u << bits;
     for (int rb = rb_lo; rb < rb_hi; ++rb)
         for (int kt = 0; kt < KT; ++kt) {
-            uint8_t *tile = dst + tile_offset(rb, kt, KT, bits, group);
+            uint8_t *tile = dst + tile_off(m, rb, kt, KT, nrb, bits, group);
             const int R0 = rb * kTileRows, K0 = kt * kTileK;
             uint8_t *plane2 = tile;                                // 32 lanes x 16 B
             uint8_t *plane1 = tile + (bits >= 2 ? 512 : 0);        // 32 lanes x 8 B
@@ -115,13 +117,13 @@ static bool pack_matrix(int rows, int cols, int bits, int group, const uint8_t *
     return true;
 }
 
-static void unpack_matrix(int rows, int cols, int bits, int group, const uint8_t *src,
+static void unpack_matrix(int m, int rows, int cols, int bits, int group, const uint8_t *src,
                           uint8_t *codes, uint16_t *scale, uint16_t *zero)
 {
-    const int KT = cols / kTileK, ng = cols / group, gpt = kTileK / group;
+    const int KT = cols / kTileK, ng = cols / group, gpt = kTileK / group, nrb = rows / kBlockRows;
     for (int rb = 0; rb < rows / kTileRows; ++rb)
         for (int kt = 0; kt < KT; ++kt) {
-            const uint8_t *tile = src + tile_offset(rb, kt, KT, bits, group);
+            const uint8_t *tile = src + tile_off(m, rb, kt, KT, nrb, bits, group);
             const int R0 = rb * kTileRows, K0 = kt * kTileK;
             const uint8_t *plane2 = tile, *plane1 = tile + (bits >= 2 ? 512 : 0);
             for (int lane = 0; lane < 32; ++lane) {
@@ -223,7 +225,7 @@ int mc_pack_experts_host(const mc_shape *shape, const int8_t *bits_host,
             const Item &it = items[i];
             int rows = it.m < 2 ? shape->F : shape->H, cols = it.m < 2 ? shape->H : shape->F;
             int k = 3 * it.e + it.m;
-            if (!pack_matrix(rows, cols, bits_host[it.e], shape->group, codes_host[k], scale_host[k],
+            if (!pack_matrix(it.m, rows, cols, bits_host[it.e], shape->group, codes_host[k], scale_host[k],
                              zero_host[k], base + off[it.e][it.m], it.rb_lo, it.rb_hi)) {
                 bad[id] = k;
                 return;
@@ -257,8 +259,8 @@ int mc_unpack_experts_host(const void *packed_host, size_t packed_bytes, int exp
     if (expert < 0 || expert >= hd->E || mat < 0 || mat > 2)
         return set_error(MC_ERR_INVALID_ARG, "expert %d / matrix %d out of range", expert, mat);
     int rows = mat < 2 ? hd->F : hd->H, cols = mat < 2 ? hd->H : hd->F;
-    unpack_matrix(rows, cols, hd->bits[expert], hd->group, (const uint8_t *)packed_host + hd->mat_off[expert][mat],
-                  codes_host, scale_host, zero_host);
+    unpack_matrix(mat, rows, cols, hd->bits[expert], hd->group,
+                  (const uint8_t *)packed_host + hd->mat_off[expert][mat], codes_host, scale_host, zero_host);
     return MC_OK;
 }
 

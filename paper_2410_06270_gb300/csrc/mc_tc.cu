@@ -359,7 +359,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_kernel(ExpertParams p)
                     mbar_arrive_expect_tx(&sh->full[slot], kFragBytes + tabf * 4 + STB);
                     bulk_g2s(dst + kSlotBImg, vimg + vt * kFragBytes, kFragBytes, &sh->full[slot]);
                     bulk_g2s(dst + kSlotTab, vtab + vt * tabf, tabf * 4, &sh->full[slot]);
-                    bulk_g2s_stream(dst + kSlotPack, mat + ((size_t)I.blk * KTm + kt) * STB, STB, &sh->full[slot],
+                    bulk_g2s_stream(dst + kSlotPack,
+                                    mat + supertile_off(I.mat, I.blk, kt, KTm,
+                                                        (I.mat < 2 ? p.F : p.H) / kBlockRows, STB),
+                                    STB, &sh->full[slot],
                                     pol);
                     sh->issued = it + 1;
                 }
