@@ -129,7 +129,7 @@ __device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1
 
 // ------------------------------------------------------- code -> fp16 pairs --
 // (w & field_mask) | exponent constant: an fp16 pair reading (2^E + q) with
-// E = 10 - width * position (see mc_layout.h).
+// E = 10 - (mantissa bit of the field) (see mc_layout.h).
 
 __device__ __forceinline__ uint32_t lop_and_or(uint32_t w, uint32_t mask, uint32_t c)
 {
@@ -141,7 +141,7 @@ __device__ __forceinline__ uint32_t lop_and_or(uint32_t w, uint32_t mask, uint32
 // fp16 exponent constants, both halves.
 #define MC_C(e) (((uint32_t)(e) << 10) * 0x00010001u)
 
-// 2-bit plane word -> 8 registers (positions 0..7)
+// 2-bit code word -> 8 registers (positions 0..7)
 __device__ __forceinline__ void cvt2(uint32_t w, uint32_t (&r)[8])
 {
     r[0] = lop_and_or(w, 0x00030003u, MC_C(25));
@@ -155,34 +155,49 @@ __device__ __forceinline__ void cvt2(uint32_t w, uint32_t (&r)[8])
     r[7] = lop_and_or(v, 0x00300030u, MC_C(21));
 }
 
-// 1-bit plane word, positions [p0, p0+8) -> 8 registers.  HI4 scales by 4
-// (exponent + 2), which is how the third bit of a 3-bit code is weighted.
-template <bool HI4>
+// 1-bit code word, positions [p0, p0+8) -> 8 registers (p0 = 0 or 8).
 __device__ __forceinline__ void cvt1_half(uint32_t w, int p0, uint32_t (&r)[8])
 {
-    constexpr int b = HI4 ? 27 : 25;
-    uint32_t v = w >> 10;
+    const uint32_t v = w >> 10;
     if (p0 == 0) {
 #pragma unroll
-        for (int p = 0; p < 8; ++p) r[p] = lop_and_or(w, 0x00010001u << p, MC_C(b - p));
+        for (int p = 0; p < 8; ++p) r[p] = lop_and_or(w, 0x00010001u << p, MC_C(25 - p));
     } else {
-        r[0] = lop_and_or(w, 0x00010001u << 8, MC_C(b - 8));
-        r[1] = lop_and_or(w, 0x00010001u << 9, MC_C(b - 9));
+        r[0] = lop_and_or(w, 0x00010001u << 8, MC_C(17));
+        r[1] = lop_and_or(w, 0x00010001u << 9, MC_C(16));
 #pragma unroll
-        for (int p = 0; p < 6; ++p) r[2 + p] = lop_and_or(v, 0x00010001u << p, MC_C(b - p));
+        for (int p = 0; p < 6; ++p) r[2 + p] = lop_and_or(v, 0x00010001u << p, MC_C(25 - p));
     }
 }
 
-// 1-bit plane word, all 16 positions -> 16 registers.
-template <bool HI4>
-__device__ __forceinline__ void cvt1(uint32_t w, uint32_t (&r)[16])
+// (x & m) | (y & ~m)
+__device__ __forceinline__ uint32_t lop_sel(uint32_t x, uint32_t y, uint32_t m)
 {
-    constexpr int b = HI4 ? 27 : 25;
-    const uint32_t v = w >> 10;
+    uint32_t r;
+    asm("lop3.b32 %0, %1, %2, %3, 0xE4;" : "=r"(r) : "r"(x), "r"(y), "r"(m));
+    return r;
+}
+
+// 3-bit code words (6 per lane) -> the 8 registers of pairs 8qd .. 8qd+7.
+// Pairs j < 30 take one LOP3 each (fields at mantissa bits 1, 4, 7 directly,
+// fields at bits 10, 13 after a shift by 10); pairs 30 and 31 gather their
+// three bits from bit 0 / 16 of three words.
+__device__ __forceinline__ uint32_t cvt3_pair(const uint32_t (&w)[6], int j)
+{
+    if (j < 30) {
+        const int i = j / 5, p = j % 5;
+        if (p < 3) return lop_and_or(w[i], 0x00070007u << (1 + 3 * p), MC_C(24 - 3 * p));
+        return lop_and_or(w[i] >> 10, 0x00070007u << (3 * (p - 3)), MC_C(25 - 3 * (p - 3)));
+    }
+    const int b = 3 * (j - 30);
+    const uint32_t t = lop_sel(w[b], w[b + 1] << 1, 0x00010001u);
+    return lop_and_or(lop_sel(t, w[b + 2] << 2, 0x00030003u), 0x00070007u, MC_C(25));
+}
+
+__device__ __forceinline__ void cvt3(const uint32_t (&w)[6], int qd, uint32_t (&r)[8])
+{
 #pragma unroll
-    for (int p = 0; p < 10; ++p) r[p] = lop_and_or(w, 0x00010001u << p, MC_C(b - p));
-#pragma unroll
-    for (int p = 0; p < 6; ++p) r[10 + p] = lop_and_or(v, 0x00010001u << p, MC_C(b - p));
+    for (int i = 0; i < 8; ++i) r[i] = cvt3_pair(w, 8 * qd + i);
 }
 
 __device__ __forceinline__ float silu(float g) { return g / (1.0f + __expf(-g)); }

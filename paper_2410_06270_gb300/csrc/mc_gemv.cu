@@ -23,7 +23,7 @@
 //        h = silu(W1 x) * (W3 x) in registers and the CTA writes W2's vector
 //        blocks.
 //   W2:  streams = two 128-row blocks of W2; the epilogue writes fp32 outputs.
-// Decoding costs one ALU instruction per two weights of a bit plane, so the
+// Decoding costs about one ALU instruction per two weights, so the
 // consumers are kept lean: this path is bound by HBM bandwidth on the packed
 // weight bytes only while the decode keeps up with it.
 #include "mc_host.h"
@@ -94,9 +94,9 @@ __device__ __forceinline__ bool header_ok(const ExpertParams &p, int e)
 //     4 fp16 values at columns 64(s/4) + 16t + 4(s%4) .. +3 of pair 8j + lane/4;
 //   then the offset tables of pairs 8j .. 8j+7, [n][group][8 floats]:
 //     [O2 half 0, O2 half 1, X, O1 half 0, O3 half 0, O3 half 1, X, O1 half 1]
-//   (X = sum of the group's inputs, O_b = sum of the b-bit plane offsets times
-//   the inputs for the rows of one half, O3 = O2 + 4 O1; mc_layout.h), so that a
-//   2- or 3-bit fold reads its O pair and X with one 16-byte load.
+//   (X = sum of the group's inputs, O_b = sum of the b-bit field offsets times
+//   the inputs for the rows of one half; mc_layout.h), so that a 2- or 3-bit
+//   fold reads its O pair and X with one 16-byte load.
 // Threads share the fragment entries; one warp per table item.
 __device__ __forceinline__ void write_vec_block(const __half *rows, int j, int group, uint8_t *dst, int tid,
                                                 int nthreads, int warp, int nwarps, int lane)
@@ -111,7 +111,7 @@ __device__ __forceinline__ void write_vec_block(const __half *rows, int j, int g
     float *tab = reinterpret_cast<float *>(dst + kVecFragBytes);
     for (int item = warp; item < 8 * gpt; item += nwarps) {
         const int nl = item / gpt, gi = item % gpt, n = 8 * j + nl;
-        float tb[5] = {0, 0, 0, 0, 0};
+        float tb[7] = {0, 0, 0, 0, 0, 0, 0};
         for (int c = gi * group + lane; c < (gi + 1) * group; c += 32) {
             const float v = __half2float(rows[n * kTileK + c]);
             const int j0 = pair_of_col(c, 0), j1 = pair_of_col(c, 1);
@@ -120,15 +120,17 @@ __device__ __forceinline__ void write_vec_block(const __half *rows, int j, int g
             tb[2] = fmaf(off1(j1), v, tb[2]);
             tb[3] = fmaf(off2(j0), v, tb[3]);
             tb[4] = fmaf(off2(j1), v, tb[4]);
+            tb[5] = fmaf(off3(j0), v, tb[5]);
+            tb[6] = fmaf(off3(j1), v, tb[6]);
         }
 #pragma unroll
-        for (int k = 0; k < 5; ++k)
+        for (int k = 0; k < 7; ++k)
 #pragma unroll
             for (int m = 16; m >= 1; m >>= 1) tb[k] += __shfl_xor_sync(0xffffffffu, tb[k], m);
         if (lane == 0) {
             float4 *d = reinterpret_cast<float4 *>(tab + (size_t)item * kTabFloats);
             d[0] = make_float4(tb[3], tb[4], tb[0], tb[1]);
-            d[1] = make_float4(tb[3] + 4.f * tb[1], tb[4] + 4.f * tb[2], tb[0], tb[2]);
+            d[1] = make_float4(tb[5], tb[6], tb[0], tb[2]);
         }
     }
 }
@@ -207,14 +209,16 @@ __device__ __forceinline__ void load_tile(const uint8_t *tile, int lane, TileReg
     for (int g = 0; g < GPT; ++g) t.meta[g] = *reinterpret_cast<const uint2 *>(mt + 64 * g + (lane >> 2) * 8);
 }
 
-// A-fragment registers of k-steps 2qd, 2qd+1: r (low / only plane), rh (3-bit
-// high plane, weighted x4 through its exponent).
+// A-fragment registers of k-steps 2qd, 2qd+1 (pairs 8qd .. 8qd+7).
 template <int BITS, int GPT>
-__device__ __forceinline__ void decode_qd(const TileRegs<BITS, GPT> &t, int qd, uint32_t (&r)[8], uint32_t (&rh)[8])
+__device__ __forceinline__ void decode_qd(const TileRegs<BITS, GPT> &t, int qd, uint32_t (&r)[8])
 {
-    if (BITS == 1) cvt1_half<false>(t.c1[qd >> 1], 8 * (qd & 1), r);
-    if (BITS >= 2) cvt2(t.c2[qd], r);
-    if (BITS == 3) cvt1_half<true>(t.c1[qd >> 1], 8 * (qd & 1), rh);
+    if (BITS == 1) cvt1_half(t.c1[qd >> 1], 8 * (qd & 1), r);
+    if (BITS == 2) cvt2(t.c2[qd], r);
+    if (BITS == 3) {
+        const uint32_t w[6] = {t.c2[0], t.c2[1], t.c2[2], t.c2[3], t.c1[0], t.c1[1]};
+        cvt3(w, qd, r);
+    }
 }
 
 // y += s * (acc0 + acc1 - O - z X) for the lane's four C-fragment entries:
@@ -233,8 +237,8 @@ __device__ __forceinline__ void fold(float (&y)[4], const float (&a0)[4], const 
 // One consumer warp, one 128-column step of its 16-row tile in both streams:
 // decode, mma and fold.  y*[j][c]: C-fragment layout, rows g8 / g8+8 of the
 // tile, pairs 8j + 2t + {0,1}.  vec0 / vec1: the step's vector blocks of
-// n-tiles 0 / 1.  Two accumulators per tile and n-tile keep the dependent mma
-// chains short: 1/2-bit by k-step parity, 3-bit low plane / high plane.
+// n-tiles 0 / 1.  Two accumulators per tile and n-tile (by k-step parity) keep
+// the dependent mma chains short.
 template <int NT, int BITS, int GPT>
 __device__ __forceinline__ void step2(const uint8_t *tA, const uint8_t *tB, const uint8_t *vec0, const uint8_t *vec1,
                                       int lane, float (&yA)[NT][4], float (&yB)[NT][4])
@@ -246,35 +250,26 @@ __device__ __forceinline__ void step2(const uint8_t *tA, const uint8_t *tB, cons
     float accA[2][NT][4], accB[2][NT][4];
 #pragma unroll
     for (int qd = 0; qd < 4; ++qd) {
-        uint32_t ra[8], rha[8], rb[8], rhb[8];
-        decode_qd<BITS, GPT>(RA, qd, ra, rha);
-        decode_qd<BITS, GPT>(RB, qd, rb, rhb);
+        uint32_t ra[8], rb[8];
+        decode_qd<BITS, GPT>(RA, qd, ra);
+        decode_qd<BITS, GPT>(RB, qd, rb);
         uint4 bq[NT];
 #pragma unroll
         for (int j = 0; j < NT; ++j) bq[j] = reinterpret_cast<const uint4 *>(j ? vec1 : vec0)[qd * 32 + lane];
 #pragma unroll
         for (int kk = 0; kk < 2; ++kk) {
             const int s = 2 * qd + kk;
-            // the first k-step of a group (of each parity chain) starts from zero
-            const bool first = BITS == 3 ? (s % SPG == 0) : (s % SPG < 2);
+            // the first k-step of a group in each parity chain starts from zero
+            const bool first = s % SPG < 2;
 #pragma unroll
             for (int j = 0; j < NT; ++j) {
                 const uint32_t b0 = kk ? bq[j].z : bq[j].x, b1 = kk ? bq[j].w : bq[j].y;
-                const int ca = BITS == 3 ? 0 : kk;
                 if (first) {
-                    mma_acc<true>(accA[ca][j], ra + 4 * kk, b0, b1);
-                    mma_acc<true>(accB[ca][j], rb + 4 * kk, b0, b1);
-                    if (BITS == 3) {
-                        mma_acc<true>(accA[1][j], rha + 4 * kk, b0, b1);
-                        mma_acc<true>(accB[1][j], rhb + 4 * kk, b0, b1);
-                    }
+                    mma_acc<true>(accA[kk][j], ra + 4 * kk, b0, b1);
+                    mma_acc<true>(accB[kk][j], rb + 4 * kk, b0, b1);
                 } else {
-                    mma_acc<false>(accA[ca][j], ra + 4 * kk, b0, b1);
-                    mma_acc<false>(accB[ca][j], rb + 4 * kk, b0, b1);
-                    if (BITS == 3) {
-                        mma_acc<false>(accA[1][j], rha + 4 * kk, b0, b1);
-                        mma_acc<false>(accB[1][j], rhb + 4 * kk, b0, b1);
-                    }
+                    mma_acc<false>(accA[kk][j], ra + 4 * kk, b0, b1);
+                    mma_acc<false>(accB[kk][j], rb + 4 * kk, b0, b1);
                 }
             }
             if (s % SPG == SPG - 1) {

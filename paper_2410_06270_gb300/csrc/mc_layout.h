@@ -22,21 +22,25 @@
 // so groups of 64 and of 128 are both whole k-steps.
 //
 // Code words of a lane (b = bits):
-//   2-bit field plane, 4 words: word i holds pairs 8i..8i+7; pair position
-//       p = j%8 has its low-column code at bits [2p, 2p+1] and its high-column
-//       code at bits [16+2p, 17+2p].
-//   1-bit field plane, 2 words: word i holds pairs 16i..16i+15; position
-//       p = j%16 at bit p (low column) and bit 16+p (high column).
-//   b = 1: one 1-bit plane;  b = 2: one 2-bit plane;
-//   b = 3: a 2-bit plane of q & 3 followed by a 1-bit plane of q >> 2.
-// Code bytes of a tile: plane-major, then lane-major (lane l's words contiguous):
-//   [2-bit plane: 32 lanes x 16 B][1-bit plane: 32 lanes x 8 B] (as present).
+//   b = 1: 2 words, word i holds pairs 16i..16i+15; pair position p = j%16 has
+//       its low-column code at bit p and its high-column code at bit 16+p.
+//   b = 2: 4 words, word i holds pairs 8i..8i+7; position p = j%8 at bits
+//       [2p, 2p+1] (low column) and [16+2p, 17+2p] (high column).
+//   b = 3: 6 words.  Word i holds pairs 5i..5i+4 (i < 6, j < 30); position
+//       p = j%5 has its low-column code at bits [f, f+2], f = 1, 4, 7, 10, 13
+//       for p = 0..4, and its high-column code at bits [16+f, 18+f].  The
+//       remaining bits 0 and 16 of the six words hold pairs 30 and 31: bit c of
+//       the low- (high-) column code of pair 30 + u is bit 0 (16) of word 3u + c.
+// Code bytes of a tile, lane-major inside each part:
+//   b = 1: [32 lanes x 8 B]    b = 2: [32 lanes x 16 B]
+//   b = 3: [32 lanes x 16 B: words 0..3][32 lanes x 8 B: words 4, 5]
 // Meta bytes of a tile: [group-in-tile][g8 = 0..7][s(r0), z(r0), s(r1), z(r1)] fp16.
 //
-// Decoding without shifts per field: a field at mantissa position p' of an fp16
-// whose exponent field is set to 15 + E reads as 2^E + q * 2^(E + width*p' - 10);
-// choosing E = 10 - width*p' makes it (2^E + q).  The constant 2^E ("offset")
-// depends only on the field position, so sum_k (off_k + q_k) x_k - sum_k off_k x_k
+// Decoding without shifts per field: a field at mantissa bit f of an fp16 whose
+// exponent field is set to 15 + E reads as 2^E + q * 2^(E + f - 10); choosing
+// E = 10 - f makes it (2^E + q).  Fields above the mantissa (bits 10..15 of a
+// half) are first shifted down by 10.  The constant 2^E ("offset") depends only
+// on the field position, so sum_k (off_k + q_k) x_k - sum_k off_k x_k
 // = sum_k q_k x_k, and the second sum is a per-(vector, group) table.
 #pragma once
 #include <stdint.h>
@@ -54,7 +58,7 @@ constexpr int kTileK = 128;
 constexpr int kBlockRows = 128;   // rows of a supertile
 constexpr int kTilesPerBlock = 8;
 constexpr uint32_t kMagic = 0x4B50434Du;  // "MCPK"
-constexpr uint32_t kFormatVersion = 3;
+constexpr uint32_t kFormatVersion = 4;
 constexpr int kMaxE = 16;
 constexpr int kHeaderBytes = 4096;
 
@@ -112,18 +116,51 @@ MC_HD int pair_of_col(int col, int half)
     return 4 * s + 2 * u2 + half;
 }
 
-// field position inside its word -> offset value 2^E
+// Where bit c of the code of pair j sits for a lane: word index and bit inside
+// it; h = 0 for the pair's low column, 1 for its high column.
+MC_HD void code_bit(int bits, int j, int h, int c, int &word, int &bit)
+{
+    if (bits == 1) {
+        word = j >> 4;
+        bit = (j & 15) + 16 * h;
+    } else if (bits == 2) {
+        word = j >> 3;
+        bit = 2 * (j & 7) + c + 16 * h;
+    } else if (j < 30) {
+        word = j / 5;
+        bit = 1 + 3 * (j % 5) + c + 16 * h;
+    } else {
+        word = 3 * (j - 30) + c;
+        bit = 16 * h;
+    }
+}
+// byte offset of code word w of lane `lane` inside a tile
+MC_HD int code_word_off(int bits, int lane, int w)
+{
+    if (bits == 1) return 8 * lane + 4 * w;
+    if (bits == 2) return 16 * lane + 4 * w;
+    return w < 4 ? 16 * lane + 4 * w : 512 + 8 * lane + 4 * (w - 4);
+}
+
+// mantissa bit of the field of pair j after the decoder's shift -> offset 2^E
 MC_HD int off2_pos(int j) { int p = j & 7; return p < 5 ? p : p - 5; }
 MC_HD int off1_pos(int j) { int p = j & 15; return p < 10 ? p : p - 10; }
+MC_HD int off3_bit(int j)
+{
+    if (j >= 30) return 0;
+    const int f = 1 + 3 * (j % 5);
+    return f < 10 ? f : f - 10;
+}
 MC_HD float off2(int j) { return (float)(1 << (10 - 2 * off2_pos(j))); }
 MC_HD float off1(int j) { return (float)(1 << (10 - off1_pos(j))); }
+MC_HD float off3(int j) { return (float)(1 << (10 - off3_bit(j))); }
 
-// Per (vector, group) table of 8 floats used by the expert kernels:
+// Per (vector, group) table of 8 floats used by the tensor-core expert kernels:
 //   [0] X = sum of the group's fp16 inputs
-//   [1],[2] O1 for row halves 0/1  (1-bit plane offsets)
-//   [3],[4] O2 for row halves 0/1  (2-bit plane offsets)
-//   [5],[6] O3 = O2 + 4*O1          (3-bit: low plane + 4 x high plane)
-//   [7] unused
+//   [1] unused
+//   [2],[3] O1 for row halves 0/1  (sum of 1-bit offsets times the inputs)
+//   [4],[5] O2 for row halves 0/1  (2-bit offsets)
+//   [6],[7] O3 for row halves 0/1  (3-bit offsets)
 constexpr int kTabFloats = 8;
 
 }  // namespace mc

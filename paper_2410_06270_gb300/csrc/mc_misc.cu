@@ -25,32 +25,21 @@ __global__ void unpack_kernel(const uint8_t *packed, uint64_t mat_off, int mat, 
     const int rb = tile_id / KT, kt = tile_id % KT;
     const uint8_t *tile = packed + mat_off + tile_off(mat, rb, kt, KT, rows / kBlockRows, bits, group);
     const int R0 = rb * kTileRows, K0 = kt * kTileK;
-    uint32_t w2[4] = {0, 0, 0, 0}, w1[2] = {0, 0};
-    if (bits >= 2) {
-        uint4 v = *reinterpret_cast<const uint4 *>(tile + 16 * lane);
-        w2[0] = v.x; w2[1] = v.y; w2[2] = v.z; w2[3] = v.w;
-    }
-    if (bits != 2) {
-        uint2 v = *reinterpret_cast<const uint2 *>(tile + (bits >= 2 ? 512 : 0) + 8 * lane);
-        w1[0] = v.x; w1[1] = v.y;
-    }
+    uint32_t w[6] = {0, 0, 0, 0, 0, 0};
+    for (int wi = 0; wi < 2 * bits; ++wi) w[wi] = *reinterpret_cast<const uint32_t *>(tile + code_word_off(bits, lane, wi));
     for (int j = 0; j < 32; ++j) {
         int row, col;
         pair_pos(lane, j, row, col);
-        uint32_t qa = 0, qb = 0;
-        if (bits >= 2) {
-            int p = j & 7;
-            qa = (w2[j >> 3] >> (2 * p)) & 3u;
-            qb = (w2[j >> 3] >> (16 + 2 * p)) & 3u;
-        }
-        if (bits != 2) {
-            int p = j & 15, sh = bits == 1 ? 0 : 2;
-            qa |= ((w1[j >> 4] >> p) & 1u) << sh;
-            qb |= ((w1[j >> 4] >> (16 + p)) & 1u) << sh;
-        }
         uint8_t *d = codes + (size_t)(R0 + row) * cols + K0 + col;
-        d[0] = (uint8_t)qa;
-        d[1] = (uint8_t)qb;
+        for (int h = 0; h < 2; ++h) {
+            uint32_t q = 0;
+            for (int c = 0; c < bits; ++c) {
+                int wi, bi;
+                code_bit(bits, j, h, c, wi, bi);
+                q |= ((w[wi] >> bi) & 1u) << c;
+            }
+            d[h] = (uint8_t)q;
+        }
     }
     if (lane < 8 * gpt) {
         const int gi = lane >> 3, g8 = lane & 7;

@@ -78,28 +78,23 @@ static bool pack_matrix(int m, int rows, int cols, int bits, int group, const ui
         for (int kt = 0; kt < KT; ++kt) {
             uint8_t *tile = dst + tile_off(m, rb, kt, KT, nrb, bits, group);
             const int R0 = rb * kTileRows, K0 = kt * kTileK;
-            uint8_t *plane2 = tile;                                // 32 lanes x 16 B
-            uint8_t *plane1 = tile + (bits >= 2 ? 512 : 0);        // 32 lanes x 8 B
             for (int lane = 0; lane < 32; ++lane) {
-                uint32_t w2[4] = {0, 0, 0, 0}, w1[2] = {0, 0};
+                uint32_t w[6] = {0, 0, 0, 0, 0, 0};
                 for (int j = 0; j < 32; ++j) {
                     int row, col;
                     pair_pos(lane, j, row, col);
                     const uint8_t *src = codes + (size_t)(R0 + row) * cols + K0 + col;
-                    uint32_t qa = src[0], qb = src[1];
-                    if (qa >= lim || qb >= lim) return false;
-                    if (bits >= 2) {
-                        int p = j & 7;
-                        w2[j >> 3] |= ((qa & 3u) << (2 * p)) | ((qb & 3u) << (16 + 2 * p));
-                    }
-                    if (bits != 2) {
-                        int p = j & 15;
-                        uint32_t ha = bits == 1 ? qa : (qa >> 2), hb = bits == 1 ? qb : (qb >> 2);
-                        w1[j >> 4] |= (ha << p) | (hb << (16 + p));
+                    for (int h = 0; h < 2; ++h) {
+                        const uint32_t q = src[h];
+                        if (q >= lim) return false;
+                        for (int c = 0; c < bits; ++c) {
+                            int wi, bi;
+                            code_bit(bits, j, h, c, wi, bi);
+                            w[wi] |= ((q >> c) & 1u) << bi;
+                        }
                     }
                 }
-                if (bits >= 2) memcpy(plane2 + 16 * lane, w2, 16);
-                if (bits != 2) memcpy(plane1 + 8 * lane, w1, 8);
+                for (int wi = 0; wi < 2 * bits; ++wi) memcpy(tile + code_word_off(bits, lane, wi), &w[wi], 4);
             }
             uint16_t *meta = (uint16_t *)(tile + tile_code_bytes(bits));
             for (int gi = 0; gi < gpt; ++gi) {
@@ -125,30 +120,22 @@ static void unpack_matrix(int m, int rows, int cols, int bits, int group, const 
         for (int kt = 0; kt < KT; ++kt) {
             const uint8_t *tile = src + tile_off(m, rb, kt, KT, nrb, bits, group);
             const int R0 = rb * kTileRows, K0 = kt * kTileK;
-            const uint8_t *plane2 = tile, *plane1 = tile + (bits >= 2 ? 512 : 0);
             for (int lane = 0; lane < 32; ++lane) {
-                uint32_t w2[4] = {0, 0, 0, 0}, w1[2] = {0, 0};
-                if (bits >= 2) memcpy(w2, plane2 + 16 * lane, 16);
-                if (bits != 2) memcpy(w1, plane1 + 8 * lane, 8);
+                uint32_t w[6] = {0, 0, 0, 0, 0, 0};
+                for (int wi = 0; wi < 2 * bits; ++wi) memcpy(&w[wi], tile + code_word_off(bits, lane, wi), 4);
                 for (int j = 0; j < 32; ++j) {
                     int row, col;
                     pair_pos(lane, j, row, col);
-                    uint32_t qa = 0, qb = 0;
-                    if (bits >= 2) {
-                        int p = j & 7;
-                        qa = (w2[j >> 3] >> (2 * p)) & 3u;
-                        qb = (w2[j >> 3] >> (16 + 2 * p)) & 3u;
-                    }
-                    if (bits != 2) {
-                        int p = j & 15;
-                        uint32_t ha = (w1[j >> 4] >> p) & 1u, hb = (w1[j >> 4] >> (16 + p)) & 1u;
-                        int sh = bits == 1 ? 0 : 2;
-                        qa |= ha << sh;
-                        qb |= hb << sh;
-                    }
                     uint8_t *d = codes + (size_t)(R0 + row) * cols + K0 + col;
-                    d[0] = (uint8_t)qa;
-                    d[1] = (uint8_t)qb;
+                    for (int h = 0; h < 2; ++h) {
+                        uint32_t q = 0;
+                        for (int c = 0; c < bits; ++c) {
+                            int wi, bi;
+                            code_bit(bits, j, h, c, wi, bi);
+                            q |= ((w[wi] >> bi) & 1u) << c;
+                        }
+                        d[h] = (uint8_t)q;
+                    }
                 }
             }
             const uint16_t *meta = (const uint16_t *)(tile + tile_code_bytes(bits));

@@ -29,9 +29,9 @@ constexpr int kTcProd = 12;                   // producer warp
 constexpr int kTcMma = 13;                    // MMA warp
 constexpr int kTcThreads = 14 * 32;
 constexpr int kTcMaxSlots = 16;
-constexpr int kTcNA = 3;                      // A atom buffers (32 KB each: low + high plane)
+constexpr int kTcNA = 3;                      // A atom buffers (16 KB each)
 constexpr int kTcND = 8;                      // TMEM accumulators of 16 columns
-constexpr int kABufBytes = 2 * 16384;
+constexpr int kABufBytes = 16384;
 constexpr int kSlotBImg = 0;                  // 4096 B
 constexpr int kSlotTab = 4096;                // <= 1024 B
 constexpr int kSlotPack = 5120;               // <= 7168 B
@@ -90,7 +90,7 @@ __device__ __forceinline__ void tc_tables(const __half *rows, int ntok, int grou
     const int gpt = kTileK / group;
     for (int item = warp; item < ntok * gpt; item += nwarps) {
         const int n = item / gpt, gi = item % gpt;
-        float tb[5] = {0, 0, 0, 0, 0};
+        float tb[7] = {0, 0, 0, 0, 0, 0, 0};
         for (int c = gi * group + lane; c < (gi + 1) * group; c += 32) {
             const float v = __half2float(rows[n * kTileK + c]);
             const int j0 = pair_of_col(c, 0), j1 = pair_of_col(c, 1);
@@ -99,15 +99,17 @@ __device__ __forceinline__ void tc_tables(const __half *rows, int ntok, int grou
             tb[2] = fmaf(off1(j1), v, tb[2]);
             tb[3] = fmaf(off2(j0), v, tb[3]);
             tb[4] = fmaf(off2(j1), v, tb[4]);
+            tb[5] = fmaf(off3(j0), v, tb[5]);
+            tb[6] = fmaf(off3(j1), v, tb[6]);
         }
 #pragma unroll
-        for (int k = 0; k < 5; ++k)
+        for (int k = 0; k < 7; ++k)
 #pragma unroll
             for (int m = 16; m >= 1; m >>= 1) tb[k] += __shfl_xor_sync(0xffffffffu, tb[k], m);
         if (lane == 0) {
             float4 *d = reinterpret_cast<float4 *>(dst + (size_t)item * kTabFloats);
             d[0] = make_float4(tb[0], 0.f, tb[1], tb[2]);
-            d[1] = make_float4(tb[3], tb[4], tb[3] + 4.f * tb[1], tb[4] + 4.f * tb[2]);
+            d[1] = make_float4(tb[3], tb[4], tb[5], tb[6]);
         }
     }
 }
@@ -234,20 +236,19 @@ __device__ __forceinline__ void tc_convert(const uint8_t *tile, int lane, int rb
     const int r0 = rbase + g8, r1 = r0 + 8;
 #pragma unroll
     for (int qd = 0; qd < 4; ++qd) {
-        uint32_t r[8], rh[8];
-        if (BITS == 1) cvt1_half<false>(c1[qd >> 1], 8 * (qd & 1), r);
-        if (BITS >= 2) cvt2(c2[qd], r);
-        if (BITS == 3) cvt1_half<true>(c1[qd >> 1], 8 * (qd & 1), rh);
+        uint32_t r[8];
+        if (BITS == 1) cvt1_half(c1[qd >> 1], 8 * (qd & 1), r);
+        if (BITS == 2) cvt2(c2[qd], r);
+        if (BITS == 3) {
+            const uint32_t w[6] = {c2[0], c2[1], c2[2], c2[3], c1[0], c1[1]};
+            cvt3(w, qd, r);
+        }
         uint8_t *ab = (qd >> 1) ? abuf1 : abuf0;
         const int chunk = 2 * t + (qd & 1);
         const uint32_t o0 = r0 * 128u + ((uint32_t)(chunk ^ (r0 & 7)) << 4);
         const uint32_t o1 = r1 * 128u + ((uint32_t)(chunk ^ (r1 & 7)) << 4);
         *reinterpret_cast<uint4 *>(ab + o0) = make_uint4(r[0], r[2], r[4], r[6]);
         *reinterpret_cast<uint4 *>(ab + o1) = make_uint4(r[1], r[3], r[5], r[7]);
-        if (BITS == 3) {
-            *reinterpret_cast<uint4 *>(ab + 16384 + o0) = make_uint4(rh[0], rh[2], rh[4], rh[6]);
-            *reinterpret_cast<uint4 *>(ab + 16384 + o1) = make_uint4(rh[1], rh[3], rh[5], rh[7]);
-        }
     }
 }
 
@@ -437,7 +438,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) tc_kernel(ExpertParams p)
                     for (int sub = 0; sub < 4; ++sub) {
                         const uint64_t bd = umma_desc_sw128(bimg + h * 2048 + sub * 32);
                         umma_f16(dt, umma_desc_sw128(ab + sub * 32), bd, idesc, !(first && sub == 0));
-                        if (bits == 3) umma_f16(dt, umma_desc_sw128(ab + 16384 + sub * 32), bd, idesc, true);
                     }
                     umma_commit(&sh->a_empty[ai]);
                     if (gpt == 2 || h == 1) umma_commit(&sh->d_full[ds]);
