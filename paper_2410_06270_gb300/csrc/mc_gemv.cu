@@ -12,13 +12,14 @@
 //     [vector blocks of n-tile 0][of n-tile 1]      one copy each
 //   The packed layout interleaves the two streams step by step (mc_layout.h), so
 //   a stage is a few large copies: small copies cap the streaming bandwidth well
-//   below the HBM peak.  Eight consumer warps each own one 16-row tile of BOTH
-//   streams (the B fragments and tables are loaded once for the two).  Code
+//   below the HBM peak.  Consumer warps own 16-row tiles: kTPW = 2 gives eight
+//   warps with tile tl of BOTH streams (the B fragments and tables are loaded
+//   once for the two), kTPW = 1 sixteen warps with one tile each.  Code
 //   words become fp16 mma.sync A fragments with one LOP3 per register
-//   (mc_layout.h), and every quantisation group is folded as
-//       y += s * (acc - O - z * X)
-//   where acc = sum_k (off_k + q_k) x_k, O = sum_k off_k x_k, X = sum_k x_k, i.e.
-//   y += s * sum_k (q_k - z) x_k, the group-wise dequantised product.
+//   (mc_layout.h), and every quantisation group is accumulated from
+//       acc = -(O + z X) + sum_k (off_k + q_k) x_k = sum_k (q_k - z) x_k
+//   (O = sum_k off_k x_k, X = sum_k x_k from the vector block's tables) and
+//   folded as y += s * acc, the group-wise dequantised product.
 //   W13: streams = W1 and W3 rows of a 128-row block; each warp forms
 //        h = silu(W1 x) * (W3 x) in registers and the CTA writes W2's vector
 //        blocks.
@@ -32,11 +33,18 @@
 
 namespace mc {
 
-constexpr int kCW = 8;                      // consumer warps (tile tl of both streams)
+#ifndef MC_GEMV_TPW
+#define MC_GEMV_TPW 1
+#endif
+constexpr int kTPW = MC_GEMV_TPW;            // 16-row tiles per consumer warp (1 or 2)
+constexpr int kCW = 16 / kTPW;              // consumer warps
 constexpr int kGemvThreads = (kCW + 1) * 32;
 constexpr int kMaxSlots = 16;
 constexpr int kRingOff = 1024;
-constexpr int kKPS = 2;                     // 128-column steps per ring stage
+#ifndef MC_GEMV_KPS
+#define MC_GEMV_KPS 2
+#endif
+constexpr int kKPS = MC_GEMV_KPS;           // 128-column steps per ring stage
 
 struct RingShared {
     uint64_t cbar;  // consumer-warp barrier of the W13 epilogue (bounded waits)
@@ -44,7 +52,9 @@ struct RingShared {
     volatile int issued;
     int slot_item[kMaxSlots];
     int slot_kc[kMaxSlots];  // column steps held by the stage (1..kKPS)
+    ChunkInfo slot_ci[kMaxSlots];  // the stage's chunk
 };
+static_assert(256 + sizeof(RingShared) <= 1024, "ring header");
 
 constexpr int kVecMax = kVecFragBytes + 8 * 2 * kTabFloats * 4;  // vec_bytes(64), the largest
 
@@ -52,11 +62,12 @@ __host__ __device__ inline int slot_bytes(int group)
 {
     return kKPS * 2 * supertile_bytes(3, group) + 2 * kKPS * kVecMax;
 }
-constexpr int kHsBytes = kChunk * kTileK * 2;  // h tile [16][128] fp16 (two of them)
+constexpr int kHsBytes = kChunk * kTileK * 2;           // h tile [16][128] fp16 (two of them)
+constexpr int kXbufBytes = kTPW == 1 ? 8 * 32 * 8 * 4 : 0;  // W3 results handed to the W1 warps
 
 __host__ __device__ inline size_t gemv_smem(int nslots, int group)
 {
-    return kRingOff + (size_t)nslots * slot_bytes(group) + 2 * kHsBytes;
+    return kRingOff + (size_t)nslots * slot_bytes(group) + 2 * kHsBytes + kXbufBytes + 8 * 32 * sizeof(uint2);
 }
 
 // Bounded wait that gives up as soon as another thread of the CTA aborted.
@@ -88,7 +99,47 @@ __device__ __forceinline__ bool header_ok(const ExpertParams &p, int e)
            hd->mat_off[e][2] == p.mat_off[e][2];
 }
 
-// Vector block of n-tile j built from a [16][128] fp16 tile in shared memory:
+// D += A * B, m16n8k16, fp16 inputs, fp32 accumulate (not volatile, so the
+// compiler may schedule it).
+__device__ __forceinline__ void mma_acc(float (&d)[4], const uint32_t *a, uint32_t b0, uint32_t b1)
+{
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// Offset tables as a matrix product.  For pairs n of a vector block and one
+// quantisation group, the table slots are
+//     T[r][n] = sum_c M[r][c] x_n[c],   r = 0..7,
+// with the rows of M the coefficients of the table layout below: off2(half 0),
+// off2(half 1), 1, off1(half 0), off3(half 0), off3(half 1), 1, off1(half 1)
+// (off_b(half) of column c = the b-bit field offset of the pair holding column
+// c in that row half, mc_layout.h).  M is a constant fp16 matrix (powers of
+// two), so one m16n8k16 mma per k-step forms the tables of eight pairs, with
+// the B fragments of the main product.  tab_afrag[s][lane] holds the A
+// fragment registers a0, a2 of k-step s (rows 8..15 of M are zero).
+__device__ __forceinline__ float tab_coef(int r, int col)
+{
+    const int jp = pair_of_col(col, (r == 1 || r == 5 || r == 7) ? 1 : 0);
+    if (r == 2 || r == 6) return 1.f;
+    if (r == 0 || r == 1) return off2(jp);
+    if (r == 3 || r == 7) return off1(jp);
+    return off3(jp);
+}
+
+__device__ __forceinline__ void build_tab_afrag(uint2 *afr, int tid, int nthreads)
+{
+    for (int idx = tid; idx < 8 * 32; idx += nthreads) {
+        const int s = idx >> 5, lane = idx & 31, g8 = lane >> 2, t = lane & 3;
+        const int col0 = 64 * (s >> 2) + 16 * t + 4 * (s & 3);
+        const __half2 lo = __floats2half2_rn(tab_coef(g8, col0), tab_coef(g8, col0 + 1));
+        const __half2 hi = __floats2half2_rn(tab_coef(g8, col0 + 2), tab_coef(g8, col0 + 3));
+        afr[idx] = make_uint2(*reinterpret_cast<const uint32_t *>(&lo), *reinterpret_cast<const uint32_t *>(&hi));
+    }
+}
+
+// Vector blocks (n-tiles j < NT) built from a [16][128] fp16 tile in shared
+// memory; block j at dst + j * jstride:
 //   fragments, 256 entries of 8 bytes ordered [s/2][lane][s%2] (one 16-byte load
 //     gives a lane its B fragments of k-steps 2q and 2q+1); an entry holds the
 //     4 fp16 values at columns 64(s/4) + 16t + 4(s%4) .. +3 of pair 8j + lane/4;
@@ -97,40 +148,33 @@ __device__ __forceinline__ bool header_ok(const ExpertParams &p, int e)
 //   (X = sum of the group's inputs, O_b = sum of the b-bit field offsets times
 //   the inputs for the rows of one half; mc_layout.h), so that a 2- or 3-bit
 //   fold reads its O pair and X with one 16-byte load.
-// Threads share the fragment entries; one warp per table item.
-__device__ __forceinline__ void write_vec_block(const __half *rows, int j, int group, uint8_t *dst, int tid,
-                                                int nthreads, int warp, int nwarps, int lane)
+// All threads copy fragment entries; warp j forms block j's tables.
+__device__ __forceinline__ void write_vec_blocks(const __half *rows, int NT, int group, uint8_t *dst, size_t jstride,
+                                                 const uint2 *afr, int tid, int nthreads)
 {
-    for (int idx = tid; idx < 256; idx += nthreads) {
-        const int s = 2 * ((idx >> 6) & 3) + (idx & 1), ln = (idx >> 1) & 31;
+    for (int idx = tid; idx < NT * 256; idx += nthreads) {
+        const int j = idx >> 8, s = 2 * ((idx >> 6) & 3) + (idx & 1), ln = (idx >> 1) & 31;
         const int n = 8 * j + (ln >> 2), t = ln & 3;
         const int col = 64 * (s >> 2) + 16 * t + 4 * (s & 3);
-        reinterpret_cast<uint2 *>(dst)[idx] = *reinterpret_cast<const uint2 *>(rows + n * kTileK + col);
+        reinterpret_cast<uint2 *>(dst + j * jstride)[idx & 255] =
+            *reinterpret_cast<const uint2 *>(rows + n * kTileK + col);
     }
-    const int gpt = kTileK / group;
-    float *tab = reinterpret_cast<float *>(dst + kVecFragBytes);
-    for (int item = warp; item < 8 * gpt; item += nwarps) {
-        const int nl = item / gpt, gi = item % gpt, n = 8 * j + nl;
-        float tb[7] = {0, 0, 0, 0, 0, 0, 0};
-        for (int c = gi * group + lane; c < (gi + 1) * group; c += 32) {
-            const float v = __half2float(rows[n * kTileK + c]);
-            const int j0 = pair_of_col(c, 0), j1 = pair_of_col(c, 1);
-            tb[0] += v;
-            tb[1] = fmaf(off1(j0), v, tb[1]);
-            tb[2] = fmaf(off1(j1), v, tb[2]);
-            tb[3] = fmaf(off2(j0), v, tb[3]);
-            tb[4] = fmaf(off2(j1), v, tb[4]);
-            tb[5] = fmaf(off3(j0), v, tb[5]);
-            tb[6] = fmaf(off3(j1), v, tb[6]);
+    const int warp = tid >> 5, lane = tid & 31;
+    if (warp < NT) {
+        const int j = warp, g8 = lane >> 2, t = lane & 3, gpt = kTileK / group;
+        float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+#pragma unroll
+        for (int s = 0; s < 8; ++s) {
+            const int col0 = 64 * (s >> 2) + 16 * t + 4 * (s & 3);
+            const uint2 b = *reinterpret_cast<const uint2 *>(rows + (8 * j + g8) * kTileK + col0);
+            const uint2 a = afr[s * 32 + lane];
+            const uint32_t af[4] = {a.x, 0u, a.y, 0u};
+            mma_acc(acc[gpt == 2 ? (s >> 2) : 0], af, b.x, b.y);
         }
-#pragma unroll
-        for (int k = 0; k < 7; ++k)
-#pragma unroll
-            for (int m = 16; m >= 1; m >>= 1) tb[k] += __shfl_xor_sync(0xffffffffu, tb[k], m);
-        if (lane == 0) {
-            float4 *d = reinterpret_cast<float4 *>(tab + (size_t)item * kTabFloats);
-            d[0] = make_float4(tb[3], tb[4], tb[0], tb[1]);
-            d[1] = make_float4(tb[5], tb[6], tb[0], tb[2]);
+        float *tab = reinterpret_cast<float *>(dst + j * jstride + kVecFragBytes);
+        for (int gi = 0; gi < gpt; ++gi) {
+            tab[((2 * t) * gpt + gi) * kTabFloats + g8] = acc[gi][0];
+            tab[((2 * t + 1) * gpt + gi) * kTabFloats + g8] = acc[gi][1];
         }
     }
 }
@@ -139,8 +183,10 @@ __device__ __forceinline__ void write_vec_block(const __half *rows, int j, int g
 __global__ void __launch_bounds__(256) frag_x_kernel(ExpertParams p)
 {
     __shared__ __align__(16) __half xs[kChunk * kTileK];
+    __shared__ uint2 afr[8 * 32];
     const int k = blockIdx.x, kt = blockIdx.y, KT = p.H / kTileK;
     if (k >= *p.nchunks) return;
+    build_tab_afrag(afr, threadIdx.x, 256);
     const ChunkInfo ci = p.chunks[k];
     const int NT = ci.nv > 8 ? 2 : 1;
     const int tid = threadIdx.x;
@@ -164,27 +210,11 @@ __global__ void __launch_bounds__(256) frag_x_kernel(ExpertParams p)
         *reinterpret_cast<uint4 *>(xs + n * kTileK + c8) = out;
     }
     __syncthreads();
-    for (int j = 0; j < NT; ++j)
-        write_vec_block(xs, j, p.group, p.xvec + vec_off(k, j, kt, KT, p.group), tid, 256, tid >> 5, 8, tid & 31);
+    write_vec_blocks(xs, NT, p.group, p.xvec + vec_off(k, 0, kt, KT, p.group),
+                     vec_off(0, 1, 0, KT, p.group), afr, tid, 256);
 }
 
 // --------------------------------------------------------------- one step --
-
-// D = A * B (+ C), m16n8k16, fp16 inputs, fp32 accumulate; ZERO: C = 0.
-template <bool ZERO>
-__device__ __forceinline__ void mma_acc(float (&d)[4], const uint32_t *a, uint32_t b0, uint32_t b1)
-{
-    if (ZERO)
-        asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-            "{%10,%10,%10,%10};"
-            : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
-            : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(0.f));
-    else
-        asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-            "{%0,%1,%2,%3};"
-            : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-            : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
 
 // The code words and fp16 (scale, zero) pairs one lane needs from a tile.
 template <int BITS, int GPT>
@@ -221,59 +251,33 @@ __device__ __forceinline__ void decode_qd(const TileRegs<BITS, GPT> &t, int qd, 
     }
 }
 
-// y += s * (acc0 + acc1 - O - z X) for the lane's four C-fragment entries:
-// entries 0/1 are row g8 with pairs 2t / 2t+1, entries 2/3 row g8+8.
-__device__ __forceinline__ void fold(float (&y)[4], const float (&a0)[4], const float (&a1)[4], uint2 meta,
-                                     float2 O0, float2 O1, float X0, float X1)
-{
-    const __half2 *m2 = reinterpret_cast<const __half2 *>(&meta);
-    const float2 sz0 = __half22float2(m2[0]), sz1 = __half22float2(m2[1]);
-    y[0] = fmaf(sz0.x, a0[0] + a1[0] - O0.x - sz0.y * X0, y[0]);
-    y[1] = fmaf(sz0.x, a0[1] + a1[1] - O1.x - sz0.y * X1, y[1]);
-    y[2] = fmaf(sz1.x, a0[2] + a1[2] - O0.y - sz1.y * X0, y[2]);
-    y[3] = fmaf(sz1.x, a0[3] + a1[3] - O1.y - sz1.y * X1, y[3]);
-}
-
-// One consumer warp, one 128-column step of its 16-row tile in both streams:
-// decode, mma and fold.  y*[j][c]: C-fragment layout, rows g8 / g8+8 of the
-// tile, pairs 8j + 2t + {0,1}.  vec0 / vec1: the step's vector blocks of
-// n-tiles 0 / 1.  Two accumulators per tile and n-tile (by k-step parity) keep
-// the dependent mma chains short.
-template <int NT, int BITS, int GPT>
-__device__ __forceinline__ void step2(const uint8_t *tA, const uint8_t *tB, const uint8_t *vec0, const uint8_t *vec1,
-                                      int lane, float (&yA)[NT][4], float (&yB)[NT][4])
+// One consumer warp, one 128-column step of its NTL 16-row tiles: decode, mma
+// and fold.  y[u][j][c]: tile u, C-fragment layout (rows g8 / g8+8 of the tile,
+// pairs 8j + 2t + {0,1}).  vec0 / vec1: the step's vector blocks of n-tiles
+// 0 / 1, shared by the tiles.  Each group's accumulator starts at
+// -(O + z X), so after the group's mma chain it holds sum_k (q_k - z) x_k and
+// the fold is a single y += s * acc.
+template <int NT, int BITS, int GPT, int NTL>
+__device__ __forceinline__ void step_tiles(const uint8_t *const (&tile)[NTL], const uint8_t *vec0,
+                                           const uint8_t *vec1, int lane, float (&y)[NTL][NT][4])
 {
     constexpr int SPG = 8 / GPT;  // k-steps per quantisation group
-    TileRegs<BITS, GPT> RA, RB;
-    load_tile<BITS, GPT>(tA, lane, RA);
-    load_tile<BITS, GPT>(tB, lane, RB);
-    float accA[2][NT][4], accB[2][NT][4];
+    TileRegs<BITS, GPT> R[NTL];
+#pragma unroll
+    for (int u = 0; u < NTL; ++u) load_tile<BITS, GPT>(tile[u], lane, R[u]);
+    float acc[NTL][NT][4];
 #pragma unroll
     for (int qd = 0; qd < 4; ++qd) {
-        uint32_t ra[8], rb[8];
-        decode_qd<BITS, GPT>(RA, qd, ra);
-        decode_qd<BITS, GPT>(RB, qd, rb);
+        uint32_t r[NTL][8];
+#pragma unroll
+        for (int u = 0; u < NTL; ++u) decode_qd<BITS, GPT>(R[u], qd, r[u]);
         uint4 bq[NT];
 #pragma unroll
         for (int j = 0; j < NT; ++j) bq[j] = reinterpret_cast<const uint4 *>(j ? vec1 : vec0)[qd * 32 + lane];
 #pragma unroll
         for (int kk = 0; kk < 2; ++kk) {
-            const int s = 2 * qd + kk;
-            // the first k-step of a group in each parity chain starts from zero
-            const bool first = s % SPG < 2;
-#pragma unroll
-            for (int j = 0; j < NT; ++j) {
-                const uint32_t b0 = kk ? bq[j].z : bq[j].x, b1 = kk ? bq[j].w : bq[j].y;
-                if (first) {
-                    mma_acc<true>(accA[kk][j], ra + 4 * kk, b0, b1);
-                    mma_acc<true>(accB[kk][j], rb + 4 * kk, b0, b1);
-                } else {
-                    mma_acc<false>(accA[kk][j], ra + 4 * kk, b0, b1);
-                    mma_acc<false>(accB[kk][j], rb + 4 * kk, b0, b1);
-                }
-            }
-            if (s % SPG == SPG - 1) {
-                const int gi = s / SPG;
+            const int s = 2 * qd + kk, gi = s / SPG;
+            if (s % SPG == 0) {
 #pragma unroll
                 for (int j = 0; j < NT; ++j) {
                     const float *T0 = reinterpret_cast<const float *>((j ? vec1 : vec0) + kVecFragBytes) +
@@ -296,8 +300,35 @@ __device__ __forceinline__ void step2(const uint8_t *tA, const uint8_t *tB, cons
                         X0 = u0.z;
                         X1 = u1.z;
                     }
-                    fold(yA[j], accA[0][j], accA[1][j], RA.meta[gi], O0, O1, X0, X1);
-                    fold(yB[j], accB[0][j], accB[1][j], RB.meta[gi], O0, O1, X0, X1);
+#pragma unroll
+                    for (int u = 0; u < NTL; ++u) {
+                        const __half2 *m2 = reinterpret_cast<const __half2 *>(&R[u].meta[gi]);
+                        const float z0 = __high2float(m2[0]), z1 = __high2float(m2[1]);
+                        acc[u][j][0] = fmaf(-z0, X0, -O0.x);
+                        acc[u][j][1] = fmaf(-z0, X1, -O1.x);
+                        acc[u][j][2] = fmaf(-z1, X0, -O0.y);
+                        acc[u][j][3] = fmaf(-z1, X1, -O1.y);
+                    }
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < NT; ++j) {
+                const uint32_t b0 = kk ? bq[j].z : bq[j].x, b1 = kk ? bq[j].w : bq[j].y;
+#pragma unroll
+                for (int u = 0; u < NTL; ++u) mma_acc(acc[u][j], r[u] + 4 * kk, b0, b1);
+            }
+            if (s % SPG == SPG - 1) {
+#pragma unroll
+                for (int u = 0; u < NTL; ++u) {
+                    const __half2 *m2 = reinterpret_cast<const __half2 *>(&R[u].meta[gi]);
+                    const float s0 = __low2float(m2[0]), s1 = __low2float(m2[1]);
+#pragma unroll
+                    for (int j = 0; j < NT; ++j) {
+                        y[u][j][0] = fmaf(s0, acc[u][j][0], y[u][j][0]);
+                        y[u][j][1] = fmaf(s0, acc[u][j][1], y[u][j][1]);
+                        y[u][j][2] = fmaf(s1, acc[u][j][2], y[u][j][2]);
+                        y[u][j][3] = fmaf(s1, acc[u][j][3], y[u][j][3]);
+                    }
                 }
             }
         }
@@ -312,12 +343,12 @@ struct Item {
 };
 
 template <bool W13>
-__device__ __forceinline__ Item decode_item(const ExpertParams &p, int item, int U)
+__device__ __forceinline__ Item decode_item(const ExpertParams &p, int item, int U, const ChunkInfo &ci)
 {
     Item it;
     it.k = item / U;
     it.u = item % U;
-    it.ci = p.chunks[it.k];
+    it.ci = ci;
     if (W13) {
         it.blkA = it.blkB = it.u;
         it.kt0 = 0;
@@ -340,29 +371,47 @@ struct Ring {
     uint64_t *full, *empty;
     const uint8_t *base;
     int S, SB, vec_off0, VB;
+    const uint2 *afr;  // A fragments of the table matrix
 };
 
-// One work item for one consumer warp (tile tl of both streams): all its
-// stages, then the epilogue.  The first stage's full barrier has already been
-// waited for; the ring position (slot, phase) advances by one per stage.
-//   W13: h = silu(W1 x) * (W3 x) for the warp's 16 rows goes to the h tile
-//        (double-buffered by item parity), the consumer warps meet once, and
-//        together write W2's vector blocks of this 128-row block.
-//   W2:  fp32 outputs of the split, rows of both blocks.
+// All consumer warps meet at the CTA's consumer barrier (bounded); false once
+// the CTA aborted.
+__device__ __forceinline__ bool consumer_sync(const ExpertParams &p, RingShared *sh, int lane, int &uses)
+{
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sh->cbar);
+    return wait_or_abort(&sh->cbar, (uses++) & 1, p, sh);
+}
+
+// One work item for one consumer warp: all its stages, then the epilogue.  The
+// first stage's full barrier has already been waited for; the ring position
+// (slot, phase) advances by one per stage.
+//   kTPW = 2: the warp owns tile tl of both streams.
+//   kTPW = 1: the warp owns tile tl of stream x.
+//   W13: h = silu(W1 x) * (W3 x) for the item's rows goes to the h tile
+//        (double-buffered by item parity; with one tile per warp the W3 results
+//        pass through xbuf first), then the consumer warps together write W2's
+//        vector blocks of this 128-row block.
+//   W2:  fp32 outputs of the split.
 template <bool W13, int NT, int BITS, int GPT>
 __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, const Ring &R, const Item &I, int nrb,
-                                      int tl, int lane, int &slot, uint32_t &phase, __half *hs2, int &items)
+                                         int x, int tl, int lane, int &slot, uint32_t &phase, float *xbuf,
+                                         __half *hs2, int &items, int &cbar_uses)
 {
     constexpr int group = kTileK / GPT;
     const int STB = supertile_bytes(BITS, group), TB = tile_bytes(BITS, group);
     const int pw = W13 ? 2 : w2_pair_width(I.blkA >> 1, nrb);
     const int step_bytes = pw * STB;
-    const int offA = tl * TB, offB = (pw == 2 ? STB : 0) + tl * TB;  // lone W2 block: stream B repeats A
-    float yA[NT][4], yB[NT][4];
+    // a lone W2 block (odd row-block count): stream B repeats stream A, unused
+    const int offB = (pw == 2 ? STB : 0) + tl * TB;
+    const int off[2] = {kTPW == 2 ? tl * TB : (x ? offB : tl * TB), offB};
+    float y[kTPW][NT][4];
 #pragma unroll
-    for (int j = 0; j < NT; ++j)
+    for (int u = 0; u < kTPW; ++u)
 #pragma unroll
-        for (int c = 0; c < 4; ++c) yA[j][c] = yB[j][c] = 0.f;
+        for (int j = 0; j < NT; ++j)
+#pragma unroll
+            for (int c = 0; c < 4; ++c) y[u][j][c] = 0.f;
     for (int i = 0; i < I.nkt; i += kKPS) {
         if (i > 0 && !wait_or_abort(&R.full[slot], phase, p, sh)) return false;
         const uint8_t *base = R.base + (size_t)slot * R.SB;
@@ -370,9 +419,13 @@ __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, 
         const uint8_t *v0 = base + R.vec_off0, *v1 = v0 + kKPS * R.VB;
 #pragma unroll
         for (int kk = 0; kk < kKPS; ++kk)
-            if (kk < kc)
-                step2<NT, BITS, GPT>(base + kk * step_bytes + offA, base + kk * step_bytes + offB, v0 + kk * R.VB,
-                                     v1 + kk * R.VB, lane, yA, yB);
+            if (kk < kc) {
+                const uint8_t *st = base + kk * step_bytes;
+                const uint8_t *t[kTPW];
+#pragma unroll
+                for (int u = 0; u < kTPW; ++u) t[u] = st + off[u];
+                step_tiles<NT, BITS, GPT, kTPW>(t, v0 + kk * R.VB, v1 + kk * R.VB, lane, y);
+            }
         __syncwarp();
         if (lane == 0) mbar_arrive(&R.empty[slot]);
         if (++slot == R.S) {
@@ -383,26 +436,42 @@ __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, 
     const int g8 = lane >> 2, t2 = 2 * (lane & 3);
     if (W13) {
         __half *hs = hs2 + (items & 1) * (kChunk * kTileK);
-#pragma unroll
-        for (int j = 0; j < NT; ++j)
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                const int n = 8 * j + t2 + (c & 1);
-                const int r = tl * 16 + g8 + 8 * (c >> 1);
-                const float hv = n < I.ci.nv ? silu(yA[j][c]) * yB[j][c] : 0.f;
-                hs[n * kTileK + r] = __float2half_rn(hv);
-            }
-        // every warp finished the previous item's vector blocks before it got here,
-        // so after this barrier the other h buffer is free again
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sh->cbar);
-        if (!wait_or_abort(&sh->cbar, items & 1, p, sh)) return false;
         ++items;
+        float u[NT][4];
+        if (kTPW == 2) {
+#pragma unroll
+            for (int j = 0; j < NT; ++j)
+#pragma unroll
+                for (int c = 0; c < 4; ++c) u[j][c] = y[kTPW - 1][j][c];
+        } else {
+            float4 *xb = reinterpret_cast<float4 *>(xbuf + (tl * 32 + lane) * 8);
+            if (x == 1)
+#pragma unroll
+                for (int j = 0; j < NT; ++j) xb[j] = make_float4(y[0][j][0], y[0][j][1], y[0][j][2], y[0][j][3]);
+            if (!consumer_sync(p, sh, lane, cbar_uses)) return false;
+#pragma unroll
+            for (int j = 0; j < NT; ++j) {
+                const float4 v = xb[j];
+                u[j][0] = v.x; u[j][1] = v.y; u[j][2] = v.z; u[j][3] = v.w;
+            }
+        }
+        if (kTPW == 2 || x == 0)
+#pragma unroll
+            for (int j = 0; j < NT; ++j)
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    const int n = 8 * j + t2 + (c & 1);
+                    const int r = tl * 16 + g8 + 8 * (c >> 1);
+                    const float hv = n < I.ci.nv ? silu(y[0][j][c]) * u[j][c] : 0.f;
+                    hs[n * kTileK + r] = __float2half_rn(hv);
+                }
+        // every warp finished the previous item's vector blocks before it got
+        // here, so after this barrier the other h buffer is free again
+        if (!consumer_sync(p, sh, lane, cbar_uses)) return false;
         // the item's 128 rows are W2's column step I.u
         const int KT2 = p.F / kTileK;
-        for (int j = 0; j < NT; ++j)
-            write_vec_block(hs, j, group, p.hvec + vec_off(I.k, j, I.u, KT2, group), threadIdx.x, kCW * 32, tl,
-                            kCW, lane);
+        write_vec_blocks(hs, NT, group, p.hvec + vec_off(I.k, 0, I.u, KT2, group), vec_off(0, 1, 0, KT2, group),
+                         R.afr, threadIdx.x, kCW * 32);
     } else {
         float *out = p.opart + (size_t)I.ks * p.Pmax * p.H;
 #pragma unroll
@@ -413,8 +482,12 @@ __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, 
                 const int r = tl * 16 + g8 + 8 * (c >> 1);
                 if (n < I.ci.nv) {
                     float *o = out + (size_t)(I.ci.pair_base + n) * p.H;
-                    o[I.blkA * kBlockRows + r] = yA[j][c];
-                    if (I.blkB >= 0) o[I.blkB * kBlockRows + r] = yB[j][c];
+                    if (kTPW == 2) {
+                        o[I.blkA * kBlockRows + r] = y[0][j][c];
+                        if (I.blkB >= 0) o[I.blkB * kBlockRows + r] = y[kTPW - 1][j][c];
+                    } else if (x == 0 || I.blkB >= 0) {
+                        o[(x ? I.blkB : I.blkA) * kBlockRows + r] = y[0][j][c];
+                    }
                 }
             }
     }
@@ -433,6 +506,8 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
     const int SB = slot_bytes(group), VB = vec_bytes(group);
     const int vec_off0 = kKPS * 2 * supertile_bytes(3, group);
     __half *hs2 = reinterpret_cast<__half *>(smem + kRingOff + (size_t)S * SB);
+    float *xbuf = reinterpret_cast<float *>(smem + kRingOff + (size_t)S * SB + 2 * kHsBytes);
+    uint2 *afr = reinterpret_cast<uint2 *>(smem + kRingOff + (size_t)S * SB + 2 * kHsBytes + kXbufBytes);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nrb = W13 ? p.F / kBlockRows : p.H / kBlockRows;  // 128-row blocks of the matrix
     const int U = W13 ? nrb : ((nrb + 1) / 2) * p.KS;
@@ -449,6 +524,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
         sh->issued = 0;
         fence_mbar_init();
     }
+    if (W13) build_tab_afrag(afr, threadIdx.x, kGemvThreads);
     __syncthreads();
 
     if (warp == kCW) {
@@ -463,7 +539,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
             while (ok) {
                 const int item = atomicAdd(&p.counters[W13 ? 0 : 1], 1);
                 if (item >= total) break;
-                const Item I = decode_item<W13>(p, item, U);
+                const Item I = decode_item<W13>(p, item, U, p.chunks[item / U]);
                 const int e = I.ci.e, bits = I.ci.bits, NT = I.ci.nv > 8 ? 2 : 1;
                 if (!((verified >> e) & 1u)) {
                     if (!header_ok(p, e)) {
@@ -491,6 +567,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
                     }
                     const int kc = min(kKPS, I.nkt - i);
                     sh->slot_item[slot] = item;
+                    sh->slot_ci[slot] = I.ci;
                     sh->slot_kc[slot] = kc;
                     uint8_t *dst = ring + (size_t)slot * SB;
                     const uint32_t wb = (uint32_t)(kc * pw * STB), vb = (uint32_t)(kc * VB);
@@ -513,17 +590,19 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
         }
     } else {
         // --------------------------------------------------------- consumers --
-        const Ring R{full, empty, ring, S, SB, vec_off0, VB};
-        int slot = 0, items = 0;
+        const Ring R{full, empty, ring, S, SB, vec_off0, VB, afr};
+        const int x = kTPW == 2 ? 0 : warp >> 3, tl = warp & 7;
+        int slot = 0, items = 0, cbar_uses = 0;
         uint32_t phase = 0;
         while (true) {
             if (!wait_or_abort(&full[slot], phase, p, sh)) break;
             const int item = sh->slot_item[slot];
             if (item < 0) break;
-            const Item I = decode_item<W13>(p, item, U);
+            const Item I = decode_item<W13>(p, item, U, sh->slot_ci[slot]);
             const int sel = (I.ci.bits - 1) * 2 + (I.ci.nv > 8 ? 1 : 0);
             bool ok;
-#define MC_RUN(NT_, B_) run_item<W13, NT_, B_, GPT>(p, sh, R, I, nrb, warp, lane, slot, phase, hs2, items)
+#define MC_RUN(NT_, B_) \
+    run_item<W13, NT_, B_, GPT>(p, sh, R, I, nrb, x, tl, lane, slot, phase, xbuf, hs2, items, cbar_uses)
             switch (sel) {
             case 0: ok = MC_RUN(1, 1); break;
             case 1: ok = MC_RUN(2, 1); break;
