@@ -159,6 +159,33 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
                    int32_t *topk_idx_out, float *topk_w_out, uint8_t *pruned_out,
                    void *stream);
 
+/* mc_moe_forward without a workspace: the same layer (routing, ODP, experts on
+ * the mma.sync path, combine), with its scratch in a fixed 16 MiB device array
+ * that belongs to the library (one per device).  The paper has no counterpart;
+ * this entry point exists for callers that must not allocate device memory once
+ * they are running: a serving loop that freezes its memory plan at start-up, a
+ * plug-in whose device memory belongs to a host framework, a plain C caller
+ * with no device allocator of its own.  It allocates nothing.
+ *   Arguments as mc_moe_forward; no workspace and no routing outputs.
+ *   status_dev: optional device int32; when given, device-side errors
+ *     (MC_ERR_TIMEOUT, MC_ERR_BAD_PACK, MC_ERR_RANGE) are recorded there and it
+ *     must hold 0 when the call starts.  When NULL, they go to a status word in
+ *     the scratch, which each call clears (cudaMemsetAsync on `stream`) before
+ *     its kernels and which the caller cannot read.  No other byte of the
+ *     scratch needs an initial value.
+ *   Limit: the scratch must hold the call's buffers; a (shape, T) that needs
+ *     more than 16 MiB returns MC_ERR_INVALID_ARG with the size in the message
+ *     (at the Mixtral-8x7b shape, H 4096, F 14336, group 128, that is T > 52).
+ *   Set-up: the first call on a device, made with that device current, looks up
+ *     the scratch's address once (cudaGetSymbolAddress); make that first call
+ *     before any stream capture.
+ *   Concurrency: every call on a device uses the same scratch, so calls whose
+ *     kernels may overlap (other streams, other host threads) race and corrupt
+ *     each other's results; order them (one stream, or events). */
+int mc_moe_forward_static(const void *x, const void *gate_w, int T, const mc_shape *shape,
+                          const int8_t *bits_host, const void *packed_dev, float mu,
+                          const uint8_t *protect, void *y, int32_t *status_dev, void *stream);
+
 /* Choose the expert path of mc_moe_forward: 0 = automatic, 1 = the mma.sync
  * grouped GEMV (small batches), 2 = the tcgen05 tensor-memory kernels.
  * Process-wide; returns the previous value. */

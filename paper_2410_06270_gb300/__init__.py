@@ -62,6 +62,7 @@ def load():
         "mc_route": (I, [P, P, I, S, F32, P, P, P, P, P, P, P]),
         "mc_moe_workspace_size": (Z, [S, I]),
         "mc_moe_forward": (I, [P, P, I, S, P, P, F32, P, P, P, Z, P, P, P, P]),
+        "mc_moe_forward_static": (I, [P, P, I, S, P, P, F32, P, P, P, P]),
         "mc_set_path": (I, [I]),
         "mc_set_debug": (I, [I, ctypes.c_ulonglong]),
         "mc_check_status": (I, [P, P]),
@@ -257,6 +258,23 @@ def moe_forward(x, gate_w, shape: Shape, bits, packed_dev, mu: float = 0.0, prot
                                  _ptr(idx), _ptr(w), _ptr(pr), _stream()))
     if routing:
         return y, {"idx": idx, "w": w, "pruned": pr}
+    return y
+
+
+def moe_forward_static(x, gate_w, shape: Shape, bits, packed_dev, mu: float = 0.0, protect=None, y=None,
+                       status=None):
+    """mc_moe_forward_static: the layer with the library's fixed device scratch
+    instead of a workspace.  `y` (bf16 [T,H]) and `status` (device int32, zeroed by
+    the caller; None = the scratch's own status word) must already exist when the
+    caller may not allocate."""
+    import torch
+    T = x.shape[0]
+    if y is None:
+        y = torch.empty_like(x)
+    b = _bits(bits)
+    _check(load().mc_moe_forward_static(_ptr(x), _ptr(gate_w), T, ctypes.byref(shape), b.ctypes.data,
+                                        _ptr(packed_dev), float(mu), _ptr(protect), _ptr(y), _ptr(status),
+                                        _stream()))
     return y
 
 
