@@ -186,8 +186,10 @@ int mc_moe_forward_static(const void *x, const void *gate_w, int T, const mc_sha
                           const int8_t *bits_host, const void *packed_dev, float mu,
                           const uint8_t *protect, void *y, int32_t *status_dev, void *stream);
 
-/* Choose the expert path of mc_moe_forward: 0 = automatic, 1 = the mma.sync
- * grouped GEMV (small batches), 2 = the tcgen05 tensor-memory kernels.
+/* Choose the expert path of mc_moe_forward: 0 = automatic (the GEMV below 512
+ * kept-or-not pairs, 2T < 512, else the GEMM), 1 = the mma.sync grouped GEMV
+ * (decode), 2 = the tcgen05 grouped GEMV with chunks of 16 pairs, 3 = the
+ * tcgen05 grouped GEMM with token blocks of 128 pairs (prefill).
  * Process-wide; returns the previous value. */
 int mc_set_path(int path);
 

@@ -14,6 +14,8 @@
 namespace mc {
 
 static std::atomic<int> g_path{0};
+// pairs (2 T) from which mc_moe_forward's automatic choice is the prefill GEMM
+constexpr int kPrefillPairs = 512;
 static std::atomic<int> g_debug{0};
 static std::atomic<unsigned long long> g_timeout_ns{1000000000ull};  // 1 s
 static uint64_t *g_trace = nullptr;
@@ -51,8 +53,9 @@ struct Workspace {
     float *htab;
     float *gu;
     uint8_t *xvec, *hvec;
+    uint8_t *ximg, *himg;
     float *opart;
-    int max_chunks, KS;
+    int max_chunks, max_blocks, KS;
     size_t total;
 };
 
@@ -87,6 +90,9 @@ static Workspace carve(const mc_shape *s, int T, void *base)
     w.gu = (float *)take(MC * 2 * (size_t)s->F * kChunk * 4);
     w.xvec = (uint8_t *)take(MC * 2 * (s->H / kTileK) * (size_t)vec_bytes(s->group));
     w.hvec = (uint8_t *)take(MC * 2 * (s->F / kTileK) * (size_t)vec_bytes(s->group));
+    w.max_blocks = max_blocks_for(T, s->E);
+    w.ximg = (uint8_t *)take(img_buffer_bytes(w.max_blocks, s->H));
+    w.himg = (uint8_t *)take(img_buffer_bytes(w.max_blocks, s->F));
     w.opart = (float *)take((size_t)w.KS * P * s->H * 4);
     w.total = off;
     return w;
@@ -174,6 +180,7 @@ int mc_route(const void *x, const void *gate_w, int T, const mc_shape *shape, fl
     pp.E = shape->E;
     pp.offsets = expert_offsets;
     pp.perm = perm;
+    pp.chunk = kChunk;
     return launch_route(rp, pp, (cudaStream_t)stream);
 }
 
@@ -196,6 +203,10 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     if (ws_bytes < ws.total)
         return set_error(MC_ERR_INVALID_ARG, "workspace has %zu bytes, needs %zu", ws_bytes, ws.total);
     cudaStream_t st = (cudaStream_t)stream;
+    // expert path: many pairs per expert -> tensor-core grouped GEMM (prefill),
+    // few -> mma.sync grouped GEMV (decode); mc_set_path overrides
+    int path = g_path;
+    if (path == 0) path = 2 * T >= kPrefillPairs ? 3 : 1;
 
     RouteParams rp;
     memset(&rp, 0, sizeof rp);
@@ -225,6 +236,7 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     pp.chunks = ws.chunks;
     pp.nchunks = ws.nchunks;
     pp.counters = ws.counters;
+    pp.chunk = path == 3 ? 128 : kChunk;
     rc = launch_route(rp, pp, st);
     if (rc) return rc;
 
@@ -250,8 +262,11 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     ep.gu = ws.gu;
     ep.xvec = ws.xvec;
     ep.hvec = ws.hvec;
+    ep.ximg = ws.ximg;
+    ep.himg = ws.himg;
+    ep.max_blocks = ws.max_blocks;
     ep.opart = ws.opart;
-    ep.KS = ws.KS;
+    ep.KS = path == 3 ? 1 : ws.KS;  // the GEMM's W2 pass covers all of F at once
     ep.Pmax = 2 * T;
     ep.max_chunks = ws.max_chunks;
     ep.status = ws.status;
@@ -259,8 +274,7 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     ep.debug = g_debug;
     ep.trace = g_trace;
     ep.trace_steps = g_trace_steps;
-    // decode-sized work: mma.sync GEMV; path 2 forces the tcgen05 kernels
-    rc = g_path == 2 ? launch_tc(ep, st) : launch_gemv(ep, st);
+    rc = path == 3 ? launch_gemm(ep, st) : path == 2 ? launch_tc(ep, st) : launch_gemv(ep, st);
     if (rc) return rc;
 
     CombineParams cp;
@@ -269,7 +283,7 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     cp.inv = ws.inv;
     cp.T = T;
     cp.H = shape->H;
-    cp.KS = ws.KS;
+    cp.KS = ep.KS;
     cp.Pmax = 2 * T;
     cp.y = (__nv_bfloat16 *)y;
     return launch_combine(cp, st);

@@ -1,0 +1,553 @@
+// mc_gemm.cu -- prefill-path expert kernels (many pairs per expert): grouped
+// dequant-GEMM on the 5th-generation tensor cores (Eq. 1's E_i on PMQ weights,
+// Sec. 2.2, batched over the pairs routed to each expert).
+//
+// x_img_kernel: per token block (<= 128 pairs of one expert, from the block
+//   list) and 128-column step, the fp16 activations of the block's pairs as the
+//   K-major SW128 image the MMA reads (rows = pairs, zero rows past the block),
+//   with the columns of every K = 16 slice ordered like the A operand below.
+// gemm_kernel<W13>: persistent, one CTA per SM, warp-specialised:
+//   producer warp      claims items (a token block x a 128-row block of W1|W3,
+//                      or x a 256-row block pair of W2) from an atomic counter and
+//                      streams per 128-column step one ring stage
+//                      [activation image 32 KB][packed weights of both streams]
+//                      with cp.async.bulk;
+//   converter warps 0-3 turn the packed codes (the decode path's layout) into
+//                      fp16 (q - z) s and store them into tensor memory with
+//                      tcgen05.st 16x256b, whose thread -> (lane, column) order is
+//                      the mma fragment order the packed tiles are stored in;
+//   MMA thread         tcgen05.mma kind::f16, M = 128 rows, N = 128 pairs,
+//                      K = 16, A from tensor memory, B from the image, fp32
+//                      accumulators in tensor memory (one per stream);
+//   epilogue warps 4-7 W13: h = silu(W1 x) * (W3 x) -> fp16 image of W2's input
+//                      (the same image layout, one 128-column step per row block);
+//                      W2: fp32 outputs per pair.
+// Tensor memory (512 columns): accumulators of streams 0/1 at columns 0 / 128,
+// two A buffers of 2 x 64 columns at 256 / 384.
+#include "mc_host.h"
+#include "mc_kernels.h"
+#include "mc_profile.h"
+#include "mc_umma.cuh"
+
+namespace mc {
+
+constexpr int kGN = 128;                  // pairs per token block (MMA N)
+constexpr int kImgBytes = kGN * kTileK * 2;  // one 128-column step image: 32 KB
+constexpr int kGWBytes = 2 * 8 * (256 * 3 + 128);  // weights of both streams, 3-bit, group 64
+constexpr int kGStage = kImgBytes + kGWBytes;      // 47104 = 46 KB (1024-aligned stages)
+constexpr int kGSlots = 4;
+constexpr int kGHdr = 1024;
+constexpr int kGStaging = kImgBytes;               // epilogue staging of one h image
+constexpr size_t kGSmem = kGHdr + (size_t)kGSlots * kGStage + kGStaging;
+constexpr int kGConv0 = 0, kGEpi0 = 4, kGProd = 8, kGMma = 9;
+constexpr int kGThreads = 10 * 32;
+constexpr int kGRuns = kMaxE;
+constexpr int kGItemRing = 8;
+static_assert(kGStage % 1024 == 0, "stage alignment");
+
+// Byte offset of (pair row n, column c of the 128-column step) in an image: two
+// 64-column SW128 atoms; inside an atom the four 4-column groups of every
+// 16-column run are transposed with the four K = 16 slices, so that K slice s of
+// atom a holds, in order, columns 64a + 16t + 4s + {0..3} for t = 0..3 -- the
+// columns the converter stores into tensor-memory columns 2t / 2t+1 of slice s.
+__host__ __device__ __forceinline__ uint32_t img_off(int n, int c)
+{
+    const int a = c >> 6, cc = c & 63;
+    const int t = cc >> 4, s = (cc >> 2) & 3, e = cc & 3;
+    return (uint32_t)a * 16384u + sw128_offset((uint32_t)n, (uint32_t)(16 * s + 4 * t + e));
+}
+
+struct GStage {
+    int item, kt, first, last;  // item id, column step, first / last step of the item
+    int k, u;                   // token block, unit (row block or row-block pair)
+    ChunkInfo ci;
+};
+
+struct GItem {
+    int k, u;
+    ChunkInfo ci;
+};
+
+struct GShared {
+    uint64_t full[kGSlots], empty[kGSlots];
+    uint64_t afull[2], aempty[2];
+    uint64_t dfull, dempty, esync, drain;
+    uint32_t tmem_base;
+    volatile int abort;
+    volatile int issued;
+    volatile int end_items;  // items this CTA's MMA thread completed, set once it saw the end marker
+    int nruns;
+    int run_first[kGRuns], run_nb[kGRuns], run_base[kGRuns + 1];
+    GStage stage[kGSlots];
+    GItem items[kGItemRing];
+};
+static_assert(sizeof(GShared) <= kGHdr, "gemm header");
+
+__device__ __forceinline__ bool g_wait(uint64_t *bar, uint32_t parity, const ExpertParams &p, GShared *sh)
+{
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    while (true) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (sh->abort) return false;
+        if (globaltimer_ns() - t0 > p.timeout_ns) {
+            set_status(p.status, MC_ERR_TIMEOUT);
+            sh->abort = 1;
+            return false;
+        }
+    }
+}
+
+__device__ __forceinline__ bool g_header_ok(const ExpertParams &p, int e)
+{
+    const PackHeader *hd = reinterpret_cast<const PackHeader *>(p.packed);
+    return hd->magic == kMagic && hd->version == kFormatVersion && hd->E == p.E && hd->H == p.H &&
+           hd->F == p.F && hd->group == p.group && hd->bits[e] == p.bits[e] &&
+           hd->mat_off[e][0] == p.mat_off[e][0] && hd->mat_off[e][1] == p.mat_off[e][1] &&
+           hd->mat_off[e][2] == p.mat_off[e][2];
+}
+
+// ------------------------------------------------------------------ x image --
+__global__ void __launch_bounds__(256) x_img_kernel(ExpertParams p)
+{
+    const int k = blockIdx.x, kt = blockIdx.y, KT = p.H / kTileK;
+    if (k >= *p.nchunks) return;
+    const ChunkInfo ci = p.chunks[k];
+    const int n = threadIdx.x >> 1, half = threadIdx.x & 1;
+    uint8_t *img = p.ximg + ((size_t)k * KT + kt) * kImgBytes;
+    bool bad = false;
+    const __nv_bfloat16 *src = nullptr;
+    if (n < ci.nv) src = p.x + (size_t)(p.perm[ci.pair_base + n] >> 1) * p.H + kt * kTileK + 64 * half;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+        uint4 raw = make_uint4(0, 0, 0, 0);
+        if (src) raw = reinterpret_cast<const uint4 *>(src)[q];
+        const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&raw);
+        uint32_t h[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f = __bfloat1622float2(b2[i]);
+            bad |= !(fabsf(f.x) <= 65504.f) || !(fabsf(f.y) <= 65504.f);
+            const __half2 v = __floats2half2_rn(f.x, f.y);
+            h[i] = *reinterpret_cast<const uint32_t *>(&v);
+        }
+        const int c = 64 * half + 8 * q;  // columns c .. c+7: two 4-column groups
+        *reinterpret_cast<uint2 *>(img + img_off(n, c)) = make_uint2(h[0], h[1]);
+        *reinterpret_cast<uint2 *>(img + img_off(n, c + 4)) = make_uint2(h[2], h[3]);
+    }
+    if (bad) set_status(p.status, MC_ERR_RANGE);
+}
+
+// -------------------------------------------------------------- converters --
+
+// Exponent-constant bits of pair j (the fp16 2^E the decoder adds, both halves).
+template <int BITS>
+__device__ __forceinline__ uint32_t pair_offset_bits(int j)
+{
+    const int f = BITS == 1 ? off1_pos(j) : BITS == 2 ? 2 * off2_pos(j) : off3_bit(j);
+    return MC_C(25 - f);
+}
+
+__device__ __forceinline__ uint32_t h2_bits(__half2 v) { return *reinterpret_cast<const uint32_t *>(&v); }
+__device__ __forceinline__ __half2 bits_h2(uint32_t v) { return *reinterpret_cast<const __half2 *>(&v); }
+
+// One 16-row tile, one 128-column step: 32 fp16 pairs (q - z) s per lane, in the
+// order tcgen05.st 16x256b.x8 takes them: per k-step s, the A-fragment registers
+// a0, a2, a1, a3 (rows g8 / g8+8, k pairs t / t+4).
+template <int BITS, int GPT>
+__device__ __forceinline__ void convert_tile(const uint8_t *tile, int lane, uint32_t (&out)[32])
+{
+    uint32_t c2[4] = {0, 0, 0, 0}, c1[2] = {0, 0};
+    if (BITS >= 2) {
+        const uint4 v = *reinterpret_cast<const uint4 *>(tile + 16 * lane);
+        c2[0] = v.x; c2[1] = v.y; c2[2] = v.z; c2[3] = v.w;
+    }
+    if (BITS != 2) {
+        const uint2 v = *reinterpret_cast<const uint2 *>(tile + (BITS == 3 ? 512 : 0) + 8 * lane);
+        c1[0] = v.x; c1[1] = v.y;
+    }
+    const uint8_t *mt = tile + tile_code_bytes(BITS);
+    __half2 s2[GPT][2], nz2[GPT][2];  // [group][row half]: (s, s) and (-z s, -z s)
+#pragma unroll
+    for (int g = 0; g < GPT; ++g) {
+        const uint2 m = *reinterpret_cast<const uint2 *>(mt + 64 * g + (lane >> 2) * 8);
+        const __half2 a = bits_h2(m.x), b = bits_h2(m.y);  // (s0, z0), (s1, z1)
+        const float sa = __low2float(a), za = __high2float(a), sb = __low2float(b), zb = __high2float(b);
+        s2[g][0] = __floats2half2_rn(sa, sa);
+        s2[g][1] = __floats2half2_rn(sb, sb);
+        nz2[g][0] = __floats2half2_rn(-za * sa, -za * sa);
+        nz2[g][1] = __floats2half2_rn(-zb * sb, -zb * sb);
+    }
+#pragma unroll
+    for (int qd = 0; qd < 4; ++qd) {
+        uint32_t r[8];
+        if (BITS == 1) cvt1_half(c1[qd >> 1], 8 * (qd & 1), r);
+        if (BITS == 2) cvt2(c2[qd], r);
+        if (BITS == 3) {
+            const uint32_t w[6] = {c2[0], c2[1], c2[2], c2[3], c1[0], c1[1]};
+            cvt3(w, qd, r);
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const int j = 8 * qd + i, s = j >> 2, rho = j & 3;
+            const int gi = GPT == 2 ? (s >> 2) : 0;
+            const __half2 q = __hsub2(bits_h2(r[i]), bits_h2(pair_offset_bits<BITS>(j)));  // exact
+            const __half2 w = __hfma2(q, s2[gi][rho & 1], nz2[gi][rho & 1]);
+            // st order per k-step: a0 (rho 0), a2 (rho 2), a1 (rho 1), a3 (rho 3)
+            const int slot = rho == 0 ? 0 : rho == 2 ? 1 : rho == 1 ? 2 : 3;
+            out[4 * s + slot] = h2_bits(w);
+        }
+    }
+}
+
+__device__ __forceinline__ void tmem_st_16x256_x8(uint32_t taddr, const uint32_t (&v)[32])
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.16x256b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
+        "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]),
+        "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]),
+        "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
+        : "memory");
+}
+
+template <int GPT>
+__device__ __forceinline__ void convert_store(const uint8_t *tile, int bits, int lane, uint32_t taddr)
+{
+    uint32_t v[32];
+    if (bits == 1) convert_tile<1, GPT>(tile, lane, v);
+    else if (bits == 2) convert_tile<2, GPT>(tile, lane, v);
+    else convert_tile<3, GPT>(tile, lane, v);
+    tmem_st_16x256_x8(taddr, v);
+}
+
+// ------------------------------------------------------------- epilogue --
+
+__device__ __forceinline__ void tmem_ld_x16(uint32_t taddr, float (&v)[16])
+{
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Epilogue warps meet (bounded); false once the CTA aborted.
+__device__ __forceinline__ bool epi_sync(const ExpertParams &p, GShared *sh, int lane, int &uses)
+{
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sh->esync);
+    return g_wait(&sh->esync, (uses++) & 1, p, sh);
+}
+
+// ------------------------------------------------------------------ kernel --
+
+template <bool W13, int GPT>
+__global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
+{
+    extern __shared__ __align__(1024) uint8_t smem[];
+    GShared *sh = reinterpret_cast<GShared *>(smem);
+    uint8_t *ring = smem + kGHdr;
+    uint8_t *staging = smem + kGHdr + (size_t)kGSlots * kGStage;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int group = kTileK / GPT;
+    const int nrb = W13 ? p.F / kBlockRows : p.H / kBlockRows;
+    const int U = W13 ? nrb : (nrb + 1) / 2;
+    const int KTm = W13 ? p.H / kTileK : p.F / kTileK;  // column steps (K)
+    const uint8_t *img_base = W13 ? p.ximg : p.himg;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kGSlots; ++s) {
+            mbar_init(&sh->full[s], 1);
+            mbar_init(&sh->empty[s], 1 + 4);  // MMA commit + converter warps
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&sh->afull[b], 4);
+            mbar_init(&sh->aempty[b], 1);
+        }
+        mbar_init(&sh->dfull, 1);
+        mbar_init(&sh->dempty, 4);
+        mbar_init(&sh->esync, 4);
+        mbar_init(&sh->drain, 1);
+        sh->abort = 0;
+        sh->issued = 0;
+        sh->end_items = 0x7fffffff;
+        // runs of token blocks per expert (the block list is grouped by expert)
+        const int nb = *p.nchunks;
+        int r = 0, base = 0;
+        for (int k = 0; k < nb; ++k) {
+            if (k == 0 || p.chunks[k].e != p.chunks[k - 1].e) {
+                if (r > 0) base += sh->run_nb[r - 1] * U;
+                sh->run_first[r] = k;
+                sh->run_nb[r] = 0;
+                sh->run_base[r] = base;
+                ++r;
+            }
+            sh->run_nb[r - 1]++;
+        }
+        sh->nruns = r;
+        sh->run_base[r] = r > 0 ? base + sh->run_nb[r - 1] * U : 0;
+        fence_mbar_init();
+    }
+    if (warp == kGMma) tmem_alloc(&sh->tmem_base, 512);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tbase = sh->tmem_base;
+    const int total = sh->run_base[sh->nruns];
+
+    if (warp == kGProd) {
+        // ------------------------------------------------------------ producer --
+        if (lane == 0 && !(p.debug & kDebugNoProducer)) {
+            const uint64_t pol = policy_evict_first();
+            int it = 0, nitem = 0;
+            bool ok = true;
+            uint32_t verified = 0;
+            while (ok) {
+                const int item = atomicAdd(&p.counters[W13 ? 2 : 3], 1);
+                if (item >= total) break;
+                int r = 0;
+                while (r + 1 < sh->nruns && item >= sh->run_base[r + 1]) ++r;
+                const int local = item - sh->run_base[r], nbr = sh->run_nb[r];
+                const int u = local / nbr, k = sh->run_first[r] + local % nbr;
+                const ChunkInfo ci = p.chunks[k];
+                const int e = ci.e, bits = ci.bits;
+                if (!((verified >> e) & 1u)) {
+                    if (!g_header_ok(p, e)) {
+                        set_status(p.status, MC_ERR_BAD_PACK);
+                        sh->abort = 1;
+                        ok = false;
+                        break;
+                    }
+                    verified |= 1u << e;
+                }
+                GItem gi;
+                gi.k = k;
+                gi.u = u;
+                gi.ci = ci;
+                sh->items[nitem % kGItemRing] = gi;
+                ++nitem;
+                const int STB = supertile_bytes(bits, group);
+                const int pw = W13 ? 2 : w2_pair_width(u, nrb);
+                const uint8_t *wsrc = p.packed + p.mat_off[e][W13 ? 0 : 2] +
+                                      supertile_off(W13 ? 0 : 2, W13 ? u : 2 * u, 0, KTm, nrb, STB);
+                const uint8_t *isrc = img_base + (size_t)k * KTm * kImgBytes;
+                for (int kt = 0; kt < KTm; ++kt, ++it) {
+                    const int slot = it % kGSlots;
+                    if (it >= kGSlots && !g_wait(&sh->empty[slot], ((it / kGSlots) - 1) & 1, p, sh)) {
+                        ok = false;
+                        break;
+                    }
+                    GStage &st = sh->stage[slot];
+                    st.item = item;
+                    st.kt = kt;
+                    st.first = kt == 0;
+                    st.last = kt == KTm - 1;
+                    st.k = k;
+                    st.u = u;
+                    st.ci = ci;
+                    uint8_t *dst = ring + (size_t)slot * kGStage;
+                    const uint32_t wb = (uint32_t)(pw * STB);
+                    mbar_arrive_expect_tx(&sh->full[slot], (uint32_t)kImgBytes + wb);
+                    bulk_g2s(dst, isrc + (size_t)kt * kImgBytes, kImgBytes, &sh->full[slot]);
+                    bulk_g2s_stream(dst + kImgBytes, wsrc + (size_t)kt * pw * STB, wb, &sh->full[slot], pol);
+                    sh->issued = it + 1;
+                }
+            }
+            if (ok) {
+                const int slot = it % kGSlots;
+                if (it < kGSlots || g_wait(&sh->empty[slot], ((it / kGSlots) - 1) & 1, p, sh)) {
+                    sh->stage[slot].item = -1;
+                    mbar_arrive(&sh->full[slot]);
+                }
+            }
+        }
+    } else if (warp < kGEpi0) {
+        // ---------------------------------------------------------- converters --
+        // warp q: tensor-memory lanes 32q .. 32q+31 = rows of tiles 2q, 2q+1
+        const int q = warp - kGConv0;
+        for (int it = 0;; ++it) {
+            const int slot = it % kGSlots, b = it & 1;
+            if (!g_wait(&sh->full[slot], (it / kGSlots) & 1, p, sh)) break;
+            const GStage st = sh->stage[slot];
+            if (st.item < 0) break;
+            if (it >= 2 && !g_wait(&sh->aempty[b], ((it >> 1) - 1) & 1, p, sh)) break;
+            tc_fence_after();
+            const int bits = st.ci.bits, STB = supertile_bytes(bits, group), TB = tile_bytes(bits, group);
+            const int nstream = W13 ? 2 : w2_pair_width(st.u, nrb);
+            const uint8_t *w = ring + (size_t)slot * kGStage + kImgBytes;
+            const uint32_t abuf = tbase + 256u + 128u * (uint32_t)b;
+            for (int x = 0; x < nstream; ++x)
+                for (int u2 = 0; u2 < 2; ++u2) {
+                    const uint8_t *tile = w + x * STB + (2 * q + u2) * TB;
+                    const uint32_t taddr = abuf + 64u * (uint32_t)x + ((uint32_t)(32 * q + 16 * u2) << 16);
+                    convert_store<GPT>(tile, bits, lane, taddr);
+                }
+            tmem_st_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(&sh->afull[b]);
+                mbar_arrive(&sh->empty[slot]);
+            }
+        }
+    } else if (warp == kGMma) {
+        // ----------------------------------------------------------------- MMA --
+        if (lane == 0) {
+            const uint32_t idesc = umma_idesc_f16(128, kGN);
+            int nitem = 0;
+            for (int it = 0;; ++it) {
+                const int slot = it % kGSlots, b = it & 1;
+                if (!g_wait(&sh->full[slot], (it / kGSlots) & 1, p, sh)) break;
+                const GStage st = sh->stage[slot];
+                if (st.item < 0) break;
+                if (!g_wait(&sh->afull[b], (it >> 1) & 1, p, sh)) break;
+                if (st.first && nitem > 0 && !g_wait(&sh->dempty, (nitem - 1) & 1, p, sh)) break;
+                tc_fence_after();
+                const int nstream = W13 ? 2 : w2_pair_width(st.u, nrb);
+                const uint8_t *img = ring + (size_t)slot * kGStage;
+                const uint32_t abuf = tbase + 256u + 128u * (uint32_t)b;
+                for (int x = 0; x < nstream; ++x)
+#pragma unroll
+                    for (int s = 0; s < 8; ++s) {
+                        const uint64_t bd = umma_desc_sw128(img + (s >> 2) * 16384 + (s & 3) * 32);
+                        umma_f16_ts(tbase + 128u * (uint32_t)x, abuf + 64u * (uint32_t)x + 8u * (uint32_t)s, bd,
+                                    idesc, !(st.first && s == 0));
+                    }
+                umma_commit(&sh->aempty[b]);
+                umma_commit(&sh->empty[slot]);
+                if (st.last) {
+                    umma_commit(&sh->dfull);
+                    ++nitem;
+                }
+            }
+            // every MMA this thread issued has completed (and with it every commit
+            // to dfull) before the epilogue is told that no item follows and
+            // before TMEM is released
+            umma_commit(&sh->drain);
+            const uint64_t t0 = globaltimer_ns();
+            while (!mbar_try_wait(&sh->drain, 0))
+                if (globaltimer_ns() - t0 > p.timeout_ns) break;
+            // the epilogue has taken the last item before dfull completes once more,
+            // so that it never sees two completions of dfull in one wait
+            if (nitem == 0 || g_wait(&sh->dempty, (nitem - 1) & 1, p, sh)) {
+                sh->end_items = nitem;
+                mbar_arrive(&sh->dfull);
+            }
+        }
+    } else if (warp >= kGEpi0 && warp < kGEpi0 + 4) {
+        // ------------------------------------------------------------ epilogue --
+        const int ew = warp - kGEpi0;   // tensor-memory lanes 32 ew .. 32 ew + 31
+        const int row = 32 * ew + lane;  // row of the 128-row block
+        const int tid = threadIdx.x - 32 * kGEpi0;
+        int uses = 0;
+        for (int ic = 0;; ++ic) {
+            if (!g_wait(&sh->dfull, ic & 1, p, sh)) break;
+            if (ic >= sh->end_items) break;
+            tc_fence_after();
+            const GItem gi = sh->items[ic % kGItemRing];
+            const uint32_t lane_addr = (uint32_t)(32 * ew) << 16;
+            if (W13) {
+                bool bad = false;
+                for (int n0 = 0; n0 < kGN; n0 += 16) {
+                    float g[16], v[16];
+                    tmem_ld_x16(tbase + lane_addr + (uint32_t)n0, g);
+                    tmem_ld_x16(tbase + lane_addr + 128u + (uint32_t)n0, v);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        const float h = silu(g[i]) * v[i];
+                        bad |= !(fabsf(h) <= 65504.f);
+                        *reinterpret_cast<__half *>(staging + img_off(n0 + i, row)) = __float2half_rn(h);
+                    }
+                }
+                if (bad) set_status(p.status, MC_ERR_RANGE);
+            } else {
+                const int nstream = w2_pair_width(gi.u, nrb);
+                for (int x = 0; x < nstream; ++x) {
+                    const int blk = 2 * gi.u + x;
+                    for (int n0 = 0; n0 < kGN; n0 += 16) {
+                        float v[16];
+                        tmem_ld_x16(tbase + lane_addr + 128u * (uint32_t)x + (uint32_t)n0, v);
+#pragma unroll
+                        for (int i = 0; i < 16; ++i)
+                            if (n0 + i < gi.ci.nv)
+                                p.opart[(size_t)(gi.ci.pair_base + n0 + i) * p.H + blk * kBlockRows + row] = v[i];
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sh->dempty);
+            if (W13) {
+                // the image of W2's column step gi.u for token block gi.k
+                if (!epi_sync(p, sh, lane, uses)) break;
+                uint4 *dst = reinterpret_cast<uint4 *>(p.himg + ((size_t)gi.k * (p.F / kTileK) + gi.u) * kImgBytes);
+                const uint4 *src = reinterpret_cast<const uint4 *>(staging);
+                for (int i = tid; i < kImgBytes / 16; i += 128) dst[i] = src[i];
+                if (!epi_sync(p, sh, lane, uses)) break;
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (threadIdx.x == 0 && sh->abort) {
+        for (int it = max(0, sh->issued - kGSlots); it < sh->issued; ++it) {
+            const uint64_t t0 = globaltimer_ns();
+            while (!mbar_try_wait(&sh->full[it % kGSlots], (it / kGSlots) & 1))
+                if (globaltimer_ns() - t0 > p.timeout_ns) break;
+        }
+    }
+    if (warp == kGMma) {
+        tc_fence_after();
+        tmem_dealloc(tbase, 512);
+    }
+}
+
+// --------------------------------------------------------------- launcher --
+
+int launch_gemm(ExpertParams ep, cudaStream_t st)
+{
+    int dev = 0, maxsm = 0, nsm = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err == cudaSuccess) err = cudaDeviceGetAttribute(&maxsm, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    if (err == cudaSuccess) err = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "device query: %s", cudaGetErrorString(err));
+    if ((size_t)maxsm < kGSmem) return set_error(MC_ERR_UNSUPPORTED, "not enough shared memory for the GEMM ring");
+    if (!ep.ximg || !ep.himg) return set_error(MC_ERR_INVALID_ARG, "prefill path without image buffers");
+    auto k13 = ep.group == 64 ? gemm_kernel<true, 2> : gemm_kernel<true, 1>;
+    auto k2 = ep.group == 64 ? gemm_kernel<false, 2> : gemm_kernel<false, 1>;
+    err = cudaFuncSetAttribute(k13, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGSmem);
+    if (err == cudaSuccess) err = cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGSmem);
+    if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(err));
+
+    profile_begin(kKGemmGather, st);
+    x_img_kernel<<<dim3(ep.max_blocks, ep.H / kTileK), 256, 0, st>>>(ep);
+    profile_end(kKGemmGather, st);
+    err = cudaGetLastError();
+    if (err == cudaSuccess) {
+        profile_begin(kKGemmW13, st);
+        k13<<<nsm, kGThreads, kGSmem, st>>>(ep);
+        profile_end(kKGemmW13, st);
+        err = cudaGetLastError();
+    }
+    if (err == cudaSuccess) {
+        profile_begin(kKGemmW2, st);
+        k2<<<nsm, kGThreads, kGSmem, st>>>(ep);
+        profile_end(kKGemmW2, st);
+        err = cudaGetLastError();
+    }
+    if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "GEMM launch: %s", cudaGetErrorString(err));
+    return MC_OK;
+}
+
+size_t img_buffer_bytes(int max_blocks, int cols) { return (size_t)max_blocks * (cols / kTileK) * kImgBytes; }
+int max_blocks_for(int T, int E) { return (2 * T + kGN - 1) / kGN + E; }
+
+}  // namespace mc

@@ -62,6 +62,7 @@ struct PermuteParams {
     ChunkInfo *chunks;    // [max_chunks] or null
     int32_t *nchunks;     // [1]
     int32_t *counters;    // [4] work counters of the expert kernels, reset here
+    int chunk;            // pairs per work chunk: 16 (GEMV paths) or 128 (prefill GEMM)
 };
 
 // Decode-path expert kernels (persistent, mma.sync).
@@ -82,6 +83,9 @@ struct ExpertParams {
     float *gu;               // [max_chunks][2][F][16] W1 / W3 results (tensor-core path)
     uint8_t *xvec;           // [max_chunks][2][H/128] vector blocks of x (mma.sync path)
     uint8_t *hvec;           // [max_chunks][2][F/128] vector blocks of h (mma.sync path)
+    uint8_t *ximg;           // [max_blocks][H/128] 32 KB activation images (prefill path)
+    uint8_t *himg;           // [max_blocks][F/128] 32 KB h images (prefill path)
+    int max_blocks;          // token blocks of <= 128 pairs (prefill path)
     float *opart;            // [KS, Pmax, H]  expert outputs (fp32), pair order
     int KS;                  // column splits of the W2 pass
     int Pmax;                // 2 * T
@@ -110,6 +114,9 @@ struct CombineParams {
 int launch_route(const RouteParams &rp, const PermuteParams &pp, cudaStream_t st);
 int launch_gemv(ExpertParams ep, cudaStream_t st);   // mma.sync path
 int launch_tc(ExpertParams ep, cudaStream_t st);     // tcgen05 path
+int launch_gemm(ExpertParams ep, cudaStream_t st);   // prefill path (tcgen05 grouped GEMM)
+size_t img_buffer_bytes(int max_blocks, int cols);
+int max_blocks_for(int T, int E);
 int launch_combine(const CombineParams &cp, cudaStream_t st);
 int max_chunks_for(int T, int E);
 

@@ -152,6 +152,7 @@ extern "C" int mc_moe_forward_static(const void *x, const void *gate_w, int T, c
     pp.chunks = ws.chunks;
     pp.nchunks = ws.nchunks;
     pp.counters = ws.counters;
+    pp.chunk = kChunk;
     if ((rc = launch_route(rp, pp, st))) return rc;
 
     ExpertParams ep;

@@ -122,16 +122,16 @@ __global__ void __launch_bounds__(1024) permute_kernel(PermuteParams p)
         }
         p.offsets[p.E] = s;
         if (p.chunks) {
-            // work chunks of <= 16 pairs, experts with more bits first
+            // work chunks of <= p.chunk pairs, experts with more bits first
             int k = 0;
             for (int b = 3; b >= 1; --b)
                 for (int e = 0; e < p.E; ++e) {
                     if (p.bits[e] != b) continue;
-                    for (int c = 0; c < cnt[e]; c += kChunk) {
+                    for (int c = 0; c < cnt[e]; c += p.chunk) {
                         ChunkInfo ci;
                         ci.e = e;
                         ci.pair_base = run[e] + c;
-                        ci.nv = min(kChunk, cnt[e] - c);
+                        ci.nv = min(p.chunk, cnt[e] - c);
                         ci.bits = b;
                         p.chunks[k++] = ci;
                     }
