@@ -8,7 +8,7 @@ quoted on.  A step is one mc_moe_forward (gate, top-2, ODP, permutation, W1|W3
 GEMV + SwiGLU, W2 GEMV, combine) on resident device inputs.  Packed weights
 rotate over several device copies so that no step finds its weights in L2.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload decode16|decode1|decode4]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload decode16|decode1|decode4|prefill4096]
   python bench.py --impl reference ...   (the CPU oracle on the host cores)
 
 Under torchrun every rank runs an independent replica (the layer does not need a
@@ -33,7 +33,8 @@ sys.path.insert(0, ROOT)
 import synth  # noqa: E402
 
 METRIC = "Mixed-bit MoE-layer tokens/s; % HBM roofline (decode), % TC peak (prefill)"
-WORKLOADS = {"decode16": 16, "decode4": 4, "decode1": 1}
+WORKLOADS = {"decode16": ("decode", 16), "decode4": ("decode", 4), "decode1": ("decode", 1),
+             "prefill4096": ("prefill", 4096)}
 
 
 def _peaks():
@@ -48,7 +49,7 @@ def _peaks():
 class Clocks:
     """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
 
-    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    Q = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
@@ -60,12 +61,14 @@ class Clocks:
     def start(self):
         try:
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.Q,
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except Exception:
             self.proc = None
 
-    def stop(self):
+    def stop(self, window=None):
+        """Median SM clock and the throttle reasons seen; samples restricted to
+        `window` = (t0, t1) host wall-clock seconds when any fall inside it."""
         if self.proc is None:
             return None
         self.proc.terminate()
@@ -74,24 +77,29 @@ class Clocks:
         except Exception:
             self.proc.kill()
             out, _ = self.proc.communicate()
-        sm, mx, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        rows = []
         for line in out.strip().splitlines():
             f = [x.strip() for x in line.split(",")]
-            if len(f) < 9:
+            if len(f) < 10:
                 continue
             try:
-                sm.append(float(f[1]))
-                mx.append(float(f[2]))
-            except ValueError:
+                ts = time.mktime(time.strptime(f[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                ts += float("0." + f[0].split(".")[1]) if "." in f[0] else 0.0
+                rows.append((ts, float(f[2]), float(f[3]), [n for n, v in zip(names, f[6:10])
+                                                            if v.lower().startswith("active")]))
+            except (ValueError, IndexError):
                 continue
-            for n, v in zip(names, f[5:9]):
-                if v.lower().startswith("active"):
-                    reasons.add(n)
-        if not sm:
+        if not rows:
             return None
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
-                "reasons": sorted(reasons)}
+        where = "run"
+        if window is not None:
+            inside = [r for r in rows if window[0] - 0.05 <= r[0] <= window[1] + 0.05]
+            if inside:
+                rows, where = inside, "timed region"
+        reasons = sorted({n for r in rows for n in r[3]})
+        return {"sm_mhz": statistics.median(r[1] for r in rows), "sm_max_mhz": max(r[2] for r in rows),
+                "samples": len(rows), "window": where, "reasons": reasons}
 
 
 def _dist():
@@ -139,26 +147,52 @@ def run_reference(args):
     world, rank, _ = _dist()
     if rank != 0:
         return 0
-    T = WORKLOADS[args.workload]
-    L = synth.config_decode(T=T)
-    steps = []
+    kind, T, L = _workload(args.workload)
+    steps = args.steps if args.steps else 3
+    vals = []
     cb = None
-    for i in range(args.warmup + args.steps):
-        r = cpu_baseline(L, budget_s=4.0)
+    budget = min(4.0, 150.0 / (args.warmup + steps))  # the whole run stays within a few minutes
+    for i in range(args.warmup + steps):
+        r = cpu_baseline(L, budget_s=budget)
         if i >= args.warmup:
-            steps.append(r["value"])
+            vals.append(r["value"])
             cb = r
-    v = statistics.median(steps)
+    v = statistics.median(vals)
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": args.gpus,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * T / v, "higher_is_better": True,
+            "steps": steps, "warmup": args.warmup, "ms_per_step": 1000.0 * T / v, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": "mixtral-8x7b MoE layer decode, %d tokens, H 4096, F 14336, 8 experts, "
-                                   "top-2, group 128, bits sum 20, ODP off" % T},
+            "config": {"workload": _describe(kind, T, L)},
             "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cb["cores"], "kind": "oracle",
                              "sample": cb["sample"]},
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     return 0
+
+
+def _workload(name):
+    kind, T = WORKLOADS[name]
+    L = synth.config_decode(T=T) if kind == "decode" else synth.config_prefill(T=T)
+    return kind, T, L
+
+
+def _describe(kind, T, L):
+    return ("mixtral-8x7b MoE layer %s, %d tokens, H 4096, F 14336, 8 experts, top-2, group 128, bits %s "
+            "(mean %.2f), ODP off%s" % (kind, T, list(map(int, L.bits)), L.mean_bits(),
+                                         ", expert loads skewed ~4:1" if kind == "prefill" else ""))
+
+
+def _traffic(kernel, workload):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, if it was
+    taken on the kernel's current source (else None)."""
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            d = json.load(f)[kernel + "/" + workload]
+        with open(os.path.join(ROOT, "paper_2410_06270_gb300", "csrc", d["source"]), "rb") as f:
+            sha = hashlib.sha256(f.read()).hexdigest()
+        return float(d["bytes_per_launch"]) if sha == d["source_sha256"] else None
+    except Exception:
+        return None
 
 
 def run(args):
@@ -172,8 +206,8 @@ def run(args):
     if world > 1:
         dist.init_process_group("nccl")
     dev = torch.device("cuda", local)
-    T = WORKLOADS[args.workload]
-    L = synth.config_decode(T=T)
+    kind, T, L = _workload(args.workload)
+    steps = args.steps if args.steps else (2000 if kind == "decode" else 100)
     shape = mc.Shape(L.E, L.H, L.F, L.group)
     flat = lambda a: [a[e][m] for e in range(L.E) for m in range(3)]
     packed_host = mc.pack_experts_host(shape, L.bits, flat(L.codes), flat(L.scale), flat(L.zero))
@@ -184,38 +218,54 @@ def run(args):
     gw = torch.from_numpy(L.gate.view(np.int16).copy()).view(torch.bfloat16).to(dev)
     ws = mc.alloc_workspace(shape, T, dev)
     y = torch.empty_like(x)
-    idx = None
 
     def step(i):
         return mc.moe_forward(x, gw, shape, L.bits, packed[i % nsets], 0.0, None, y=y, workspace=ws)
 
-    # routing once, to know which experts a step touches (fixed inputs)
+    # routing once, to know which experts a step touches and how many pairs it keeps (fixed inputs)
     _, r = mc.moe_forward(x, gw, shape, L.bits, packed[0], 0.0, None, y=y, workspace=ws, routing=True)
     mc.check_status(ws)
     idx = r["idx"].cpu().numpy()
+    pairs = int(2 * T - int(r["pruned"].sum().item()))
     touched = sorted(set(idx.reshape(-1).tolist()))
     alg_bytes, w13_bytes = _algorithmic_bytes(shape, L.bits, touched, T, L.H)
+    w13_flops = 4.0 * L.H * L.F * pairs          # W1 and W3: 2 x (2 H F) per kept pair
+    layer_flops = 6.0 * L.H * L.F * pairs + 2.0 * L.H * L.E * T
+    rk = "gemv_w13" if kind == "decode" else "gemm_w13"
 
+    clocks = Clocks(local)
+    clocks.start()
     for i in range(args.warmup):
         step(i)
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
-    clocks = Clocks(local)
-    clocks.start()
+    # timed region: K steps; the library records events around the roofline kernel only
+    mc.profile_select([rk])
     mc.profile_enable(True)
     stream = torch.cuda.current_stream()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
+    t_wall0 = time.time()
     e0.record(stream)
-    for i in range(args.steps):
+    for i in range(steps):
         step(i)
     e1.record(stream)
     torch.cuda.synchronize()
+    t_wall1 = time.time()
     mc.profile_enable(False)
     prof = mc.profile_read()
     ms = e0.elapsed_time(e1)
     mc.check_status(ws)
+    cl = clocks.stop((t_wall0, t_wall1))
+    # per-kernel breakdown: a separate profiled pass (every kernel bracketed by events)
+    mc.profile_select(None)
+    mc.profile_enable(True)
+    for i in range(min(steps, 50)):
+        step(i)
+    torch.cuda.synchronize()
+    mc.profile_enable(False)
+    breakdown = mc.profile_read()
     # end to end through the public API: pinned host input -> device -> layer -> host
     xh = torch.empty(x.shape, dtype=x.dtype, pin_memory=True)
     xh.copy_(x.cpu())
@@ -223,14 +273,13 @@ def run(args):
     torch.cuda.synchronize()
     e2, e3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e2.record(stream)
-    for i in range(args.steps):
+    for i in range(steps):
         x.copy_(xh, non_blocking=True)
         step(i)
         yh.copy_(y, non_blocking=True)
     e3.record(stream)
     torch.cuda.synchronize()
     ms_e2e = e2.elapsed_time(e3)
-    cl = clocks.stop()
 
     t_local = torch.tensor([ms, ms_e2e], dtype=torch.float64, device=dev)
     if world > 1:
@@ -243,32 +292,42 @@ def run(args):
         return 0
 
     hbm, bf16, src = _peaks()
-    w13_ms, w13_n = prof.get("gemv_w13", (0.0, 0))
-    avg = w13_ms / max(w13_n, 1)
-    achieved = w13_bytes / (avg * 1e-3) / 1e9 if avg > 0 else None
-    launches = sum(n for _, n in prof.values())
-    value = world * T * args.steps / (ms * 1e-3)
-    e2e = world * T * args.steps / (ms_e2e * 1e-3)
-    layer_gbs = alg_bytes * args.steps / (ms * 1e-3) / 1e9
+    k_ms, k_n = prof.get(rk, (0.0, 0))
+    avg = k_ms / max(k_n, 1)
+    value = world * T * steps / (ms * 1e-3)
+    e2e = world * T * steps / (ms_e2e * 1e-3)
+    if kind == "decode":
+        achieved = w13_bytes / (avg * 1e-3) / 1e9 if avg > 0 else None
+        layer_gbs = alg_bytes * steps / (ms * 1e-3) / 1e9
+        roof = {"bound": "hbm", "kernel": rk, "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                "frac": (achieved / hbm) if achieved else None, "traffic": _traffic(rk, args.workload),
+                "peak_source": "%s (MEASURED_PEAKS.json hbm_gbs)" % src if src == "measured" else src,
+                "algorithmic_bytes_per_launch": w13_bytes, "layer_gbs": layer_gbs, "layer_frac": layer_gbs / hbm}
+    else:
+        sustained = _peak_sustained() or bf16
+        achieved = w13_flops / (avg * 1e-3) / 1e12 if avg > 0 else None
+        layer_tf = layer_flops * steps / (ms * 1e-3) / 1e12
+        roof = {"bound": "tensor", "kernel": rk, "achieved": achieved, "peak": sustained, "unit": "TFLOP/s",
+                "frac": (achieved / sustained) if achieved else None, "traffic": _traffic(rk, args.workload),
+                "peak_source": "%s (MEASURED_PEAKS.json bf16_tflops_sustained; fp16 has the bf16 rate)" % src
+                               if src == "measured" else src,
+                "frac_of_burst_peak": (achieved / bf16) if achieved else None,
+                "algorithmic_flops_per_launch": w13_flops, "layer_tflops": layer_tf,
+                "layer_frac": layer_tf / sustained, "kept_pairs": pairs}
     line = {
-        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": steps,
+        "warmup": args.warmup, "ms_per_step": ms / steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f16 x {1,2,3}-bit codes, fp32 accumulate", "data": "synthetic",
-        "config": {"workload": "mixtral-8x7b MoE layer decode, %d tokens, H 4096, F 14336, 8 experts, top-2, "
-                               "group 128, bits %s (mean %.2f), ODP off" % (T, list(map(int, L.bits)), L.mean_bits()),
+        "config": {"workload": _describe(kind, T, L),
                    "global_batch": T * world, "parallelism": "replicas" if world > 1 else "single",
                    "l2": "inputs larger than L2: %d rotating copies of the %.0f MB packed weights"
                          % (nsets, packed_host.nbytes / 1e6),
                    "touched_experts": len(touched)},
-        "roofline": {"bound": "hbm", "kernel": "gemv_w13", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                     "frac": (achieved / hbm) if achieved else None, "traffic": None,
-                     "peak_source": "%s (MEASURED_PEAKS.json hbm_gbs)" % src if src == "measured" else src,
-                     "algorithmic_bytes_per_launch": w13_bytes,
-                     "layer_gbs": layer_gbs, "layer_frac": layer_gbs / hbm},
-        "kernels_ms_per_step": {k: v[0] / max(v[1], 1) for k, v in prof.items()},
+        "roofline": roof,
+        "kernels_ms_per_step": {k: v[0] / max(v[1], 1) for k, v in breakdown.items()},
         "e2e": {"value": e2e, "unit": "tokens/s", "h2d_bytes_per_step": int(x.numel() * 2),
                 "d2h_bytes_per_step": int(y.numel() * 2)},
-        "gpu_launches": launches,
+        "gpu_launches": _launches_per_step(breakdown, min(steps, 50)) * steps,
         "clocks": cl,
     }
     if not args.no_cpu_baseline:
@@ -279,10 +338,22 @@ def run(args):
     return 0
 
 
+def _launches_per_step(breakdown, n):
+    return int(round(sum(c for _, c in breakdown.values()) / max(n, 1)))
+
+
+def _peak_sustained():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops_sustained"])
+    except Exception:
+        return None
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=0, help="timed steps (default: 2000 decode, 100 prefill)")
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="mc", choices=["mc", "reference"])
     ap.add_argument("--workload", default="decode16", choices=sorted(WORKLOADS))

@@ -224,6 +224,10 @@ int mc_check_status(void *workspace, void *stream);
  * gemv_w13, gemv_w2, combine, gemm_gather, gemm_w13, gemm_w2, rmsnorm, glu) and
  * clears the records.  Not for use inside CUDA graph capture. */
 int mc_profile_enable(int on);
+/* Bit mask of the kernel ids recorded while profiling is on (default: all), so
+ * that a benchmark can time one kernel with two events per launch and leave the
+ * others unperturbed.  Returns the previous mask. */
+unsigned mc_profile_select(unsigned mask);
 int mc_profile_read(double *ms_out, int *count_out, int n);
 const char *mc_profile_name(int id);
 

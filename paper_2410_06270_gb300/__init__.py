@@ -71,6 +71,7 @@ def load():
         "mc_selftest_umma": (I, [P, P, P, I, I, P, P]),
         "mc_set_trace": (I, [P, I]),
         "mc_profile_enable": (I, [I]),
+        "mc_profile_select": (ctypes.c_uint, [ctypes.c_uint]),
         "mc_profile_read": (I, [P, P, I]),
         "mc_profile_name": (ctypes.c_char_p, [I]),
     }
@@ -314,6 +315,15 @@ N_KERNELS = 10
 
 def profile_enable(on: bool = True) -> bool:
     return bool(load().mc_profile_enable(1 if on else 0))
+
+
+def profile_select(names) -> None:
+    """Record only the named kernels (None = all) while profiling is on."""
+    if names is None:
+        load().mc_profile_select(0xFFFFFFFF)
+        return
+    ids = [i for i in range(N_KERNELS) if load().mc_profile_name(i).decode() in set(names)]
+    load().mc_profile_select(sum(1 << i for i in ids))
 
 
 def profile_read() -> dict:

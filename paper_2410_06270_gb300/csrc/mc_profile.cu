@@ -14,6 +14,7 @@ struct Rec {
 };
 std::mutex g_mu;
 bool g_on = false;
+unsigned g_mask = ~0u;  // kernel ids recorded while on
 std::vector<Rec> g_recs;
 std::vector<cudaEvent_t> g_pool;
 cudaEvent_t g_pending[kKCount];
@@ -37,7 +38,7 @@ bool profile_on() { return g_on; }
 
 void profile_begin(int id, cudaStream_t st)
 {
-    if (!g_on) return;
+    if (!g_on || !((g_mask >> id) & 1u)) return;
     std::lock_guard<std::mutex> lk(g_mu);
     g_pending[id] = take_event();
     cudaEventRecord(g_pending[id], st);
@@ -45,7 +46,7 @@ void profile_begin(int id, cudaStream_t st)
 
 void profile_end(int id, cudaStream_t st)
 {
-    if (!g_on) return;
+    if (!g_on || !((g_mask >> id) & 1u)) return;
     std::lock_guard<std::mutex> lk(g_mu);
     cudaEvent_t b = take_event();
     cudaEventRecord(b, st);
@@ -63,6 +64,14 @@ int mc_profile_enable(int on)
     std::lock_guard<std::mutex> lk(g_mu);
     int old = g_on;
     g_on = on != 0;
+    return old;
+}
+
+unsigned mc_profile_select(unsigned mask)
+{
+    std::lock_guard<std::mutex> lk(g_mu);
+    const unsigned old = g_mask;
+    g_mask = mask;
     return old;
 }
 
