@@ -12,7 +12,7 @@
 //                      streams per 128-column step one ring stage
 //                      [activation image 32 KB][packed weights of both streams]
 //                      with cp.async.bulk;
-//   converter warps 0-3 turn the packed codes (the decode path's layout) into
+//   converter warps (8) turn the packed codes (the decode path's layout) into
 //                      fp16 (q - z) s and store them into tensor memory with
 //                      tcgen05.st 16x256b, whose thread -> (lane, column) order is
 //                      the mma fragment order the packed tiles are stored in;
@@ -39,8 +39,10 @@ constexpr int kGSlots = 4;
 constexpr int kGHdr = 1024;
 constexpr int kGStaging = kImgBytes;               // epilogue staging of one h image
 constexpr size_t kGSmem = kGHdr + (size_t)kGSlots * kGStage + kGStaging;
-constexpr int kGConv0 = 0, kGEpi0 = 4, kGProd = 8, kGMma = 9;
-constexpr int kGThreads = 10 * 32;
+// warps 0-3 and 8-11 convert (warp w: tensor-memory lanes 32 (w % 4) + 16 (w / 8)
+// .. +15, one 16-row tile per stream), 4-7 run the epilogue, 12 produces, 13 issues MMAs
+constexpr int kGEpi0 = 4, kGProd = 12, kGMma = 13, kGConv = 8;
+constexpr int kGThreads = 14 * 32;
 constexpr int kGRuns = kMaxE;
 constexpr int kGItemRing = 8;
 static_assert(kGStage % 1024 == 0, "stage alignment");
@@ -265,10 +267,10 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
     if (threadIdx.x == 0) {
         for (int s = 0; s < kGSlots; ++s) {
             mbar_init(&sh->full[s], 1);
-            mbar_init(&sh->empty[s], 1 + 4);  // MMA commit + converter warps
+            mbar_init(&sh->empty[s], 1 + kGConv);  // MMA commit + converter warps
         }
         for (int b = 0; b < 2; ++b) {
-            mbar_init(&sh->afull[b], 4);
+            mbar_init(&sh->afull[b], kGConv);
             mbar_init(&sh->aempty[b], 1);
         }
         mbar_init(&sh->dfull, 1);
@@ -368,10 +370,10 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
                 }
             }
         }
-    } else if (warp < kGEpi0) {
+    } else if (warp < kGEpi0 || (warp >= 8 && warp < 12)) {
         // ---------------------------------------------------------- converters --
-        // warp q: tensor-memory lanes 32q .. 32q+31 = rows of tiles 2q, 2q+1
-        const int q = warp - kGConv0;
+        // tensor-memory lanes 32q + 16 u2 .. +15 = the rows of tile 2q + u2
+        const int q = warp & 3, u2 = warp >> 3;
         for (int it = 0;; ++it) {
             const int slot = it % kGSlots, b = it & 1;
             if (!g_wait(&sh->full[slot], (it / kGSlots) & 1, p, sh)) break;
@@ -383,12 +385,11 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
             const int nstream = W13 ? 2 : w2_pair_width(st.u, nrb);
             const uint8_t *w = ring + (size_t)slot * kGStage + kImgBytes;
             const uint32_t abuf = tbase + 256u + 128u * (uint32_t)b;
-            for (int x = 0; x < nstream; ++x)
-                for (int u2 = 0; u2 < 2; ++u2) {
-                    const uint8_t *tile = w + x * STB + (2 * q + u2) * TB;
-                    const uint32_t taddr = abuf + 64u * (uint32_t)x + ((uint32_t)(32 * q + 16 * u2) << 16);
-                    convert_store<GPT>(tile, bits, lane, taddr);
-                }
+            for (int x = 0; x < nstream; ++x) {
+                const uint8_t *tile = w + x * STB + (2 * q + u2) * TB;
+                const uint32_t taddr = abuf + 64u * (uint32_t)x + ((uint32_t)(32 * q + 16 * u2) << 16);
+                convert_store<GPT>(tile, bits, lane, taddr);
+            }
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
