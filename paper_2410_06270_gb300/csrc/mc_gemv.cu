@@ -76,7 +76,7 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, co
     if (mbar_try_wait(bar, parity)) return true;
     uint64_t t0 = globaltimer_ns();
     while (true) {
-        if (mbar_try_wait(bar, parity)) return true;
+        if (mbar_try_wait_sleep(bar, parity, kWaitHintNs)) return true;
         if (sh->abort) return false;
         if (globaltimer_ns() - t0 > p.timeout_ns) {
             set_status(p.status, MC_ERR_TIMEOUT);

@@ -60,7 +60,7 @@ __device__ __forceinline__ bool tc_wait(uint64_t *bar, uint32_t parity, const Ex
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     while (true) {
-        if (mbar_try_wait(bar, parity)) return true;
+        if (mbar_try_wait_sleep(bar, parity, kWaitHintNs)) return true;
         if (sh->abort) return false;
         if (globaltimer_ns() - t0 > p.timeout_ns) {
             set_status(p.status, MC_ERR_TIMEOUT);
