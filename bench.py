@@ -8,7 +8,8 @@ quoted on.  A step is one mc_moe_forward (gate, top-2, ODP, permutation, W1|W3
 GEMV + SwiGLU, W2 GEMV, combine) on resident device inputs.  Packed weights
 rotate over several device copies so that no step finds its weights in L2.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload decode16|decode1|decode4|prefill4096]
+  python bench.py [--gpus N] [--steps K] [--warmup W]
+                  [--workload decode16|decode1|decode4|prefill4096|odp256|odp256_b16|odp256_b13]
   python bench.py --impl reference ...   (the CPU oracle on the host cores)
 
 Under torchrun every rank runs an independent replica (the layer does not need a
@@ -34,7 +35,10 @@ import synth  # noqa: E402
 
 METRIC = "Mixed-bit MoE-layer tokens/s; % HBM roofline (decode), % TC peak (prefill)"
 WORKLOADS = {"decode16": ("decode", 16), "decode4": ("decode", 4), "decode1": ("decode", 1),
-             "prefill4096": ("prefill", 4096)}
+             "prefill4096": ("prefill", 4096),
+             "odp256": ("odp", 256), "odp256_b16": ("odp", 256), "odp256_b13": ("odp", 256)}
+ODP_BITS = {"odp256": 20, "odp256_b16": 16, "odp256_b13": 13}
+ODP_PRUNE = 0.15  # fraction of unprotected tokens whose secondary expert the threshold drops
 
 
 def _peaks():
@@ -148,6 +152,11 @@ def run_reference(args):
     if rank != 0:
         return 0
     kind, T, L = _workload(args.workload)
+    if kind == "odp":
+        import oracle
+        _, w, _ = oracle.route(L.x_f32(), L.gate_f32(), 0.0, L.protect)
+        ratio = w[:, 1].astype(np.float64) / w[:, 0]
+        L.mu = float(np.quantile(ratio[L.protect == 0], ODP_PRUNE))
     steps = args.steps if args.steps else 3
     vals = []
     cb = None
@@ -171,14 +180,35 @@ def run_reference(args):
 
 def _workload(name):
     kind, T = WORKLOADS[name]
-    L = synth.config_decode(T=T) if kind == "decode" else synth.config_prefill(T=T)
+    if kind == "decode":
+        L = synth.config_decode(T=T)
+    elif kind == "prefill":
+        L = synth.config_prefill(T=T)
+    else:
+        L = synth.config_odp(T=T, bits_total=ODP_BITS[name])
     return kind, T, L
 
 
 def _describe(kind, T, L):
+    if kind == "odp":
+        odp = "ODP on (mu %.4g: drops the secondary expert of %d%% of unprotected tokens), %d%% of tokens " \
+              "protected by the importance surrogate" % (L.mu, round(100 * ODP_PRUNE),
+                                                         round(100 * float(L.protect.mean())))
+    else:
+        odp = "ODP off"
     return ("mixtral-8x7b MoE layer %s, %d tokens, H 4096, F 14336, 8 experts, top-2, group 128, bits %s "
-            "(mean %.2f), ODP off%s" % (kind, T, list(map(int, L.bits)), L.mean_bits(),
-                                         ", expert loads skewed ~4:1" if kind == "prefill" else ""))
+            "(mean %.2f), %s%s" % (kind, T, list(map(int, L.bits)), L.mean_bits(), odp,
+                                   ", expert loads skewed ~4:1" if kind == "prefill" else ""))
+
+
+def _odp_threshold(mc, x, gw, shape, protect_np, protect_dev):
+    """mu that prunes ODP_PRUNE of the unprotected tokens, from the library's own
+    routing weights at mu = 0 (w1/w0 per token)."""
+    r = mc.route(x, gw, shape, 0.0, protect_dev)
+    w = r["w"].cpu().numpy().astype(np.float64)
+    ratio = w[:, 1] / w[:, 0]
+    free = ratio[protect_np == 0] if protect_np is not None else ratio
+    return float(np.quantile(free, ODP_PRUNE))
 
 
 def _traffic(kernel, workload):
@@ -207,7 +237,7 @@ def run(args):
         dist.init_process_group("nccl")
     dev = torch.device("cuda", local)
     kind, T, L = _workload(args.workload)
-    steps = args.steps if args.steps else (2000 if kind == "decode" else 100)
+    steps = args.steps if args.steps else {"decode": 2000, "odp": 1000, "prefill": 100}[kind]
     shape = mc.Shape(L.E, L.H, L.F, L.group)
     flat = lambda a: [a[e][m] for e in range(L.E) for m in range(3)]
     packed_host = mc.pack_experts_host(shape, L.bits, flat(L.codes), flat(L.scale), flat(L.zero))
@@ -216,14 +246,18 @@ def run(args):
     packed = [torch.from_numpy(packed_host).to(dev) for _ in range(nsets)]
     x = torch.from_numpy(L.x.view(np.int16).copy()).view(torch.bfloat16).to(dev)
     gw = torch.from_numpy(L.gate.view(np.int16).copy()).view(torch.bfloat16).to(dev)
+    prot = None if L.protect is None else torch.from_numpy(L.protect.copy()).to(dev)
+    if kind == "odp":
+        L.mu = _odp_threshold(mc, x, gw, shape, L.protect, prot)
+    mu = float(L.mu)
     ws = mc.alloc_workspace(shape, T, dev)
     y = torch.empty_like(x)
 
     def step(i):
-        return mc.moe_forward(x, gw, shape, L.bits, packed[i % nsets], 0.0, None, y=y, workspace=ws)
+        return mc.moe_forward(x, gw, shape, L.bits, packed[i % nsets], mu, prot, y=y, workspace=ws)
 
     # routing once, to know which experts a step touches and how many pairs it keeps (fixed inputs)
-    _, r = mc.moe_forward(x, gw, shape, L.bits, packed[0], 0.0, None, y=y, workspace=ws, routing=True)
+    _, r = mc.moe_forward(x, gw, shape, L.bits, packed[0], mu, prot, y=y, workspace=ws, routing=True)
     mc.check_status(ws)
     idx = r["idx"].cpu().numpy()
     pairs = int(2 * T - int(r["pruned"].sum().item()))
@@ -231,7 +265,7 @@ def run(args):
     alg_bytes, w13_bytes = _algorithmic_bytes(shape, L.bits, touched, T, L.H)
     w13_flops = 4.0 * L.H * L.F * pairs          # W1 and W3: 2 x (2 H F) per kept pair
     layer_flops = 6.0 * L.H * L.F * pairs + 2.0 * L.H * L.E * T
-    rk = "gemv_w13" if kind == "decode" else "gemm_w13"
+    rk = "gemv_w13" if 2 * T < 512 else "gemm_w13"  # the path mc_moe_forward picks
 
     clocks = Clocks(local)
     clocks.start()
@@ -296,7 +330,7 @@ def run(args):
     avg = k_ms / max(k_n, 1)
     value = world * T * steps / (ms * 1e-3)
     e2e = world * T * steps / (ms_e2e * 1e-3)
-    if kind == "decode":
+    if rk == "gemv_w13":
         achieved = w13_bytes / (avg * 1e-3) / 1e9 if avg > 0 else None
         layer_gbs = alg_bytes * steps / (ms * 1e-3) / 1e9
         roof = {"bound": "hbm", "kernel": rk, "achieved": achieved, "peak": hbm, "unit": "GB/s",
@@ -313,7 +347,9 @@ def run(args):
                                if src == "measured" else src,
                 "frac_of_burst_peak": (achieved / bf16) if achieved else None,
                 "algorithmic_flops_per_launch": w13_flops, "layer_tflops": layer_tf,
-                "layer_frac": layer_tf / sustained, "kept_pairs": pairs}
+                "layer_frac": layer_tf / sustained, "kept_pairs": pairs,
+                "layer_gbs": alg_bytes * steps / (ms * 1e-3) / 1e9,
+                "layer_hbm_frac": alg_bytes * steps / (ms * 1e-3) / 1e9 / hbm}
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": steps,
         "warmup": args.warmup, "ms_per_step": ms / steps, "higher_is_better": True, "scaling": "weak",

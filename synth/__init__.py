@@ -223,6 +223,31 @@ def config_decode(T=16, seed=1236, bits_total=20):
     return make_layer(T, MIXTRAL_H, MIXTRAL_F, MIXTRAL_E, 128, bits, seed)
 
 
+def importance_protect(x_bits, frac, seed):
+    """Protect mask of the ODP workload: the top `frac` of tokens by a seeded
+    importance surrogate, the L1 norm of the token's activations times a uniform
+    draw standing in for its attention mass (ties to the lower index).  Input
+    generation only: the mask is an input of the layer."""
+    x = bf16_bits_to_f32(x_bits)
+    score = np.abs(x).sum(axis=1, dtype=np.float64) * _rng(seed, 5).random(x.shape[0])
+    n = int(np.ceil(frac * x.shape[0]))
+    order = np.lexsort((np.arange(x.shape[0]), -score))  # score descending, index ascending
+    protect = np.zeros(x.shape[0], np.uint8)
+    protect[order[:n]] = 1
+    return protect
+
+
+def config_odp(T=256, seed=1238, bits_total=20, protect_frac=0.10):
+    """Mixtral-8x7b-shaped layer for ODP: 256 tokens, 10% protected by the
+    importance surrogate, bits with sum 20 / 16 / 13 (mean 2.5 / 2.0 / 1.6).  The
+    prune threshold mu is set by the caller from the layer's own routing (the
+    value that prunes ~15% of the unprotected tokens' secondary experts)."""
+    bits = bit_table(seed, 8, bits_total)
+    L = make_layer(T, MIXTRAL_H, MIXTRAL_F, MIXTRAL_E, 128, bits, seed)
+    L.protect = importance_protect(L.x, protect_frac, seed)
+    return L
+
+
 def config_prefill(T=4096, seed=1237, bits_total=20, skew=(3.0, 0.9)):
     """Mixtral-8x7b-shaped prefill layer with skewed expert loads, ODP off."""
     bits = bit_table(seed, 8, bits_total)
