@@ -216,6 +216,8 @@ __device__ __forceinline__ void cvt3(const uint32_t (&w)[6], int qd, uint32_t (&
     for (int i = 0; i < 8; ++i) r[i] = cvt3_pair(w, 8 * qd + i);
 }
 
-__device__ __forceinline__ float silu(float g) { return g / (1.0f + __expf(-g)); }
+// silu(g) = g / (1 + e^-g); the fast reciprocal-based division returns 0 once
+// e^-g overflows, which is the function's limit there.
+__device__ __forceinline__ float silu(float g) { return __fdividef(g, 1.0f + __expf(-g)); }
 
 }  // namespace mc

@@ -240,6 +240,16 @@ __device__ __forceinline__ void tmem_ld_x16(uint32_t taddr, float (&v)[16])
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+__device__ __forceinline__ void tmem_ld_x16_nowait(uint32_t taddr, uint32_t (&r)[16])
+{
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+}
+
 // Epilogue warps meet (bounded); false once the CTA aborted.
 __device__ __forceinline__ bool epi_sync(const ExpertParams &p, GShared *sh, int lane, int &uses)
 {
@@ -455,19 +465,34 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
             const GItem gi = sh->items[ic % kGItemRing];
             const uint32_t lane_addr = (uint32_t)(32 * ew) << 16;
             if (W13) {
+                // h of the thread's row for all 128 pairs, packed, so that D is released
+                // before the image is written
+                uint32_t hp[kGN / 2];
                 bool bad = false;
-                for (int n0 = 0; n0 < kGN; n0 += 16) {
-                    float g[16], v[16];
-                    tmem_ld_x16(tbase + lane_addr + (uint32_t)n0, g);
-                    tmem_ld_x16(tbase + lane_addr + 128u + (uint32_t)n0, v);
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const float h = silu(g[i]) * v[i];
-                        bad |= !(fabsf(h) <= 65504.f);
-                        *reinterpret_cast<__half *>(staging + img_off(n0 + i, row)) = __float2half_rn(h);
+                for (int n0 = 0; n0 < kGN; n0 += 16) {
+                    uint32_t g[16], v[16];
+                    tmem_ld_x16_nowait(tbase + lane_addr + (uint32_t)n0, g);
+                    tmem_ld_x16_nowait(tbase + lane_addr + 128u + (uint32_t)n0, v);
+                    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+                    for (int i = 0; i < 16; i += 2) {
+                        const float h0 = silu(__uint_as_float(g[i])) * __uint_as_float(v[i]);
+                        const float h1 = silu(__uint_as_float(g[i + 1])) * __uint_as_float(v[i + 1]);
+                        bad |= !(fabsf(h0) <= 65504.f) || !(fabsf(h1) <= 65504.f);
+                        hp[(n0 + i) / 2] = h2_bits(__floats2half2_rn(h0, h1));
                     }
                 }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sh->dempty);
                 if (bad) set_status(p.status, MC_ERR_RANGE);
+#pragma unroll
+                for (int i = 0; i < kGN / 2; ++i) {
+                    const __half2 h = bits_h2(hp[i]);
+                    *reinterpret_cast<__half *>(staging + img_off(2 * i, row)) = __low2half(h);
+                    *reinterpret_cast<__half *>(staging + img_off(2 * i + 1, row)) = __high2half(h);
+                }
             } else {
                 const int nstream = w2_pair_width(gi.u, nrb);
                 for (int x = 0; x < nstream; ++x) {
@@ -482,9 +507,11 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
                     }
                 }
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&sh->dempty);
+            if (!W13) {
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sh->dempty);
+            }
             if (W13) {
                 // the image of W2's column step gi.u for token block gi.k
                 if (!epi_sync(p, sh, lane, uses)) break;
