@@ -15,6 +15,8 @@ function states the passage of the paper it follows:
 * ``expert``                    -- the Mixtral SwiGLU expert E_i of Eq. 1.
 * ``moe_layer``                 -- Eq. 1 with Eq. 5.
 * ``rmsnorm``                   -- the normalisation between stacked layers.
+* ``stack``                     -- pre-norm residual layers h <- h + MoE(RMSNorm(h)),
+  each result rounded to bf16 where the stacked workload stores bf16.
 
 Parity status: every function is pinned by ``tests/test_oracle_pins.py`` (closed
 forms, library routines, brute force and invariants); none is "parity unpinned".
@@ -210,3 +212,29 @@ def rmsnorm(x, gamma, eps: float = 1e-5) -> np.ndarray:
     out = np.empty_like(x)
     _load().mco_rmsnorm(_ptr(x), _ptr(g), x.shape[0], float(eps), _ptr(out))
     return out
+
+
+def bf16_round(a) -> np.ndarray:
+    """Round to the nearest bf16 (ties to even), returned as fp64."""
+    f = np.ascontiguousarray(a, dtype=np.float64).astype(np.float32)
+    u = f.view(np.uint32).astype(np.uint64)
+    r = ((u + 0x7FFF + ((u >> 16) & 1)) >> 16).astype(np.uint32) << 16
+    return r.astype(np.uint32).view(np.float32).astype(np.float64)
+
+
+def stack(x, gates, mats, mus, protect=None, eps: float = 1e-5, gamma=None):
+    """Pre-norm residual stack for the rows of x (bf16 values): per layer l,
+    xn = bf16(RMSNorm(h)), y = bf16(MoE_l(xn)) with gate l and threshold mus[l],
+    h = bf16(h + y).  Every token's trajectory is independent.  Returns
+    (h after the last layer fp64 [T, H], per-layer (idx, w, pruned) list)."""
+    h = bf16_round(x)
+    T, H = h.shape
+    g = np.ones(H, np.float32) if gamma is None else gamma
+    routes = []
+    for wg, mu in zip(gates, mus):
+        xn = bf16_round(np.stack([rmsnorm(h[t], g, eps) for t in range(T)]))
+        y, idx, w, pr = moe_layer(xn, wg, mats, mu, protect)
+        h = bf16_round(h + bf16_round(y))
+        routes.append((idx, w, pr))
+    return h, routes
+

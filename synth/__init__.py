@@ -248,6 +248,21 @@ def config_odp(T=256, seed=1238, bits_total=20, protect_frac=0.10):
     return L
 
 
+def config_stack(T=32, layers=32, seed=1239, bits_total=20, protect_frac=0.10, H=MIXTRAL_H, F=MIXTRAL_F,
+                 E=MIXTRAL_E, group=128, gate_std=0.02):
+    """A stack of `layers` pre-norm MoE layers (h <- h + MoE(RMSNorm(h)), RMSNorm
+    weight 1): one seeded expert-weight set shared by every layer (the caller
+    stores one device copy per layer, so each layer streams its own weights),
+    a distinct seeded gate per layer, 10% of tokens protected by the importance
+    surrogate.  Returns (layer, gates): `layer` carries x, the experts and the
+    protect mask; gates[l] is layer l's gate (bf16 bits [E, H])."""
+    bits = bit_table(seed, E, bits_total)
+    L = make_layer(T, H, F, E, group, bits, seed, gate_std=gate_std)
+    L.protect = importance_protect(L.x, protect_frac, seed)
+    gates = [gaussian_bf16(seed, (6, l), (E, H), gate_std) for l in range(layers)]
+    return L, gates
+
+
 def config_prefill(T=4096, seed=1237, bits_total=20, skew=(3.0, 0.9)):
     """Mixtral-8x7b-shaped prefill layer with skewed expert loads, ODP off."""
     bits = bit_table(seed, 8, bits_total)

@@ -320,3 +320,50 @@ def test_rmsnorm_textbook():
     xt = torch.tensor(x)
     want = (xt * torch.rsqrt((xt * xt).mean() + 1e-5) * torch.tensor(g, dtype=torch.float64)).numpy()
     np.testing.assert_allclose(oracle.rmsnorm(x, g), want, rtol=1e-12)
+
+
+# -------------------------------------------------------------- stacking ----
+
+def test_bf16_round_matches_library_cast():
+    x = np.concatenate([np.random.default_rng(16).standard_normal(2000) * 10.0 ** np.arange(-4, 4).repeat(250),
+                        [1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8, -(1.0 + 2.0 ** -8), 0.0]])
+    want = torch.tensor(x, dtype=torch.float32).to(torch.bfloat16).double().numpy()
+    np.testing.assert_array_equal(oracle.bf16_round(x), want)
+
+
+def test_stack_with_zero_experts_is_identity():
+    """Experts whose every weight is zero (codes equal to the zero point) add
+    nothing: any number of layers returns the bf16 input."""
+    L = _rand_layer(bits=(2, 2, 2, 2))
+    for e in range(L.E):
+        for m in range(3):
+            L.codes[e][m][:] = 1
+            L.zero[e][m][:] = 1.0
+    gates = [synth.gaussian_bf16(3, (l,), (L.E, L.H), 0.1) for l in range(3)]
+    h, _ = oracle.stack(L.x_f32(), [synth.bf16_bits_to_f32(g) for g in gates], _mats(L), [0.0, 0.3, 0.0])
+    np.testing.assert_array_equal(h, L.x_f32().astype(np.float64))
+
+
+def test_stack_composes_layer_by_layer():
+    L = _rand_layer(T=6, bits=(3, 1, 2, 2))
+    gates = [synth.bf16_bits_to_f32(synth.gaussian_bf16(4, (l,), (L.E, L.H), 0.1)) for l in range(2)]
+    mats = _mats(L)
+    both, routes = oracle.stack(L.x_f32(), gates, mats, [0.2, 0.0], L.protect)
+    first, r0 = oracle.stack(L.x_f32(), gates[:1], mats, [0.2], L.protect)
+    second, r1 = oracle.stack(first, gates[1:], mats, [0.0], L.protect)
+    np.testing.assert_array_equal(both, second)
+    np.testing.assert_array_equal(routes[1][0], r1[0][0])
+
+
+def test_stack_one_layer_is_residual_of_normalised_layer():
+    """One layer with every rounding written out: bf16(x + bf16(MoE(bf16(RMSNorm x))))."""
+    L = _rand_layer(T=5, bits=(2, 3, 1, 2))
+    g = synth.bf16_bits_to_f32(synth.gaussian_bf16(5, (0,), (L.E, L.H), 0.1))
+    x = L.x_f32().astype(np.float64)
+    rms = np.sqrt((x * x).mean(axis=1, keepdims=True) + 1e-5)
+    xn = torch.tensor(x / rms, dtype=torch.float32).to(torch.bfloat16).double().numpy()
+    y, *_ = oracle.moe_layer(xn, g, _mats(L), 0.0)
+    yb = torch.tensor(y, dtype=torch.float32).to(torch.bfloat16).double().numpy()
+    want = torch.tensor(x + yb, dtype=torch.float32).to(torch.bfloat16).double().numpy()
+    h, _ = oracle.stack(L.x_f32(), [g], _mats(L), [0.0])
+    np.testing.assert_array_equal(h, want)
