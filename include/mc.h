@@ -186,6 +186,26 @@ int mc_moe_forward_static(const void *x, const void *gate_w, int T, const mc_sha
                           const int8_t *bits_host, const void *packed_dev, float mu,
                           const uint8_t *protect, void *y, int32_t *status_dev, void *stream);
 
+/* Workspace bytes of mc_stack_forward for up to T_max tokens: the layer
+ * workspace (status word first) followed by two [T_max, H] bf16 activations. */
+size_t mc_stack_workspace_size(const mc_shape *shape, int T_max);
+
+/* A stack of `layers` pre-norm residual MoE blocks, the structure of the
+ * Mixtral models the paper compresses (Sec. 3.1 model table: 32 MoE layers):
+ *   for l in 0 .. layers-1:  h <- h + MoE_l(RMSNorm_l(h))
+ * MoE_l is mc_moe_forward with gate_w[l] (device bf16 [E, H]), packed_dev[l],
+ * the bit table bits_host[l*E .. l*E+E-1] and threshold mu_host[l]; RMSNorm_l
+ * uses gamma + l*H (device bf16 [layers, H]) and eps.  h (device bf16 [T, H]) is
+ * updated in place; every intermediate is bf16.  protect (device [T] or NULL)
+ * applies to every layer.  Device-detected faults of any layer go to the status
+ * word at the start of `workspace` (mc_check_status).  All launches go to
+ * `stream` and none synchronises, so a caller may capture one call into a CUDA
+ * graph (after a first call has set the kernels' shared-memory attributes). */
+int mc_stack_forward(void *h, int T, const mc_shape *shape, int layers, const void *const *gate_w,
+                     const int8_t *bits_host, const void *const *packed_dev, const float *mu_host,
+                     const uint8_t *protect, const void *gamma, float eps, void *workspace,
+                     size_t ws_bytes, void *stream);
+
 /* Choose the expert path of mc_moe_forward: 0 = automatic (the GEMV below 512
  * kept-or-not pairs, 2T < 512, else the GEMM), 1 = the mma.sync grouped GEMV
  * (decode), 2 = the tcgen05 grouped GEMV with chunks of 16 pairs, 3 = the

@@ -226,7 +226,7 @@ def stack(x, gates, mats, mus, protect=None, eps: float = 1e-5, gamma=None):
     """Pre-norm residual stack for the rows of x (bf16 values): per layer l,
     xn = bf16(RMSNorm(h)), y = bf16(MoE_l(xn)) with gate l and threshold mus[l],
     h = bf16(h + y).  Every token's trajectory is independent.  Returns
-    (h after the last layer fp64 [T, H], per-layer (idx, w, pruned) list)."""
+    (h after the last layer fp64 [T, H], per-layer (idx, w, pruned, layer input xn))."""
     h = bf16_round(x)
     T, H = h.shape
     g = np.ones(H, np.float32) if gamma is None else gamma
@@ -235,6 +235,6 @@ def stack(x, gates, mats, mus, protect=None, eps: float = 1e-5, gamma=None):
         xn = bf16_round(np.stack([rmsnorm(h[t], g, eps) for t in range(T)]))
         y, idx, w, pr = moe_layer(xn, wg, mats, mu, protect)
         h = bf16_round(h + bf16_round(y))
-        routes.append((idx, w, pr))
+        routes.append((idx, w, pr, xn))
     return h, routes
 

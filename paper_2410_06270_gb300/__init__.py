@@ -63,6 +63,8 @@ def load():
         "mc_moe_workspace_size": (Z, [S, I]),
         "mc_moe_forward": (I, [P, P, I, S, P, P, F32, P, P, P, Z, P, P, P, P]),
         "mc_moe_forward_static": (I, [P, P, I, S, P, P, F32, P, P, P, P]),
+        "mc_stack_workspace_size": (Z, [S, I]),
+        "mc_stack_forward": (I, [P, I, S, I, P, P, P, P, P, P, F32, P, Z, P]),
         "mc_set_path": (I, [I]),
         "mc_set_debug": (I, [I, ctypes.c_ulonglong]),
         "mc_check_status": (I, [P, P]),
@@ -277,6 +279,38 @@ def moe_forward_static(x, gate_w, shape: Shape, bits, packed_dev, mu: float = 0.
                                         _ptr(packed_dev), float(mu), _ptr(protect), _ptr(y), _ptr(status),
                                         _stream()))
     return y
+
+
+def stack_workspace(shape: Shape, T: int, device="cuda"):
+    import torch
+    n = load().mc_stack_workspace_size(ctypes.byref(shape), int(T))
+    if n == 0:
+        raise MCError(ERR_INVALID_ARG, last_error())
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+class StackArgs:
+    """Host-side argument arrays of mc_stack_forward, built once per stack so that
+    repeated calls (or a captured graph) reuse the same host memory."""
+
+    def __init__(self, gates, bits, packed, mus):
+        self.layers = len(gates)
+        self.gate_ptrs = (ctypes.c_void_p * self.layers)(*[g.data_ptr() for g in gates])
+        self.packed_ptrs = (ctypes.c_void_p * self.layers)(*[p.data_ptr() for p in packed])
+        self.bits = np.ascontiguousarray(np.concatenate([_bits(b) for b in bits]), dtype=np.int8)
+        self.mus = np.ascontiguousarray(mus, dtype=np.float32)
+        self._keep = (gates, packed)
+
+
+def stack_forward(h, shape: Shape, args: StackArgs, gamma, workspace, protect=None, eps: float = 1e-5):
+    """mc_stack_forward: h (bf16 [T,H], device) updated in place."""
+    T = h.shape[0]
+    _check(load().mc_stack_forward(_ptr(h), T, ctypes.byref(shape), args.layers,
+                                   ctypes.cast(args.gate_ptrs, ctypes.c_void_p), args.bits.ctypes.data,
+                                   ctypes.cast(args.packed_ptrs, ctypes.c_void_p), args.mus.ctypes.data,
+                                   _ptr(protect), _ptr(gamma), float(eps), _ptr(workspace), workspace.numel(),
+                                   _stream()))
+    return h
 
 
 def check_status(workspace) -> None:
