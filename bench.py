@@ -9,7 +9,7 @@ GEMV + SwiGLU, W2 GEMV, combine) on resident device inputs.  Packed weights
 rotate over several device copies so that no step finds its weights in L2.
 
   python bench.py [--gpus N] [--steps K] [--warmup W]
-                  [--workload decode16|decode1|decode4|prefill4096|odp256|odp256_b16|odp256_b13]
+                  [--workload decode16|decode1|decode4|prefill4096|odp256|odp256_b16|odp256_b13|stack32]
   python bench.py --impl reference ...   (the CPU oracle on the host cores)
 
 Under torchrun every rank runs an independent replica (the layer does not need a
@@ -36,7 +36,9 @@ import synth  # noqa: E402
 METRIC = "Mixed-bit MoE-layer tokens/s; % HBM roofline (decode), % TC peak (prefill)"
 WORKLOADS = {"decode16": ("decode", 16), "decode4": ("decode", 4), "decode1": ("decode", 1),
              "prefill4096": ("prefill", 4096),
-             "odp256": ("odp", 256), "odp256_b16": ("odp", 256), "odp256_b13": ("odp", 256)}
+             "odp256": ("odp", 256), "odp256_b16": ("odp", 256), "odp256_b13": ("odp", 256),
+             "stack32": ("stack", 32)}
+STACK_LAYERS = 32
 ODP_BITS = {"odp256": 20, "odp256_b16": 16, "odp256_b13": 13}
 ODP_PRUNE = 0.15  # fraction of unprotected tokens whose secondary expert the threshold drops
 
@@ -147,11 +149,57 @@ def cpu_baseline(L, budget_s=12.0, threads=None):
                       % (n, L.T)}
 
 
+def cpu_baseline_stack(L, gates, mus, budget_s=12.0, threads=None):
+    """The oracle's 32-layer stack on a bounded sample of the workload's tokens
+    (one token's whole trajectory per host thread)."""
+    import concurrent.futures as cf
+
+    import oracle
+    mats = [[oracle.QMat(*L.mat_shape(m), L.group, int(L.bits[e]), L.codes[e][m], L.scale[e][m], L.zero[e][m])
+             for m in range(3)] for e in range(L.E)]
+    gf = [synth.bf16_bits_to_f32(g) for g in gates]
+    xf = L.x_f32()
+    run = lambda t: oracle.stack(xf[t:t + 1], gf, mats, mus, L.protect[t:t + 1])
+    cores = threads or (os.cpu_count() or 1)
+    t0 = time.perf_counter()
+    run(0)
+    one = time.perf_counter() - t0
+    n = int(max(1, min(L.T, cores, round(budget_s / max(one, 1e-3) * cores / 2))))
+    t0 = time.perf_counter()
+    with cf.ThreadPoolExecutor(min(n, cores)) as ex:
+        list(ex.map(run, range(n)))
+    dt = time.perf_counter() - t0
+    return {"value": n / dt, "unit": "tokens/s", "cores": min(n, cores), "kind": "oracle",
+            "sample": "%d of the workload's %d tokens (all %d layers per token, fp64, one token per thread)"
+                      % (n, L.T, len(gates))}
+
+
+def _stack_mus_oracle(L, gates):
+    """Per-layer thresholds from the oracle's own trajectory at mu = 0 (the
+    reference arm's counterpart of the calibration in run_stack)."""
+    import oracle
+    mats = [[oracle.QMat(*L.mat_shape(m), L.group, int(L.bits[e]), L.codes[e][m], L.scale[e][m], L.zero[e][m])
+             for m in range(3)] for e in range(L.E)]
+    gf = [synth.bf16_bits_to_f32(g) for g in gates]
+    xf = L.x_f32()
+    mus = []
+    sample = list(range(min(L.T, 8)))
+    _, routes = oracle.stack(xf[sample], gf, mats, [0.0] * len(gates), L.protect[sample])
+    for (idx, w, pr, xn) in routes:
+        ratio = w[:, 1].astype(np.float64) / w[:, 0]
+        free = ratio[L.protect[sample] == 0]
+        mus.append(float(np.quantile(free if free.size else ratio, ODP_PRUNE)))
+    return mus
+
+
 def run_reference(args):
     world, rank, _ = _dist()
     if rank != 0:
         return 0
     kind, T, L = _workload(args.workload)
+    if kind == "stack":
+        L, gates = L
+        mus = _stack_mus_oracle(L, gates)
     if kind == "odp":
         import oracle
         _, w, _ = oracle.route(L.x_f32(), L.gate_f32(), 0.0, L.protect)
@@ -162,7 +210,7 @@ def run_reference(args):
     cb = None
     budget = min(4.0, 150.0 / (args.warmup + steps))  # the whole run stays within a few minutes
     for i in range(args.warmup + steps):
-        r = cpu_baseline(L, budget_s=budget)
+        r = cpu_baseline_stack(L, gates, mus, budget_s=budget) if kind == "stack" else cpu_baseline(L, budget_s=budget)
         if i >= args.warmup:
             vals.append(r["value"])
             cb = r
@@ -184,12 +232,21 @@ def _workload(name):
         L = synth.config_decode(T=T)
     elif kind == "prefill":
         L = synth.config_prefill(T=T)
+    elif kind == "stack":
+        L = synth.config_stack(T=T, layers=STACK_LAYERS)
     else:
         L = synth.config_odp(T=T, bits_total=ODP_BITS[name])
     return kind, T, L
 
 
 def _describe(kind, T, L):
+    if kind == "stack":
+        L = L[0] if isinstance(L, tuple) else L
+        return ("mixtral-8x7b stack of %d pre-norm MoE layers (h <- h + MoE(RMSNorm(h))), %d tokens, H 4096, "
+                "F 14336, 8 experts, top-2, group 128, bits %s (mean %.2f), ODP on (per-layer mu dropping the "
+                "secondary expert of %d%% of unprotected tokens), %d%% of tokens protected, whole stack in one "
+                "CUDA graph" % (STACK_LAYERS, T, list(map(int, L.bits)), L.mean_bits(), round(100 * ODP_PRUNE),
+                                round(100 * float(L.protect.mean()))))
     if kind == "odp":
         odp = "ODP on (mu %.4g: drops the secondary expert of %d%% of unprotected tokens), %d%% of tokens " \
               "protected by the importance surrogate" % (L.mu, round(100 * ODP_PRUNE),
@@ -374,6 +431,140 @@ def run(args):
     return 0
 
 
+def run_stack(args):
+    """The 32-layer stack: one mc_stack_forward captured into a CUDA graph (with the
+    copy of the step's input into the residual stream), replayed K times."""
+    import torch
+    import torch.distributed as dist
+
+    import paper_2410_06270_gb300 as mc
+
+    world, rank, local = _dist()
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+    kind, T, (L, gates) = _workload(args.workload)
+    layers = len(gates)
+    steps = args.steps if args.steps else 100
+    shape = mc.Shape(L.E, L.H, L.F, L.group)
+    flat = lambda a: [a[e][m] for e in range(L.E) for m in range(3)]
+    packed_host = mc.pack_experts_host(shape, L.bits, flat(L.codes), flat(L.scale), flat(L.zero))
+    packs = [torch.from_numpy(packed_host).to(dev) for _ in range(layers)]  # every layer streams its own copy
+    bf = lambda b: torch.from_numpy(b.view(np.int16).copy()).view(torch.bfloat16).to(dev)
+    x0 = bf(L.x)
+    gw = [bf(g) for g in gates]
+    prot = torch.from_numpy(L.protect.copy()).to(dev)
+    gamma = torch.ones((layers, L.H), dtype=torch.bfloat16, device=dev)
+    # per-layer thresholds from this layer's own routing along the stack's trajectory at mu = 0
+    mus, touched = [], []
+    h = x0.clone()
+    wsl = mc.alloc_workspace(shape, T, dev)
+    for l in range(layers):
+        xn = mc.rmsnorm(h, gamma[l])
+        r = mc.route(xn, gw[l], shape, 0.0, prot)
+        w = r["w"].cpu().numpy().astype(np.float64)
+        mus.append(float(np.quantile((w[:, 1] / w[:, 0])[L.protect == 0], ODP_PRUNE)))
+        y, rr = mc.moe_forward(xn, gw[l], shape, L.bits, packs[l], mus[-1], prot, workspace=wsl, routing=True)
+        touched.append(sorted(set(rr["idx"].cpu().numpy().reshape(-1).tolist())))
+        h = mc.add(h, y)
+    mc.check_status(wsl)
+    args_s = mc.StackArgs(gw, [L.bits] * layers, packs, mus)
+    ws = mc.stack_workspace(shape, T, dev)
+    hs = x0.clone()
+    mc.stack_forward(hs, shape, args_s, gamma, ws, prot)  # sets the kernels' attributes before capture
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    cs = torch.cuda.Stream()
+    cs.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(cs):
+        with torch.cuda.graph(graph, stream=cs):
+            hs.copy_(x0)
+            mc.stack_forward(hs, shape, args_s, gamma, ws, prot)
+    torch.cuda.current_stream().wait_stream(cs)
+    alg = sum(_algorithmic_bytes(shape, L.bits, t, T, L.H)[0] for t in touched)
+
+    clocks = Clocks(local)
+    clocks.start()
+    for _ in range(args.warmup):
+        graph.replay()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_wall0 = time.time()
+    e0.record(stream)
+    for _ in range(steps):
+        graph.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    t_wall1 = time.time()
+    ms = e0.elapsed_time(e1)
+    mc.check_status(ws)
+    cl = clocks.stop((t_wall0, t_wall1))
+    # per-kernel breakdown: one eager profiled call
+    mc.profile_select(None)
+    mc.profile_enable(True)
+    mc.stack_forward(hs, shape, args_s, gamma, ws, prot)
+    torch.cuda.synchronize()
+    mc.profile_enable(False)
+    breakdown = mc.profile_read()
+    # end to end: pinned host input -> device -> graph -> host
+    xh = torch.empty(x0.shape, dtype=x0.dtype, pin_memory=True)
+    xh.copy_(x0.cpu())
+    yh = torch.empty(x0.shape, dtype=x0.dtype, pin_memory=True)
+    torch.cuda.synchronize()
+    e2, e3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e2.record(stream)
+    for _ in range(steps):
+        x0.copy_(xh, non_blocking=True)
+        graph.replay()
+        yh.copy_(hs, non_blocking=True)
+    e3.record(stream)
+    torch.cuda.synchronize()
+    ms_e2e = e2.elapsed_time(e3)
+    t_local = torch.tensor([ms, ms_e2e], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t_local, op=dist.ReduceOp.MAX)
+        dist.barrier()
+    ms, ms_e2e = float(t_local[0]), float(t_local[1])
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return 0
+    hbm, _, src = _peaks()
+    gbs = alg * steps / (ms * 1e-3) / 1e9
+    line = {
+        "metric": METRIC, "value": world * T * steps / (ms * 1e-3), "unit": "tokens/s", "n_gpus": world,
+        "steps": steps, "warmup": args.warmup, "ms_per_step": ms / steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f16 x {1,2,3}-bit codes, fp32 accumulate",
+        "data": "synthetic",
+        "config": {"workload": _describe(kind, T, L), "global_batch": T * world,
+                   "parallelism": "replicas" if world > 1 else "single",
+                   "l2": "inputs larger than L2: %d layers x %.0f MB packed weights, one device copy per layer"
+                         % (layers, packed_host.nbytes / 1e6),
+                   "weights": "one seeded expert set shared by the layers (separate copies), per-layer gates"},
+        "roofline": {"bound": "hbm", "kernel": "stack step (CUDA graph: %d layers of rmsnorm, route, permute, "
+                                                "GEMV W1|W3, GEMV W2, combine, add)" % layers,
+                     "achieved": gbs, "peak": hbm, "unit": "GB/s", "frac": gbs / hbm, "traffic": None,
+                     "peak_source": "%s (MEASURED_PEAKS.json hbm_gbs)" % src if src == "measured" else src,
+                     "algorithmic_bytes_per_step": alg},
+        "kernels_ms_per_step": {k: v[0] for k, v in breakdown.items()},
+        "e2e": {"value": world * T * steps / (ms_e2e * 1e-3), "unit": "tokens/s",
+                "h2d_bytes_per_step": int(x0.numel() * 2), "d2h_bytes_per_step": int(hs.numel() * 2)},
+        # the profiled kernels of one call plus one rmsnorm and one add launch per layer
+        "gpu_launches": (_launches_per_step(breakdown, 1) + 2 * layers) * steps,
+        "clocks": cl,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline_stack(L, gates, mus)
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
 def _launches_per_step(breakdown, n):
     return int(round(sum(c for _, c in breakdown.values()) / max(n, 1)))
 
@@ -399,6 +590,8 @@ def main():
         args.warmup = 3
     if args.impl == "reference":
         return run_reference(args)
+    if WORKLOADS[args.workload][0] == "stack":
+        return run_stack(args)
     return run(args)
 
 
