@@ -27,6 +27,8 @@ __global__ void __launch_bounds__(kRouteWarps * 32) route_kernel(RouteParams p)
     float acc[kMaxE];
 #pragma unroll
     for (int e = 0; e < kMaxE; ++e) acc[e] = 0.f;
+    // unrolled so that the loads of several 1024-column steps are in flight together
+#pragma unroll 4
     for (int c0 = 8 * (threadIdx.x); c0 < H; c0 += 8 * 32 * kRouteWarps) {
         uint4 raw = *reinterpret_cast<const uint4 *>(xr + c0);
         const __nv_bfloat162 *x2 = reinterpret_cast<const __nv_bfloat162 *>(&raw);
@@ -183,7 +185,9 @@ int launch_route(const RouteParams &rp, const PermuteParams &pp, cudaStream_t st
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "route launch: %s", cudaGetErrorString(err));
     profile_begin(kKPermute, st);
-    permute_kernel<<<1, 1024, 0, st>>>(pp);
+    // one thread per pair (whole warps), at most 1024: fewer threads to synchronise for small T
+    const int nt = min(1024, max(32, (2 * pp.T + 31) / 32 * 32));
+    permute_kernel<<<1, nt, 0, st>>>(pp);
     profile_end(kKPermute, st);
     err = cudaGetLastError();
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "permute launch: %s", cudaGetErrorString(err));
