@@ -34,7 +34,7 @@
 namespace mc {
 
 #ifndef MC_GEMV_TPW
-#define MC_GEMV_TPW 1
+#define MC_GEMV_TPW 2
 #endif
 constexpr int kTPW = MC_GEMV_TPW;            // 16-row tiles per consumer warp (1 or 2)
 constexpr int kCW = 16 / kTPW;              // consumer warps
@@ -42,7 +42,7 @@ constexpr int kGemvThreads = (kCW + 1) * 32;
 constexpr int kMaxSlots = 16;
 constexpr int kRingOff = 1024;
 #ifndef MC_GEMV_KPS
-#define MC_GEMV_KPS 2
+#define MC_GEMV_KPS 4
 #endif
 constexpr int kKPS = MC_GEMV_KPS;           // 128-column steps per ring stage
 
