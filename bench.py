@@ -115,6 +115,23 @@ def _dist():
     return world, rank, local
 
 
+def max_over_ranks(values, device="cpu"):
+    """Element-wise max of `values` over the ranks of the default process group
+    (the slowest replica's times); the values themselves without one."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor(list(values), dtype=torch.float64, device=device)
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.cpu()]
+
+
+def job_throughput(world, units_per_rank, steps, ms):
+    """Whole-job units per second: every rank processes units_per_rank per step;
+    the job takes the slowest rank's `ms` for `steps` steps."""
+    return world * units_per_rank * steps / (ms * 1e-3)
+
+
 def _algorithmic_bytes(shape, bits, touched, T, H):
     """Packed weight bytes of the touched experts (codes + fp16 scale/zero) plus
     the gate, activations and output.  Returns (total, w13 part)."""
@@ -395,11 +412,9 @@ def run(args):
     torch.cuda.synchronize()
     ms_e2e = e2.elapsed_time(e3)
 
-    t_local = torch.tensor([ms, ms_e2e], dtype=torch.float64, device=dev)
+    ms, ms_e2e = max_over_ranks([ms, ms_e2e], dev)
     if world > 1:
-        dist.all_reduce(t_local, op=dist.ReduceOp.MAX)
         dist.barrier()
-    ms, ms_e2e = float(t_local[0]), float(t_local[1])
     if rank != 0:
         if world > 1:
             dist.destroy_process_group()
@@ -408,8 +423,8 @@ def run(args):
     hbm, bf16, src = _peaks()
     k_ms, k_n = prof.get(rk, (0.0, 0))
     avg = k_ms / max(k_n, 1)
-    value = world * T * steps / (ms * 1e-3)
-    e2e = world * T * steps / (ms_e2e * 1e-3)
+    value = job_throughput(world, T, steps, ms)
+    e2e = job_throughput(world, T, steps, ms_e2e)
     if rk == "gemv_w13":
         achieved = w13_bytes / (avg * 1e-3) / 1e9 if avg > 0 else None
         layer_gbs = alg_bytes * steps / (ms * 1e-3) / 1e9
@@ -549,11 +564,9 @@ def run_stack(args):
     e3.record(stream)
     torch.cuda.synchronize()
     ms_e2e = e2.elapsed_time(e3)
-    t_local = torch.tensor([ms, ms_e2e], dtype=torch.float64, device=dev)
+    ms, ms_e2e = max_over_ranks([ms, ms_e2e], dev)
     if world > 1:
-        dist.all_reduce(t_local, op=dist.ReduceOp.MAX)
         dist.barrier()
-    ms, ms_e2e = float(t_local[0]), float(t_local[1])
     if rank != 0:
         if world > 1:
             dist.destroy_process_group()
@@ -561,7 +574,7 @@ def run_stack(args):
     hbm, _, src = _peaks()
     gbs = alg * steps / (ms * 1e-3) / 1e9
     line = {
-        "metric": METRIC, "value": world * T * steps / (ms * 1e-3), "unit": "tokens/s", "n_gpus": world,
+        "metric": METRIC, "value": job_throughput(world, T, steps, ms), "unit": "tokens/s", "n_gpus": world,
         "steps": steps, "warmup": args.warmup, "ms_per_step": ms / steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f16 x {1,2,3}-bit codes, fp32 accumulate",
         "data": "synthetic",
@@ -576,7 +589,7 @@ def run_stack(args):
                      "peak_source": "%s (MEASURED_PEAKS.json hbm_gbs)" % src if src == "measured" else src,
                      "algorithmic_bytes_per_step": alg},
         "kernels_ms_per_step": {k: v[0] for k, v in breakdown.items()},
-        "e2e": {"value": world * T * steps / (ms_e2e * 1e-3), "unit": "tokens/s",
+        "e2e": {"value": job_throughput(world, T, steps, ms_e2e), "unit": "tokens/s",
                 "h2d_bytes_per_step": int(x0.numel() * 2), "d2h_bytes_per_step": int(hs.numel() * 2)},
         # the profiled kernels of one call plus one rmsnorm and one add launch per layer
         "gpu_launches": (_launches_per_step(breakdown, 1) + 2 * layers) * steps,
