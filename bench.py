@@ -34,6 +34,7 @@ sys.path.insert(0, ROOT)
 import synth  # noqa: E402
 
 METRIC = "Mixed-bit MoE-layer tokens/s; % HBM roofline (decode), % TC peak (prefill)"
+HBM_NOMINAL_GBS = 7900.0  # GB300 HBM3e nominal, reported beside the measured copy peak
 WORKLOADS = {"decode16": ("decode", 16), "decode4": ("decode", 4), "decode1": ("decode", 1),
              "prefill4096": ("prefill", 4096),
              "odp256": ("odp", 256), "odp256_b16": ("odp", 256), "odp256_b13": ("odp", 256),
@@ -162,8 +163,9 @@ def cpu_baseline(L, budget_s=12.0, threads=None):
         list(ex.map(lambda t: oracle.moe_layer(xf, gf, mats, L.mu, L.protect, tokens=[t]), toks))
     dt = time.perf_counter() - t0
     return {"value": n / dt, "unit": "tokens/s", "cores": min(n, cores), "kind": "oracle",
-            "sample": "%d of the workload's %d tokens (full layer per token, fp64, one token per thread)"
-                      % (n, L.T)}
+            "single_thread_value": 1.0 / one,
+            "sample": "%d of the workload's %d tokens (full layer per token, fp64, one token per thread); "
+                      "single_thread_value: token 0 alone on one thread" % (n, L.T)}
 
 
 def cpu_baseline_stack(L, gates, mus, budget_s=12.0, threads=None):
@@ -187,8 +189,9 @@ def cpu_baseline_stack(L, gates, mus, budget_s=12.0, threads=None):
         list(ex.map(run, range(n)))
     dt = time.perf_counter() - t0
     return {"value": n / dt, "unit": "tokens/s", "cores": min(n, cores), "kind": "oracle",
-            "sample": "%d of the workload's %d tokens (all %d layers per token, fp64, one token per thread)"
-                      % (n, L.T, len(gates))}
+            "single_thread_value": 1.0 / one,
+            "sample": "%d of the workload's %d tokens (all %d layers per token, fp64, one token per thread); "
+                      "single_thread_value: token 0 alone on one thread" % (n, L.T, len(gates))}
 
 
 def _stack_mus_oracle(L, gates):
@@ -431,6 +434,7 @@ def run(args):
         roof = {"bound": "hbm", "kernel": rk, "achieved": achieved, "peak": hbm, "unit": "GB/s",
                 "frac": (achieved / hbm) if achieved else None, "traffic": _traffic(rk, args.workload),
                 "peak_source": "%s (MEASURED_PEAKS.json hbm_gbs)" % src if src == "measured" else src,
+                "frac_of_nominal_7900": (achieved / HBM_NOMINAL_GBS) if achieved else None,
                 "algorithmic_bytes_per_launch": w13_bytes, "layer_gbs": layer_gbs, "layer_frac": layer_gbs / hbm}
     else:
         sustained = _peak_sustained() or bf16
@@ -586,6 +590,7 @@ def run_stack(args):
         "roofline": {"bound": "hbm", "kernel": "stack step (CUDA graph: %d layers of rmsnorm, route, permute, "
                                                 "GEMV W1|W3, GEMV W2, combine, add)" % layers,
                      "achieved": gbs, "peak": hbm, "unit": "GB/s", "frac": gbs / hbm, "traffic": None,
+                     "frac_of_nominal_7900": gbs / HBM_NOMINAL_GBS,
                      "peak_source": "%s (MEASURED_PEAKS.json hbm_gbs)" % src if src == "measured" else src,
                      "algorithmic_bytes_per_step": alg},
         "kernels_ms_per_step": {k: v[0] for k, v in breakdown.items()},
