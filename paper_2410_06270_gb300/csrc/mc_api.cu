@@ -30,13 +30,31 @@ static int g_trace_steps = 0;
 
 static inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-// Column splits of the W2 pass: more CTAs for the small-batch (GEMV) case.
-static int choose_ks(const mc_shape *s, int T)
+// Column splits of the W2 GEMV pass.  The workspace holds up to kMaxKS splits
+// (decode sizes); the forward picks, among the divisors of F/128 that leave each
+// item at least two ring stages, the split count whose work items (estimated
+// chunks x 256-row block pairs x splits) fill the SMs' last wave best, the
+// smaller one on ties.
+constexpr int kMaxKS = 8;  // the combine reads one partial per split
+
+static int max_ks(const mc_shape *s, int T) { return T > 64 ? 1 : kMaxKS; }
+
+static int choose_ks(const mc_shape *s, int T, int nsm)
 {
-    if (T > 64) return 1;
-    int nt = s->F / kTileK;
-    for (int ks : {4, 2}) if (nt % ks == 0) return ks;
-    return 1;
+    const int nt = s->F / kTileK, npairs = (s->H / kBlockRows + 1) / 2;
+    const int chunks = 2 * T < s->E ? 2 * T : s->E;  // pairs land on distinct experts at small T
+    int best = 1;
+    double best_eff = -1.0;
+    for (int ks = 1; ks <= max_ks(s, T); ++ks) {
+        if (nt % ks || nt / ks < 8) continue;
+        const long items = (long)chunks * npairs * ks, waves = (items + nsm - 1) / nsm;
+        const double eff = (double)items / (double)(waves * nsm);
+        if (eff > best_eff + 1e-9) {
+            best_eff = eff;
+            best = ks;
+        }
+    }
+    return best;
 }
 
 struct Workspace {
@@ -69,7 +87,7 @@ static Workspace carve(const mc_shape *s, int T, void *base)
         off = align256(off + bytes);
         return r;
     };
-    w.KS = choose_ks(s, T);
+    w.KS = max_ks(s, T);  // room for the largest split count the forward may pick
     w.max_chunks = max_chunks_for(T, s->E);
     const size_t P = 2 * (size_t)T, MC = (size_t)w.max_chunks;
     const size_t tb = (size_t)tab_bytes(s->group);
@@ -266,7 +284,10 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     ep.himg = ws.himg;
     ep.max_blocks = ws.max_blocks;
     ep.opart = ws.opart;
-    ep.KS = path == 3 ? 1 : ws.KS;  // the GEMM's W2 pass covers all of F at once
+    int nsm = 0, dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return set_error(MC_ERR_CUDA, "device query failed");
+    ep.KS = path == 3 ? 1 : choose_ks(shape, T, nsm);  // the GEMM's W2 pass covers all of F at once
     ep.Pmax = 2 * T;
     ep.max_chunks = ws.max_chunks;
     ep.status = ws.status;
