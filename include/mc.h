@@ -145,7 +145,9 @@ int mc_route(const void *x, const void *gate_w, int T, const mc_shape *shape, fl
  *   packed_dev: the buffer written by mc_pack_experts for (shape, bits_host),
  *   mu, protect as in mc_route, y bf16 [T, H] output.
  *   workspace: device scratch of at least mc_moe_workspace_size(shape, T) bytes,
- *   256-byte aligned; its first 4 bytes are the status word (see mc_check_status).
+ *   256-byte aligned, ZEROED before its first use (every call leaves the parts
+ *   that need it at zero again); its first 4 bytes are the status word (see
+ *   mc_check_status).
  *   topk_idx_out int32 [T,2], topk_w_out fp32 [T,2], pruned_out uint8 [T]: optional
  *   copies of the routing decisions (NULL to skip).
  * Never synchronises and never allocates; capturable in a CUDA graph.

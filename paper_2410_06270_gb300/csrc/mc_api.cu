@@ -65,6 +65,7 @@ struct Workspace {
     int32_t *offsets, *perm, *inv;
     ChunkInfo *chunks;
     int32_t *nchunks, *counters;
+    int32_t *route_done;  // zero between calls: single-launch routing for small T
     uint8_t *xfrag;
     float *xtab;
     uint8_t *hfrag;
@@ -101,6 +102,7 @@ static Workspace carve(const mc_shape *s, int T, void *base)
     w.chunks = (ChunkInfo *)take(MC * sizeof(ChunkInfo));
     w.nchunks = (int32_t *)take(4);
     w.counters = (int32_t *)take(16);
+    w.route_done = (int32_t *)take(4);
     w.xfrag = (uint8_t *)take(MC * (s->H / kTileK) * kFragBytes);
     w.xtab = (float *)take(MC * (s->H / kTileK) * tb);
     w.hfrag = (uint8_t *)take(MC * (s->F / kTileK) * kFragBytes);
@@ -255,7 +257,7 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     pp.nchunks = ws.nchunks;
     pp.counters = ws.counters;
     pp.chunk = path == 3 ? 128 : kChunk;
-    rc = launch_route(rp, pp, st);
+    rc = launch_route(rp, pp, st, ws.route_done);
     if (rc) return rc;
 
     ExpertParams ep;

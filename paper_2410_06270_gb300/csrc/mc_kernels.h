@@ -111,7 +111,9 @@ struct CombineParams {
 };
 
 // Host launchers: MC_OK or an MC_ERR_* code with the message set.
-int launch_route(const RouteParams &rp, const PermuteParams &pp, cudaStream_t st);
+// done: a zeroed device counter enabling the single-launch routing + placement for
+// T <= 64 (left at zero), or NULL for two launches.
+int launch_route(const RouteParams &rp, const PermuteParams &pp, cudaStream_t st, int32_t *done = nullptr);
 int launch_gemv(ExpertParams ep, cudaStream_t st);   // mma.sync path
 int launch_tc(ExpertParams ep, cudaStream_t st);     // tcgen05 path
 int launch_gemm(ExpertParams ep, cudaStream_t st);   // prefill path (tcgen05 grouped GEMM)

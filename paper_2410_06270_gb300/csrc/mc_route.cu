@@ -17,11 +17,12 @@ namespace mc {
 
 constexpr int kRouteWarps = 4;
 
-__global__ void __launch_bounds__(kRouteWarps * 32) route_kernel(RouteParams p)
+// The logits of token t by the whole CTA; thread 0 takes the decision and writes
+// the outputs.
+__device__ __forceinline__ void route_token(const RouteParams &p, int t)
 {
     __shared__ float part[kRouteWarps][kMaxE];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int t = blockIdx.x;
     const int H = p.H, E = p.E;
     const __nv_bfloat16 *xr = p.x + (size_t)t * H;
     float acc[kMaxE];
@@ -59,7 +60,7 @@ __global__ void __launch_bounds__(kRouteWarps * 32) route_kernel(RouteParams p)
         if (lane == 0) part[warp][e] = acc[e];
     }
     __syncthreads();
-    if (threadIdx.x != 0) return;
+    if (threadIdx.x != 0) return;  // (route_token returns to its caller; the CTA re-joins there)
     float l[kMaxE];
     for (int e = 0; e < E; ++e) {
         float s = 0.f;
@@ -98,7 +99,11 @@ __global__ void __launch_bounds__(kRouteWarps * 32) route_kernel(RouteParams p)
     if (p.pruned_out) p.pruned_out[t] = prune ? 1 : 0;
 }
 
-__global__ void __launch_bounds__(1024) permute_kernel(PermuteParams p)
+__global__ void __launch_bounds__(kRouteWarps * 32) route_kernel(RouteParams p) { route_token(p, blockIdx.x); }
+
+// Histogram, scan, stable placement and work-chunk list by one CTA of any size
+// (whole warps).
+__device__ __forceinline__ void permute_block(const PermuteParams &p)
 {
     __shared__ int cnt[kMaxE];
     __shared__ int run[kMaxE];
@@ -111,8 +116,8 @@ __global__ void __launch_bounds__(1024) permute_kernel(PermuteParams p)
     }
     __syncthreads();
     for (int i = tid; i < NP; i += blockDim.x) {
-        bool kept = !((i & 1) && p.pruned[i >> 1]);
-        if (kept) atomicAdd(&cnt[p.idx[i]], 1);
+        bool kept = !((i & 1) && __ldcg(p.pruned + (i >> 1)));
+        if (kept) atomicAdd(&cnt[__ldcg(p.idx + i)], 1);
     }
     __syncthreads();
     if (tid == 0) {
@@ -147,8 +152,8 @@ __global__ void __launch_bounds__(1024) permute_kernel(PermuteParams p)
         int i = base + tid;
         int key = -1;
         if (i < NP) {
-            bool kept = !((i & 1) && p.pruned[i >> 1]);
-            key = kept ? p.idx[i] : -1;
+            bool kept = !((i & 1) && __ldcg(p.pruned + (i >> 1)));
+            key = kept ? __ldcg(p.idx + i) : -1;
         }
         for (int e = lane; e < kMaxE; e += 32) wcnt[warp][e] = 0;
         __syncwarp();
@@ -175,10 +180,38 @@ __global__ void __launch_bounds__(1024) permute_kernel(PermuteParams p)
     }
 }
 
+__global__ void __launch_bounds__(1024) permute_kernel(PermuteParams p) { permute_block(p); }
+
+// Routing of token blockIdx.x, then the last CTA to finish (counted on *done,
+// which it resets) places the pairs: one launch instead of two for small T.
+__global__ void __launch_bounds__(kRouteWarps * 32) route_permute_kernel(RouteParams rp, PermuteParams pp, int32_t *done)
+{
+    __shared__ int last;
+    route_token(rp, blockIdx.x);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();  // this CTA's routing outputs before the count
+        last = atomicAdd(done, 1) == (int)gridDim.x - 1;
+    }
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
+    permute_block(pp);
+    if (threadIdx.x == 0) *done = 0;
+}
+
 int max_chunks_for(int T, int E) { return (2 * T + kChunk - 1) / kChunk + E; }
 
-int launch_route(const RouteParams &rp, const PermuteParams &pp, cudaStream_t st)
+int launch_route(const RouteParams &rp, const PermuteParams &pp, cudaStream_t st, int32_t *done)
 {
+    if (done && rp.T <= 64) {
+        profile_begin(kKRoute, st);
+        route_permute_kernel<<<rp.T, kRouteWarps * 32, 0, st>>>(rp, pp, done);
+        profile_end(kKRoute, st);
+        cudaError_t err = cudaGetLastError();
+        if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "route launch: %s", cudaGetErrorString(err));
+        return MC_OK;
+    }
     profile_begin(kKRoute, st);
     route_kernel<<<rp.T, kRouteWarps * 32, 0, st>>>(rp);
     profile_end(kKRoute, st);
