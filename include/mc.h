@@ -215,10 +215,13 @@ int mc_stack_forward(void *h, int T, const mc_shape *shape, int layers, const vo
  * Process-wide; returns the previous value. */
 int mc_set_path(int path);
 
-/* Test hook: `flags` = 1 makes the expert kernels' weight producer issue no
+/* Test hook: `flags` bit 0 makes the expert kernels' weight producer issue no
  * copies, so every consumer wait reaches its bound and the status word reports
- * MC_ERR_TIMEOUT (no fault, no hang).  `timeout_ns` (0 = keep) bounds every
- * device wait (default 1 s).  Process-wide. */
+ * MC_ERR_TIMEOUT (no fault, no hang); bit 1 launches every kernel without
+ * programmatic dependent launch (by default each kernel's launch overlaps the
+ * end of the one before it on the stream; results are the same either way).
+ * `timeout_ns` (0 = keep) bounds every device wait (default 1 s).
+ * Process-wide. */
 int mc_set_debug(int flags, unsigned long long timeout_ns);
 
 /* Self-test of the tensor-core (tcgen05) building blocks used by the expert
@@ -244,13 +247,17 @@ int mc_check_status(void *workspace, void *stream);
  * synchronises on the recorded events, writes the summed milliseconds and launch
  * counts of kernel ids 0 .. n-1 (names from mc_profile_name: route, permute,
  * gemv_w13, gemv_w2, combine, gemm_gather, gemm_w13, gemm_w2, rmsnorm, glu) and
- * clears the records.  Not for use inside CUDA graph capture. */
+ * clears the records.  Inside stream capture the events become event nodes of
+ * the graph: every replay records them again, and each mc_profile_read reports
+ * the latest replay and keeps those records until mc_profile_clear. */
 int mc_profile_enable(int on);
 /* Bit mask of the kernel ids recorded while profiling is on (default: all), so
  * that a benchmark can time one kernel with two events per launch and leave the
  * others unperturbed.  Returns the previous mask. */
 unsigned mc_profile_select(unsigned mask);
 int mc_profile_read(double *ms_out, int *count_out, int n);
+/* Drops every record, including those kept for captured graphs. */
+int mc_profile_clear(void);
 const char *mc_profile_name(int id);
 
 /* RMSNorm used between stacked layers: out = x / sqrt(mean(x^2) + eps) * gamma,

@@ -75,6 +75,7 @@ def load():
         "mc_profile_enable": (I, [I]),
         "mc_profile_select": (ctypes.c_uint, [ctypes.c_uint]),
         "mc_profile_read": (I, [P, P, I]),
+        "mc_profile_clear": (I, []),
         "mc_profile_name": (ctypes.c_char_p, [I]),
     }
     for name, (res, args) in sig.items():
@@ -358,6 +359,11 @@ def profile_select(names) -> None:
         return
     ids = [i for i in range(N_KERNELS) if load().mc_profile_name(i).decode() in set(names)]
     load().mc_profile_select(sum(1 << i for i in ids))
+
+
+def profile_clear() -> None:
+    """Drop every profiling record, including those of captured graphs."""
+    _check(load().mc_profile_clear())
 
 
 def profile_read() -> dict:

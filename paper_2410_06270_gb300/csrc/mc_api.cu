@@ -35,7 +35,6 @@ static inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 // item at least two ring stages, the split count whose work items (estimated
 // chunks x 256-row block pairs x splits) fill the SMs' last wave best, the
 // smaller one on ties.
-constexpr int kMaxKS = 8;  // the combine reads one partial per split
 
 static int max_ks(const mc_shape *s, int T) { return T > 64 ? 1 : kMaxKS; }
 
@@ -130,6 +129,8 @@ static float neg_log_mu(float mu)
     if (mu <= 0.f) return INFINITY;
     return (float)(-log((double)mu));
 }
+
+bool pdl_enabled() { return !(g_debug.load() & kDebugNoPdl); }
 
 }  // namespace mc
 

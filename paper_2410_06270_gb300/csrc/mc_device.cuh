@@ -23,6 +23,15 @@ __device__ __forceinline__ uint64_t globaltimer_ns()
     return t;
 }
 
+// Programmatic dependent launch.  pdl_trigger: the next kernel on the stream may
+// be launched now (it is, once every CTA of this grid has triggered or exited).
+// pdl_wait: returns once the kernel before this one on the stream has completed
+// and its memory operations are visible; a no-op for a kernel launched without
+// programmatic serialisation.  Every kernel of the library calls pdl_wait before
+// its first global memory access.
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ uint32_t smem_u32(const void *p)
 {
     return (uint32_t)__cvta_generic_to_shared(p);

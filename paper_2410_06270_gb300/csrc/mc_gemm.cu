@@ -113,8 +113,11 @@ __device__ __forceinline__ bool g_header_ok(const ExpertParams &p, int e)
 __global__ void __launch_bounds__(256) x_img_kernel(ExpertParams p)
 {
     const int k = blockIdx.x, kt = blockIdx.y, KT = p.H / kTileK;
-    if (k >= *p.nchunks) return;
-    const ChunkInfo ci = p.chunks[k];
+    pdl_trigger();
+    pdl_wait();
+    const int nblocks = *p.nchunks;
+    const ChunkInfo ci = p.chunks[k];  // entry k < max_blocks exists even when unused
+    if (k >= nblocks) return;
     const int n = threadIdx.x >> 1, half = threadIdx.x & 1;
     uint8_t *img = p.ximg + ((size_t)k * KT + kt) * kImgBytes;
     bool bad = false;
@@ -274,6 +277,7 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
     const int KTm = W13 ? p.H / kTileK : p.F / kTileK;  // column steps (K)
     const uint8_t *img_base = W13 ? p.ximg : p.himg;
 
+    pdl_wait();
     if (threadIdx.x == 0) {
         for (int s = 0; s < kGSlots; ++s) {
             mbar_init(&sh->full[s], 1);
@@ -323,7 +327,10 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
             uint32_t verified = 0;
             while (ok) {
                 const int item = atomicAdd(&p.counters[W13 ? 2 : 3], 1);
-                if (item >= total) break;
+                if (item >= total) {
+                    pdl_trigger();  // the CTA takes no further item: the next kernel may launch
+                    break;
+                }
                 int r = 0;
                 while (r + 1 < sh->nruns && item >= sh->run_base[r + 1]) ++r;
                 const int local = item - sh->run_base[r], nbr = sh->run_nb[r];
@@ -556,20 +563,17 @@ int launch_gemm(ExpertParams ep, cudaStream_t st)
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(err));
 
     profile_begin(kKGemmGather, st);
-    x_img_kernel<<<dim3(ep.max_blocks, ep.H / kTileK), 256, 0, st>>>(ep);
+    err = launch_k(x_img_kernel, dim3(ep.max_blocks, ep.H / kTileK), dim3(256), 0, st, ep);
     profile_end(kKGemmGather, st);
-    err = cudaGetLastError();
     if (err == cudaSuccess) {
         profile_begin(kKGemmW13, st);
-        k13<<<nsm, kGThreads, kGSmem, st>>>(ep);
+        err = launch_k(k13, dim3(nsm), dim3(kGThreads), kGSmem, st, ep);
         profile_end(kKGemmW13, st);
-        err = cudaGetLastError();
     }
     if (err == cudaSuccess) {
         profile_begin(kKGemmW2, st);
-        k2<<<nsm, kGThreads, kGSmem, st>>>(ep);
+        err = launch_k(k2, dim3(nsm), dim3(kGThreads), kGSmem, st, ep);
         profile_end(kKGemmW2, st);
-        err = cudaGetLastError();
     }
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "GEMM launch: %s", cudaGetErrorString(err));
     return MC_OK;

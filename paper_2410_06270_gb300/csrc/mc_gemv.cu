@@ -90,13 +90,19 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, co
 // the expert's bit width and the byte offsets of its matrices (which depend on
 // every earlier expert's width) must match what the host computed, so no copy
 // ever reads outside the region the buffer was packed with.
-__device__ __forceinline__ bool header_ok(const ExpertParams &p, int e)
+// The packed buffer's header matches the shape, bit table and matrix offsets the
+// kernel was launched with, for every expert (its loads are all in flight together).
+__device__ __forceinline__ bool header_ok(const ExpertParams &p)
 {
     const PackHeader *hd = reinterpret_cast<const PackHeader *>(p.packed);
-    return hd->magic == kMagic && hd->version == kFormatVersion && hd->E == p.E && hd->H == p.H &&
-           hd->F == p.F && hd->group == p.group && hd->bits[e] == p.bits[e] &&
-           hd->mat_off[e][0] == p.mat_off[e][0] && hd->mat_off[e][1] == p.mat_off[e][1] &&
-           hd->mat_off[e][2] == p.mat_off[e][2];
+    bool ok = hd->magic == kMagic && hd->version == kFormatVersion && hd->E == p.E && hd->H == p.H &&
+              hd->F == p.F && hd->group == p.group;
+#pragma unroll
+    for (int e = 0; e < kMaxE; ++e)
+        if (e < p.E)
+            ok &= hd->bits[e] == p.bits[e] && hd->mat_off[e][0] == p.mat_off[e][0] &&
+                  hd->mat_off[e][1] == p.mat_off[e][1] && hd->mat_off[e][2] == p.mat_off[e][2];
+    return ok;
 }
 
 // D += A * B, m16n8k16, fp16 inputs, fp32 accumulate (not volatile, so the
@@ -185,9 +191,13 @@ __global__ void __launch_bounds__(256) frag_x_kernel(ExpertParams p)
     __shared__ __align__(16) __half xs[kChunk * kTileK];
     __shared__ uint2 afr[8 * 32];
     const int k = blockIdx.x, kt = blockIdx.y, KT = p.H / kTileK;
-    if (k >= *p.nchunks) return;
     build_tab_afrag(afr, threadIdx.x, 256);
+    pdl_trigger();
+    pdl_wait();
+    // both loads in flight together (entry k < max_chunks exists even when unused)
+    const int nchunks = *p.nchunks;
     const ChunkInfo ci = p.chunks[k];
+    if (k >= nchunks) return;
     const int NT = ci.nv > 8 ? 2 : 1;
     const int tid = threadIdx.x;
     {
@@ -525,37 +535,45 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
         fence_mbar_init();
     }
     if (W13) build_tab_afrag(afr, threadIdx.x, kGemvThreads);
+    pdl_wait();
     __syncthreads();
 
     if (warp == kCW) {
         // ---------------------------------------------------------- producer --
         if (lane == 0 && !(p.debug & kDebugNoProducer)) {
             const uint64_t pol = policy_evict_first();
-            const int total = *p.nchunks * U;
+            int *counter = &p.counters[W13 ? 0 : 1];
+            // the item count, the first claim and the header check: one round trip
+            const int nchunks = *p.nchunks;
+            int item = atomicAdd(counter, 1);
+            bool ok = header_ok(p);
+            const int total = nchunks * U;
             int it = 0, pslot = 0;
             uint32_t pphase = 0;  // phase of the ring round being filled
-            bool ok = true;
-            uint32_t verified = 0;  // experts whose packed header has been checked
-            while (ok) {
-                const int item = atomicAdd(&p.counters[W13 ? 0 : 1], 1);
-                if (item >= total) break;
-                const Item I = decode_item<W13>(p, item, U, p.chunks[item / U]);
-                const int e = I.ci.e, bits = I.ci.bits, NT = I.ci.nv > 8 ? 2 : 1;
-                if (!((verified >> e) & 1u)) {
-                    if (!header_ok(p, e)) {
-                        set_status(p.status, MC_ERR_BAD_PACK);
-                        sh->abort = 1;
-                        ok = false;
-                        break;
-                    }
-                    verified |= 1u << e;
-                }
+            if (!ok) {
+                set_status(p.status, MC_ERR_BAD_PACK);
+                sh->abort = 1;
+            }
+            ChunkInfo ci;
+            if (ok && item < total) ci = p.chunks[item / U];
+            if (item >= total) pdl_trigger();
+            while (ok && item < total) {
+                // the next item is claimed with this item's second-to-last stage and
+                // its chunk read with the last one: both round trips overlap copies
+                // already in flight, and a CTA holds at most one unstarted item
+                int next = total;
+                ChunkInfo next_ci = ci;
+                bool have_ci = false;
+                const Item I = decode_item<W13>(p, item, U, ci);
+                const int nst = (I.nkt + kKPS - 1) / kKPS, claim_at = nst > 1 ? nst - 2 : 0;
+                const int bits = I.ci.bits, NT = I.ci.nv > 8 ? 2 : 1;
+                const int e = I.ci.e;
                 const int STB = supertile_bytes(bits, group);
                 // one column step of both streams is pw contiguous supertiles
                 const int pw = W13 ? 2 : w2_pair_width(I.blkA >> 1, nrb);
                 const uint8_t *wsrc =
                     p.packed + p.mat_off[e][W13 ? 0 : 2] + supertile_off(W13 ? 0 : 2, I.blkA, I.kt0, KTm, nrb, STB);
-                for (int i = 0; i < I.nkt; i += kKPS, ++it) {
+                for (int i = 0, st = 0; i < I.nkt; i += kKPS, ++it, ++st) {
                     const int slot = pslot;
                     if (it >= S && !wait_or_abort(&empty[slot], pphase ^ 1u, p, sh)) {
                         ok = false;
@@ -577,7 +595,19 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
                         bulk_g2s(dst + vec_off0 + j * kKPS * VB, vbase + vec_off(I.k, j, I.kt0 + i, KTm, group), vb,
                                  &full[slot]);
                     sh->issued = it + 1;
+                    if (st == claim_at) {
+                        next = atomicAdd(counter, 1);
+                    } else if (st == nst - 1 && next < total) {
+                        next_ci = p.chunks[next / U];
+                        have_ci = true;
+                    }
                 }
+                if (!ok) break;
+                if (!have_ci && next < total) next_ci = p.chunks[next / U];
+                // the CTA takes no item after this one: the next kernel may launch
+                if (next >= total) pdl_trigger();
+                item = next;
+                ci = next_ci;
             }
             if (ok) {
                 // end marker: one more stage with item -1 and no data
@@ -630,24 +660,37 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
 // ---------------------------------------------------------------- combine --
 // y[t] = w0 * o[p(t,0)] + w1 * o[p(t,1)] (second term absent when pruned),
 // summing the column splits of the W2 pass in a fixed order (Eq. 1 with Eq. 5).
+//   Every load of a slot's column splits is issued before the first is used.
 __global__ void __launch_bounds__(256) combine_kernel(CombineParams p)
 {
+    pdl_trigger();
+    pdl_wait();
     const int H8 = p.H / 8;
     const int idx = blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= p.T * H8) return;
     const int t = idx / H8, c = (idx % H8) * 8;
     float out[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    const int2 q2 = *reinterpret_cast<const int2 *>(p.inv + 2 * t);
+    const float2 w2 = *reinterpret_cast<const float2 *>(p.w + 2 * t);
     for (int slot = 0; slot < 2; ++slot) {
-        const int q = p.inv[2 * t + slot];
+        const int q = slot ? q2.y : q2.x;
         if (q < 0) continue;
-        const float wt = p.w[2 * t + slot];
+        const float wt = slot ? w2.y : w2.x;
+        float4 a[kMaxKS], b[kMaxKS];
+#pragma unroll
+        for (int ks = 0; ks < kMaxKS; ++ks)
+            if (ks < p.KS) {
+                const float4 *src = reinterpret_cast<const float4 *>(p.opart + ((size_t)ks * p.Pmax + q) * p.H + c);
+                a[ks] = src[0];
+                b[ks] = src[1];
+            }
         float o[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-        for (int ks = 0; ks < p.KS; ++ks) {
-            const float4 *src = reinterpret_cast<const float4 *>(p.opart + ((size_t)ks * p.Pmax + q) * p.H + c);
-            const float4 a = src[0], b = src[1];
-            o[0] += a.x; o[1] += a.y; o[2] += a.z; o[3] += a.w;
-            o[4] += b.x; o[5] += b.y; o[6] += b.z; o[7] += b.w;
-        }
+#pragma unroll
+        for (int ks = 0; ks < kMaxKS; ++ks)
+            if (ks < p.KS) {
+                o[0] += a[ks].x; o[1] += a[ks].y; o[2] += a[ks].z; o[3] += a[ks].w;
+                o[4] += b[ks].x; o[5] += b[ks].y; o[6] += b[ks].z; o[7] += b[ks].w;
+            }
 #pragma unroll
         for (int k = 0; k < 8; ++k) out[k] = fmaf(wt, o[k], out[k]);
     }
@@ -678,20 +721,17 @@ int launch_gemv(ExpertParams ep, cudaStream_t st)
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(err));
 
     profile_begin(kKGemmGather, st);
-    frag_x_kernel<<<dim3(ep.max_chunks, ep.H / kTileK), 256, 0, st>>>(ep);
+    err = launch_k(frag_x_kernel, dim3(ep.max_chunks, ep.H / kTileK), dim3(256), 0, st, ep);
     profile_end(kKGemmGather, st);
-    err = cudaGetLastError();
     if (err == cudaSuccess) {
         profile_begin(kKGemvW13, st);
-        k13<<<nsm, kGemvThreads, sm, st>>>(ep);
+        err = launch_k(k13, dim3(nsm), dim3(kGemvThreads), sm, st, ep);
         profile_end(kKGemvW13, st);
-        err = cudaGetLastError();
     }
     if (err == cudaSuccess) {
         profile_begin(kKGemvW2, st);
-        k2<<<nsm, kGemvThreads, sm, st>>>(ep);
+        err = launch_k(k2, dim3(nsm), dim3(kGemvThreads), sm, st, ep);
         profile_end(kKGemvW2, st);
-        err = cudaGetLastError();
     }
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "GEMV launch: %s", cudaGetErrorString(err));
     return MC_OK;
@@ -700,10 +740,10 @@ int launch_gemv(ExpertParams ep, cudaStream_t st)
 int launch_combine(const CombineParams &cp, cudaStream_t st)
 {
     const int n = cp.T * (cp.H / 8);
+    if (cp.KS < 1 || cp.KS > kMaxKS) return set_error(MC_ERR_INVALID_ARG, "combine: %d column splits", cp.KS);
     profile_begin(kKCombine, st);
-    combine_kernel<<<(n + 255) / 256, 256, 0, st>>>(cp);
+    cudaError_t err = launch_k(combine_kernel, dim3((n + 255) / 256), dim3(256), 0, st, cp);
     profile_end(kKCombine, st);
-    cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "combine launch: %s", cudaGetErrorString(err));
     return MC_OK;
 }

@@ -99,8 +99,11 @@ struct ExpertParams {
 };
 
 constexpr int kDebugNoProducer = 1;
+constexpr int kDebugNoPdl = 2;  // launch without programmatic dependent launch
 // trace layout: [event][step] globaltimer ns
 enum TraceEvent { kTrProd = 0, kTrConsIn, kTrConsOut, kTrEv3, kTrEv4, kTrEv5, kTrEv6, kTrEvents };  // the copy producer never issues: waits expire
+
+constexpr int kMaxKS = 8;  // column splits of the W2 GEMV pass, at most
 
 struct CombineParams {
     const float *opart;   // [KS, Pmax, H]
@@ -109,6 +112,27 @@ struct CombineParams {
     int T, H, KS, Pmax;
     __nv_bfloat16 *y;     // [T, H]
 };
+
+// Launch with programmatic stream serialisation (unless switched off by
+// mc_set_debug bit 2): the kernel's launch and prologue overlap the end of the
+// kernel before it on the stream; the kernel itself calls pdl_wait before it
+// reads or writes global memory.
+bool pdl_enabled();
+template <typename... P, typename... A>
+inline cudaError_t launch_k(void (*kernel)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, A &&...args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl_enabled() ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<A &&>(args)...);
+}
 
 // Host launchers: MC_OK or an MC_ERR_* code with the message set.
 // done: a zeroed device counter enabling the single-launch routing + placement for

@@ -55,6 +55,8 @@ __global__ void unpack_kernel(const uint8_t *packed, uint64_t mat_off, int mat, 
 __global__ void __launch_bounds__(256) rmsnorm_kernel(const __nv_bfloat16 *x, const __nv_bfloat16 *gamma, int H,
                                                       float eps, __nv_bfloat16 *out)
 {
+    pdl_trigger();
+    pdl_wait();
     const __nv_bfloat16 *xr = x + (size_t)blockIdx.x * H;
     __shared__ float red[8];
     float ss = 0.f;
@@ -76,6 +78,8 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const __nv_bfloat16 *x, co
 
 __global__ void add_kernel(const __nv_bfloat16 *a, const __nv_bfloat16 *b, size_t n, __nv_bfloat16 *out)
 {
+    pdl_trigger();
+    pdl_wait();
     size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (i < n) out[i] = __float2bfloat16_rn(__bfloat162float(a[i]) + __bfloat162float(b[i]));
 }
@@ -114,9 +118,8 @@ int mc_rmsnorm(const void *x, const void *gamma, int T, int H, float eps, void *
     if (T < 0 || H <= 0 || !(eps >= 0.f)) return set_error(MC_ERR_INVALID_ARG, "bad T/H/eps");
     if (T == 0) return MC_OK;
     if (!x || !gamma || !out) return set_error(MC_ERR_INVALID_ARG, "NULL pointer argument");
-    rmsnorm_kernel<<<T, 256, 0, (cudaStream_t)stream>>>((const __nv_bfloat16 *)x, (const __nv_bfloat16 *)gamma, H,
-                                                        eps, (__nv_bfloat16 *)out);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_k(rmsnorm_kernel, dim3(T), dim3(256), 0, (cudaStream_t)stream, (const __nv_bfloat16 *)x,
+                             (const __nv_bfloat16 *)gamma, H, eps, (__nv_bfloat16 *)out);
     if (e != cudaSuccess) return set_error(MC_ERR_CUDA, "rmsnorm launch: %s", cudaGetErrorString(e));
     return MC_OK;
 }
@@ -126,9 +129,8 @@ int mc_add(const void *a, const void *b, size_t n, void *out, void *stream)
     clear_error();
     if (n == 0) return MC_OK;
     if (!a || !b || !out) return set_error(MC_ERR_INVALID_ARG, "NULL pointer argument");
-    add_kernel<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(
-        (const __nv_bfloat16 *)a, (const __nv_bfloat16 *)b, n, (__nv_bfloat16 *)out);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_k(add_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, (cudaStream_t)stream,
+                             (const __nv_bfloat16 *)a, (const __nv_bfloat16 *)b, n, (__nv_bfloat16 *)out);
     if (e != cudaSuccess) return set_error(MC_ERR_CUDA, "add launch: %s", cudaGetErrorString(e));
     return MC_OK;
 }

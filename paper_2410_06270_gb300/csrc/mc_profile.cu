@@ -11,6 +11,7 @@ namespace {
 struct Rec {
     int id;
     cudaEvent_t a, b;
+    bool graph;  // recorded by event nodes of a captured graph: re-recorded by every replay
 };
 std::mutex g_mu;
 bool g_on = false;
@@ -20,6 +21,19 @@ std::vector<cudaEvent_t> g_pool;
 cudaEvent_t g_pending[kKCount];
 const char *g_names[kKCount] = {"route", "permute", "gemv_w13", "gemv_w2", "combine",
                                 "gemm_gather", "gemm_w13", "gemm_w2", "rmsnorm", "glu"};
+
+// An event record on st; inside stream capture it becomes an event node of the
+// graph, so every replay of the graph records it again.
+bool record(cudaEvent_t e, cudaStream_t st)
+{
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(st, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusActive) {
+        cudaEventRecordWithFlags(e, st, cudaEventRecordExternal);
+        return true;
+    }
+    cudaEventRecord(e, st);
+    return false;
+}
 
 cudaEvent_t take_event()
 {
@@ -41,7 +55,7 @@ void profile_begin(int id, cudaStream_t st)
     if (!g_on || !((g_mask >> id) & 1u)) return;
     std::lock_guard<std::mutex> lk(g_mu);
     g_pending[id] = take_event();
-    cudaEventRecord(g_pending[id], st);
+    record(g_pending[id], st);
 }
 
 void profile_end(int id, cudaStream_t st)
@@ -49,8 +63,8 @@ void profile_end(int id, cudaStream_t st)
     if (!g_on || !((g_mask >> id) & 1u)) return;
     std::lock_guard<std::mutex> lk(g_mu);
     cudaEvent_t b = take_event();
-    cudaEventRecord(b, st);
-    g_recs.push_back({id, g_pending[id], b});
+    const bool graph = record(b, st);
+    g_recs.push_back({id, g_pending[id], b, graph});
 }
 
 }  // namespace mc
@@ -78,11 +92,13 @@ unsigned mc_profile_select(unsigned mask)
 int mc_profile_read(double *ms_out, int *count_out, int n)
 {
     clear_error();
-    std::vector<Rec> recs;
+    std::vector<Rec> recs, kept;
     {
         std::lock_guard<std::mutex> lk(g_mu);
         recs.swap(g_recs);
     }
+    for (auto &r : recs)
+        if (r.graph) kept.push_back(r);
     for (int i = 0; i < n; ++i) {
         if (ms_out) ms_out[i] = 0;
         if (count_out) count_out[i] = 0;
@@ -99,10 +115,23 @@ int mc_profile_read(double *ms_out, int *count_out, int n)
     }
     std::lock_guard<std::mutex> lk(g_mu);
     for (auto &r : recs) {
+        if (r.graph) continue;
         g_pool.push_back(r.a);
         g_pool.push_back(r.b);
     }
+    g_recs.insert(g_recs.begin(), kept.begin(), kept.end());
     return rc;
+}
+
+int mc_profile_clear(void)
+{
+    std::lock_guard<std::mutex> lk(g_mu);
+    for (auto &r : g_recs) {
+        g_pool.push_back(r.a);
+        g_pool.push_back(r.b);
+    }
+    g_recs.clear();
+    return MC_OK;
 }
 
 const char *mc_profile_name(int id) { return (id >= 0 && id < kKCount) ? g_names[id] : ""; }

@@ -2,52 +2,57 @@
 // weights, the ODP test of Eq. 5 with the token protection of Sec. 2.3.2, and the
 // permutation of kept (token, slot) pairs by expert.
 //
-// route_kernel: one CTA of 4 warps per token; each warp takes a quarter of the
-//   row (16-byte loads of x and of the gate rows), the partial logits meet in
-//   shared memory and thread 0 takes the decision in fp32.
+// route_kernel: one CTA of 16 warps per token; each thread takes 8 columns of
+//   a 4096-column round and issues all of the round's loads (x and the E gate
+//   rows, 16 bytes each) before it uses any, so a round costs one memory round
+//   trip; the partial logits meet in shared memory, warp 0 adds them up and
+//   thread 0 takes the decision in fp32.
 // permute_kernel: one CTA; histogram, exclusive scan and a stable placement with
 //   __match_any_sync ranks, so the permutation is unique (ascending token within
 //   an expert) and identical run to run.  It also lists the work chunks of the
-//   expert kernels and resets their work counters.
+//   expert kernels (one thread per expert) and resets their work counters.
 #include "mc_host.h"
 #include "mc_kernels.h"
 #include "mc_profile.h"
 
 namespace mc {
 
-constexpr int kRouteWarps = 4;
+constexpr int kRouteThreads = 512;
 
 // The logits of token t by the whole CTA; thread 0 takes the decision and writes
 // the outputs.
 __device__ __forceinline__ void route_token(const RouteParams &p, int t)
 {
-    __shared__ float part[kRouteWarps][kMaxE];
+    __shared__ float part[kRouteThreads / 32][kMaxE];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int H = p.H, E = p.E;
     const __nv_bfloat16 *xr = p.x + (size_t)t * H;
+    // the protection flag is needed only by thread 0's decision; load it now
+    const bool prot = threadIdx.x == 0 && p.protect != nullptr && p.protect[t] != 0;
     float acc[kMaxE];
 #pragma unroll
     for (int e = 0; e < kMaxE; ++e) acc[e] = 0.f;
-    // unrolled so that the loads of several 1024-column steps are in flight together
-#pragma unroll 4
-    for (int c0 = 8 * (threadIdx.x); c0 < H; c0 += 8 * 32 * kRouteWarps) {
-        uint4 raw = *reinterpret_cast<const uint4 *>(xr + c0);
+    for (int c0 = 8 * threadIdx.x; c0 < H; c0 += 8 * kRouteThreads) {
+        const uint4 raw = *reinterpret_cast<const uint4 *>(xr + c0);
+        uint4 gr[kMaxE];
+#pragma unroll
+        for (int e = 0; e < kMaxE; ++e)
+            if (e < E) gr[e] = *reinterpret_cast<const uint4 *>(p.gate + (size_t)e * H + c0);
         const __nv_bfloat162 *x2 = reinterpret_cast<const __nv_bfloat162 *>(&raw);
         float xf[8];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-            float2 f = __bfloat1622float2(x2[i]);
+            const float2 f = __bfloat1622float2(x2[i]);
             xf[2 * i] = f.x;
             xf[2 * i + 1] = f.y;
         }
 #pragma unroll
         for (int e = 0; e < kMaxE; ++e) {
             if (e < E) {
-                uint4 gr = *reinterpret_cast<const uint4 *>(p.gate + (size_t)e * H + c0);
-                const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gr);
+                const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gr[e]);
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
-                    float2 gf = __bfloat1622float2(g2[i]);
+                    const float2 gf = __bfloat1622float2(g2[i]);
                     acc[e] = fmaf(xf[2 * i], gf.x, acc[e]);
                     acc[e] = fmaf(xf[2 * i + 1], gf.y, acc[e]);
                 }
@@ -56,28 +61,41 @@ __device__ __forceinline__ void route_token(const RouteParams &p, int t)
     }
 #pragma unroll
     for (int e = 0; e < kMaxE; ++e) {
-        for (int m = 16; m >= 1; m >>= 1) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], m);
-        if (lane == 0) part[warp][e] = acc[e];
+        if (e < E) {
+            for (int m = 16; m >= 1; m >>= 1) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], m);
+            if (lane == 0) part[warp][e] = acc[e];
+        }
     }
     __syncthreads();
-    if (threadIdx.x != 0) return;  // (route_token returns to its caller; the CTA re-joins there)
+    if (warp != 0) return;  // (route_token returns to its caller; the CTA re-joins there)
+    // lane e adds up expert e's partials (warps in order), then thread 0 gathers them
+    float le = 0.f;
+    if (lane < E)
+        for (int w = 0; w < kRouteThreads / 32; ++w) le += part[w][lane];
     float l[kMaxE];
-    for (int e = 0; e < E; ++e) {
-        float s = 0.f;
-        for (int w = 0; w < kRouteWarps; ++w) s += part[w][e];
-        l[e] = s;
-    }
+#pragma unroll
+    for (int e = 0; e < kMaxE; ++e) l[e] = __shfl_sync(0xffffffffu, le, e);
+    if (lane != 0) return;
     // top-2 on fp32 logits, lower index wins ties
     int e0 = 0;
-    for (int e = 1; e < E; ++e)
-        if (l[e] > l[e0]) e0 = e;
-    int e1 = e0 == 0 ? 1 : 0;
-    for (int e = 0; e < E; ++e)
-        if (e != e0 && l[e] > l[e1]) e1 = e;
-    const float d = l[e0] - l[e1];  // >= 0
+    float b0 = l[0];
+#pragma unroll
+    for (int e = 1; e < kMaxE; ++e)
+        if (e < E && l[e] > b0) {
+            b0 = l[e];
+            e0 = e;
+        }
+    int e1 = -1;
+    float b1 = 0.f;
+#pragma unroll
+    for (int e = 0; e < kMaxE; ++e)
+        if (e < E && e != e0 && (e1 < 0 || l[e] > b1)) {
+            b1 = l[e];
+            e1 = e;
+        }
+    const float d = b0 - b1;  // >= 0
     const float r = __expf(-d);     // = p1 / p0
     float w0 = 1.f / (1.f + r), w1 = r / (1.f + r);
-    const bool prot = p.protect != nullptr && p.protect[t] != 0;
     const bool prune = !prot && (d > p.neg_log_mu);
     if (prune) {
         w0 = 1.f;
@@ -99,62 +117,79 @@ __device__ __forceinline__ void route_token(const RouteParams &p, int t)
     if (p.pruned_out) p.pruned_out[t] = prune ? 1 : 0;
 }
 
-__global__ void __launch_bounds__(kRouteWarps * 32) route_kernel(RouteParams p) { route_token(p, blockIdx.x); }
+__global__ void __launch_bounds__(kRouteThreads) route_kernel(RouteParams p)
+{
+    pdl_trigger();
+    pdl_wait();
+    route_token(p, blockIdx.x);
+}
 
 // Histogram, scan, stable placement and work-chunk list by one CTA of any size
-// (whole warps).
+// (whole warps, at most 1024 threads).
 __device__ __forceinline__ void permute_block(const PermuteParams &p)
 {
     __shared__ int cnt[kMaxE];
     __shared__ int run[kMaxE];
+    __shared__ int nbits[kMaxE];
     __shared__ int wcnt[32][kMaxE];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int NP = 2 * p.T;
+    // expert of pair i, -1 when ODP pruned it (both loads in flight together)
+    auto pair_key = [&](int i) {
+        const uint8_t pr = __ldcg(p.pruned + (i >> 1));
+        const int e = __ldcg(p.idx + i);
+        return (i & 1) && pr ? -1 : e;
+    };
+    const int key0 = tid < NP ? pair_key(tid) : -1;  // the first pass's pair, kept for the placement
     if (tid < kMaxE) {
         cnt[tid] = 0;
         run[tid] = 0;
+        int b = 0;
+#pragma unroll
+        for (int f = 0; f < kMaxE; ++f)
+            if (f == tid) b = p.bits[f];
+        nbits[tid] = b;
     }
     __syncthreads();
     for (int i = tid; i < NP; i += blockDim.x) {
-        bool kept = !((i & 1) && __ldcg(p.pruned + (i >> 1)));
-        if (kept) atomicAdd(&cnt[__ldcg(p.idx + i)], 1);
+        const int key = i == tid ? key0 : pair_key(i);
+        if (key >= 0) atomicAdd(&cnt[key], 1);
     }
     __syncthreads();
-    if (tid == 0) {
-        int s = 0;
-        for (int e = 0; e < p.E; ++e) {
-            p.offsets[e] = s;
-            run[e] = s;
-            s += cnt[e];
+    if (tid < p.E) {
+        // expert tid: its offset, and the index of its first work chunk in the
+        // order the expert kernels take them (more bits first, then by expert)
+        const int e = tid, be = nbits[e], ce = cnt[e];
+        int off = 0, k0 = 0;
+        for (int f = 0; f < p.E; ++f) {
+            const int cf = cnt[f], bf = nbits[f];
+            if (f < e) off += cf;
+            if (bf > be || (bf == be && f < e)) k0 += (cf + p.chunk - 1) / p.chunk;
         }
-        p.offsets[p.E] = s;
+        p.offsets[e] = off;
+        run[e] = off;
+        if (e == p.E - 1) p.offsets[p.E] = off + ce;
         if (p.chunks) {
-            // work chunks of <= p.chunk pairs, experts with more bits first
-            int k = 0;
-            for (int b = 3; b >= 1; --b)
-                for (int e = 0; e < p.E; ++e) {
-                    if (p.bits[e] != b) continue;
-                    for (int c = 0; c < cnt[e]; c += p.chunk) {
-                        ChunkInfo ci;
-                        ci.e = e;
-                        ci.pair_base = run[e] + c;
-                        ci.nv = min(p.chunk, cnt[e] - c);
-                        ci.bits = b;
-                        p.chunks[k++] = ci;
-                    }
-                }
-            *p.nchunks = k;
-            for (int i = 0; i < 4; ++i) p.counters[i] = 0;
+            for (int c = 0, k = k0; c < ce; c += p.chunk, ++k) {
+                ChunkInfo ci;
+                ci.e = e;
+                ci.pair_base = off + c;
+                ci.nv = min(p.chunk, ce - c);
+                ci.bits = be;
+                p.chunks[k] = ci;
+            }
+            if (e == 0) {
+                int n = 0;
+                for (int f = 0; f < p.E; ++f) n += (cnt[f] + p.chunk - 1) / p.chunk;
+                *p.nchunks = n;
+                for (int i = 0; i < 4; ++i) p.counters[i] = 0;
+            }
         }
     }
     __syncthreads();
     for (int base = 0; base < NP; base += blockDim.x) {
         int i = base + tid;
-        int key = -1;
-        if (i < NP) {
-            bool kept = !((i & 1) && __ldcg(p.pruned + (i >> 1)));
-            key = kept ? __ldcg(p.idx + i) : -1;
-        }
+        const int key = i >= NP ? -1 : base == 0 ? key0 : pair_key(i);
         for (int e = lane; e < kMaxE; e += 32) wcnt[warp][e] = 0;
         __syncwarp();
         unsigned same = __match_any_sync(0xffffffffu, key);
@@ -180,22 +215,31 @@ __device__ __forceinline__ void permute_block(const PermuteParams &p)
     }
 }
 
-__global__ void __launch_bounds__(1024) permute_kernel(PermuteParams p) { permute_block(p); }
+__global__ void __launch_bounds__(1024) permute_kernel(PermuteParams p)
+{
+    pdl_trigger();
+    pdl_wait();
+    permute_block(p);
+}
 
 // Routing of token blockIdx.x, then the last CTA to finish (counted on *done,
 // which it resets) places the pairs: one launch instead of two for small T.
-__global__ void __launch_bounds__(kRouteWarps * 32) route_permute_kernel(RouteParams rp, PermuteParams pp, int32_t *done)
+__global__ void __launch_bounds__(kRouteThreads) route_permute_kernel(RouteParams rp, PermuteParams pp, int32_t *done)
 {
     __shared__ int last;
+    pdl_trigger();
+    pdl_wait();
     route_token(rp, blockIdx.x);
     __syncthreads();
     if (threadIdx.x == 0) {
-        __threadfence();  // this CTA's routing outputs before the count
-        last = atomicAdd(done, 1) == (int)gridDim.x - 1;
+        // thread 0 wrote this CTA's routing outputs: the release orders them before
+        // the count, the acquire makes the other CTAs' outputs visible to the last
+        int prev;
+        asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], 1;" : "=r"(prev) : "l"(done) : "memory");
+        last = prev == (int)gridDim.x - 1;
     }
     __syncthreads();
     if (!last) return;
-    __threadfence();
     permute_block(pp);
     if (threadIdx.x == 0) *done = 0;
 }
@@ -204,25 +248,23 @@ int max_chunks_for(int T, int E) { return (2 * T + kChunk - 1) / kChunk + E; }
 
 int launch_route(const RouteParams &rp, const PermuteParams &pp, cudaStream_t st, int32_t *done)
 {
+    cudaError_t err;
     if (done && rp.T <= 64) {
         profile_begin(kKRoute, st);
-        route_permute_kernel<<<rp.T, kRouteWarps * 32, 0, st>>>(rp, pp, done);
+        err = launch_k(route_permute_kernel, dim3(rp.T), dim3(kRouteThreads), 0, st, rp, pp, done);
         profile_end(kKRoute, st);
-        cudaError_t err = cudaGetLastError();
         if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "route launch: %s", cudaGetErrorString(err));
         return MC_OK;
     }
     profile_begin(kKRoute, st);
-    route_kernel<<<rp.T, kRouteWarps * 32, 0, st>>>(rp);
+    err = launch_k(route_kernel, dim3(rp.T), dim3(kRouteThreads), 0, st, rp);
     profile_end(kKRoute, st);
-    cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "route launch: %s", cudaGetErrorString(err));
     profile_begin(kKPermute, st);
     // one thread per pair (whole warps), at most 1024: fewer threads to synchronise for small T
     const int nt = min(1024, max(32, (2 * pp.T + 31) / 32 * 32));
-    permute_kernel<<<1, nt, 0, st>>>(pp);
+    err = launch_k(permute_kernel, dim3(1), dim3(nt), 0, st, pp);
     profile_end(kKPermute, st);
-    err = cudaGetLastError();
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "permute launch: %s", cudaGetErrorString(err));
     return MC_OK;
 }

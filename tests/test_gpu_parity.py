@@ -183,6 +183,60 @@ def test_forward_is_deterministic(mc):
     assert torch.equal(y1.view(torch.int16), y2.view(torch.int16))
 
 
+@pytest.mark.parametrize("T", [16, 300])
+def test_forward_same_without_programmatic_launch(mc, T):
+    """Kernels launched without programmatic dependent launch (each one starts
+    only after the one before it ended) give bit-identical outputs; T = 300
+    takes the GEMM path."""
+    L = synth.make_layer(T, 256, 512, 8, 64, [3, 2, 2, 1, 3, 2, 2, 3], 81, gate_std=0.1, mu=0.3,
+                         protect_frac=0.1)
+    shape, packed = _pack(mc, L)
+    x, g, p = to_dev(L)
+    y_on = mc.moe_forward(x, g, shape, L.bits, packed, L.mu, p)
+    mc.set_debug(2, 0)
+    try:
+        y_off = mc.moe_forward(x, g, shape, L.bits, packed, L.mu, p)
+    finally:
+        mc.set_debug(0, 1_000_000_000)
+    torch.cuda.synchronize()
+    assert torch.equal(y_on.view(torch.int16), y_off.view(torch.int16))
+
+
+def test_profile_events_inside_a_captured_graph(mc):
+    """Profiling events captured into a CUDA graph are recorded again by every
+    replay: each read reports the latest replay's launches and keeps the records
+    until profile_clear."""
+    L = synth.make_layer(16, 256, 512, 8, 64, [3, 2, 2, 1, 3, 2, 2, 3], 82, gate_std=0.1)
+    shape, packed = _pack(mc, L)
+    x, g, p = to_dev(L)
+    ws = mc.alloc_workspace(shape, L.T)
+    y = torch.empty_like(x)
+    mc.moe_forward(x, g, shape, L.bits, packed, y=y, workspace=ws)
+    torch.cuda.synchronize()
+    mc.profile_clear()
+    mc.profile_select(["gemv_w13", "gemv_w2"])
+    mc.profile_enable(True)
+    gr = torch.cuda.CUDAGraph()
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        with torch.cuda.graph(gr, stream=s):
+            mc.moe_forward(x, g, shape, L.bits, packed, y=y, workspace=ws)
+    torch.cuda.current_stream().wait_stream(s)
+    mc.profile_enable(False)
+    mc.profile_select(None)
+    try:
+        for _ in range(2):
+            gr.replay()
+            pr = mc.profile_read()
+            assert set(pr) == {"gemv_w13", "gemv_w2"}
+            assert all(n == 1 and ms > 0 for ms, n in pr.values())
+    finally:
+        mc.profile_clear()
+    torch.cuda.synchronize()
+    assert mc.profile_read() == {}
+
+
 # ---------------------------------------------------------- device faults ----
 
 def test_bounded_wait_reports_timeout_and_context_survives(mc):

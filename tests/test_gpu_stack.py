@@ -107,3 +107,22 @@ def test_stack_graph_replay_equals_eager(mc, shape_name):
     torch.cuda.synchronize()
     mc.check_status(ws)
     assert torch.equal(h_eager.view(torch.int16), h_graph.view(torch.int16))
+
+
+def test_stack_same_without_programmatic_launch(mc):
+    """The stack with every kernel launched without programmatic dependent
+    launch is bit-identical to the default (overlapped launches)."""
+    L, gates = synth.config_stack(T=32, layers=6, seed=404, H=256, F=512, E=8, group=64, gate_std=0.1)
+    mus = [0.2] * len(gates)
+    shape, args, gamma, ws, prot = _setup(mc, L, gates, mus, copies=True)
+    h_on = _dev_bf16(L.x)
+    mc.stack_forward(h_on, shape, args, gamma, ws, prot)
+    mc.set_debug(2, 0)
+    try:
+        h_off = _dev_bf16(L.x)
+        mc.stack_forward(h_off, shape, args, gamma, ws, prot)
+    finally:
+        mc.set_debug(0, 1_000_000_000)
+    torch.cuda.synchronize()
+    mc.check_status(ws)
+    assert torch.equal(h_on.view(torch.int16), h_off.view(torch.int16))
