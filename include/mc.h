@@ -232,12 +232,6 @@ int mc_set_debug(int flags, unsigned long long timeout_ns);
  * *status (device int32, may be NULL).  For the test suite; not on the layer path. */
 int mc_selftest_umma(const void *A, const void *B, float *D, int N, int K, int32_t *status, void *stream);
 
-/* Profiling hook: while set, CTA 0 of every expert-kernel launch writes a
- * globaltimer timeline of its first `steps` pipeline steps into trace_dev
- * (device uint64 [7][steps]; row 0 = producer issue, row 1/2 = consumer
- * start/end of the step).  NULL turns it off.  Process-wide. */
-int mc_set_trace(unsigned long long *trace_dev, int steps);
-
 /* Synchronise `stream`, read the status word at the start of `workspace`, clear
  * it, and return MC_OK or the recorded MC_ERR_* code. */
 int mc_check_status(void *workspace, void *stream);

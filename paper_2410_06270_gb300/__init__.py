@@ -71,7 +71,6 @@ def load():
         "mc_rmsnorm": (I, [P, P, I, I, F32, P, P]),
         "mc_add": (I, [P, P, Z, P, P]),
         "mc_selftest_umma": (I, [P, P, P, I, I, P, P]),
-        "mc_set_trace": (I, [P, I]),
         "mc_profile_enable": (I, [I]),
         "mc_profile_select": (ctypes.c_uint, [ctypes.c_uint]),
         "mc_profile_read": (I, [P, P, I]),
@@ -385,6 +384,3 @@ def selftest_umma(A, B, status=None, a_in_tmem=False):
     return D
 
 
-def set_trace(buf=None, steps=0):
-    """Record CTA 0's per-step pipeline timeline into buf (int64 [7, steps] on the device)."""
-    load().mc_set_trace(_ptr(buf), int(steps))

@@ -18,8 +18,6 @@ static std::atomic<int> g_path{0};
 constexpr int kPrefillPairs = 512;
 static std::atomic<int> g_debug{0};
 static std::atomic<unsigned long long> g_timeout_ns{1000000000ull};  // 1 s
-static uint64_t *g_trace = nullptr;
-static int g_trace_steps = 0;
 
 #define MC_CUDA(call)                                                                         \
     do {                                                                                      \
@@ -153,15 +151,6 @@ int mc_set_debug(int flags, unsigned long long timeout_ns)
     return MC_OK;
 }
 
-// Profiling hook: record the per-step event timeline of CTA 0 of the next expert
-// kernel launches into trace_dev (device uint64 [7][steps]); NULL turns it off.
-int mc_set_trace(unsigned long long *trace_dev, int steps)
-{
-    g_trace = (uint64_t *)trace_dev;
-    g_trace_steps = trace_dev ? steps : 0;
-    return MC_OK;
-}
-
 size_t mc_moe_workspace_size(const mc_shape *shape, int T_max)
 {
     if (check_shape(shape) || T_max < 0) return 0;
@@ -181,7 +170,7 @@ int mc_route(const void *x, const void *gate_w, int T, const mc_shape *shape, fl
         return set_error(MC_ERR_INVALID_ARG, "NULL pointer argument");
     if (!aligned(x, 16) || !aligned(gate_w, 16))
         return set_error(MC_ERR_INVALID_ARG, "x and gate_w must be 16-byte aligned");
-    RouteParams rp;
+    RouteParams rp{};
     memset(&rp, 0, sizeof rp);
     rp.x = (const __nv_bfloat16 *)x;
     rp.gate = (const __nv_bfloat16 *)gate_w;
@@ -193,7 +182,7 @@ int mc_route(const void *x, const void *gate_w, int T, const mc_shape *shape, fl
     rp.idx = topk_idx;
     rp.w = topk_w;
     rp.pruned = pruned;
-    PermuteParams pp;
+    PermuteParams pp{};
     memset(&pp, 0, sizeof pp);
     pp.idx = topk_idx;
     pp.pruned = pruned;
@@ -229,7 +218,7 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     int path = g_path;
     if (path == 0) path = 2 * T >= kPrefillPairs ? 3 : 1;
 
-    RouteParams rp;
+    RouteParams rp{};
     memset(&rp, 0, sizeof rp);
     rp.x = (const __nv_bfloat16 *)x;
     rp.gate = (const __nv_bfloat16 *)gate_w;
@@ -244,7 +233,7 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     rp.idx_out = topk_idx_out;
     rp.w_out = topk_w_out;
     rp.pruned_out = pruned_out;
-    PermuteParams pp;
+    PermuteParams pp{};
     memset(&pp, 0, sizeof pp);
     pp.idx = ws.idx;
     pp.pruned = ws.pruned;
@@ -261,7 +250,7 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     rc = launch_route(rp, pp, st, ws.route_done);
     if (rc) return rc;
 
-    ExpertParams ep;
+    ExpertParams ep{};
     memset(&ep, 0, sizeof ep);
     ep.packed = (const uint8_t *)packed_dev;
     uint64_t total;
@@ -296,12 +285,10 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     ep.status = ws.status;
     ep.timeout_ns = g_timeout_ns;
     ep.debug = g_debug;
-    ep.trace = g_trace;
-    ep.trace_steps = g_trace_steps;
     rc = path == 3 ? launch_gemm(ep, st) : path == 2 ? launch_tc(ep, st) : launch_gemv(ep, st);
     if (rc) return rc;
 
-    CombineParams cp;
+    CombineParams cp{};
     cp.opart = ws.opart;
     cp.w = ws.w;
     cp.inv = ws.inv;

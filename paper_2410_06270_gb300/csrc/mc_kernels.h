@@ -94,14 +94,10 @@ struct ExpertParams {
     int32_t *status;
     uint64_t timeout_ns;
     int debug;               // test hooks (kDebugNoProducer)
-    uint64_t *trace;         // optional event timeline of CTA 0 (profiling), or null
-    int trace_steps;
 };
 
-constexpr int kDebugNoProducer = 1;
-constexpr int kDebugNoPdl = 2;  // launch without programmatic dependent launch
-// trace layout: [event][step] globaltimer ns
-enum TraceEvent { kTrProd = 0, kTrConsIn, kTrConsOut, kTrEv3, kTrEv4, kTrEv5, kTrEv6, kTrEvents };  // the copy producer never issues: waits expire
+constexpr int kDebugNoProducer = 1;  // the copy producer never issues: waits expire
+constexpr int kDebugNoPdl = 2;       // launch without programmatic dependent launch
 
 constexpr int kMaxKS = 8;  // column splits of the W2 GEMV pass, at most
 

@@ -127,7 +127,7 @@ extern "C" int mc_moe_forward_static(const void *x, const void *gate_w, int T, c
         if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "cudaMemsetAsync: %s", cudaGetErrorString(err));
     }
 
-    RouteParams rp;
+    RouteParams rp{};
     memset(&rp, 0, sizeof rp);
     rp.x = (const __nv_bfloat16 *)x;
     rp.gate = (const __nv_bfloat16 *)gate_w;
@@ -139,7 +139,7 @@ extern "C" int mc_moe_forward_static(const void *x, const void *gate_w, int T, c
     rp.idx = ws.idx;
     rp.w = ws.w;
     rp.pruned = ws.pruned;
-    PermuteParams pp;
+    PermuteParams pp{};
     memset(&pp, 0, sizeof pp);
     pp.idx = ws.idx;
     pp.pruned = ws.pruned;
@@ -155,7 +155,7 @@ extern "C" int mc_moe_forward_static(const void *x, const void *gate_w, int T, c
     pp.chunk = kChunk;
     if ((rc = launch_route(rp, pp, st))) return rc;
 
-    ExpertParams ep;
+    ExpertParams ep{};
     memset(&ep, 0, sizeof ep);  // the tensor-core path's buffers stay NULL: not used here
     ep.packed = (const uint8_t *)packed_dev;
     uint64_t total;
@@ -180,7 +180,7 @@ extern "C" int mc_moe_forward_static(const void *x, const void *gate_w, int T, c
     ep.timeout_ns = 1000000000ull;
     if ((rc = launch_gemv(ep, st))) return rc;
 
-    CombineParams cp;
+    CombineParams cp{};
     cp.opart = ws.opart;
     cp.w = ws.w;
     cp.inv = ws.inv;
