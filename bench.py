@@ -38,9 +38,11 @@ HBM_NOMINAL_GBS = 7900.0  # GB300 HBM3e nominal, reported beside the measured co
 WORKLOADS = {"decode16": ("decode", 16), "decode4": ("decode", 4), "decode1": ("decode", 1),
              "prefill4096": ("prefill", 4096),
              "odp256": ("odp", 256), "odp256_b16": ("odp", 256), "odp256_b13": ("odp", 256),
+             "odp256_drop": ("odp", 256),
              "stack32": ("stack", 32)}
 STACK_LAYERS = 32
-ODP_BITS = {"odp256": 20, "odp256_b16": 16, "odp256_b13": 13}
+ODP_BITS = {"odp256": 20, "odp256_b16": 16, "odp256_b13": 13, "odp256_drop": 20}
+ODP_DROP = {"odp256_drop": 0.02}  # fraction of tokens whose experts are all masked (Sec. 3.2, Fig. 9)
 ODP_PRUNE = 0.15  # fraction of unprotected tokens whose secondary expert the threshold drops
 
 
@@ -256,6 +258,8 @@ def _workload(name):
         L = synth.config_stack(T=T, layers=STACK_LAYERS)
     else:
         L = synth.config_odp(T=T, bits_total=ODP_BITS[name])
+        if name in ODP_DROP:
+            L.protect = synth.importance_mask(L.x, 0.10, ODP_DROP[name], 1238)
     return kind, T, L
 
 
@@ -266,11 +270,14 @@ def _describe(kind, T, L):
                 "F 14336, 8 experts, top-2, group 128, bits %s (mean %.2f), ODP on (per-layer mu dropping the "
                 "secondary expert of %d%% of unprotected tokens), %d%% of tokens protected, whole stack in one "
                 "CUDA graph" % (STACK_LAYERS, T, list(map(int, L.bits)), L.mean_bits(), round(100 * ODP_PRUNE),
-                                round(100 * float(L.protect.mean()))))
+                                round(100 * float((L.protect == 1).mean()))))
     if kind == "odp":
         odp = "ODP on (mu %.4g: drops the secondary expert of %d%% of unprotected tokens), %d%% of tokens " \
               "protected by the importance surrogate" % (L.mu, round(100 * ODP_PRUNE),
-                                                         round(100 * float(L.protect.mean())))
+                                                         round(100 * float((L.protect == 1).mean())))
+        if (L.protect == 2).any():
+            odp += ", the %d%% least important tokens dropped (all experts masked)" % round(
+                100 * float((L.protect == 2).mean()))
     else:
         odp = "ODP off"
     return ("mixtral-8x7b MoE layer %s, %d tokens, H 4096, F 14336, 8 experts, top-2, group 128, bits %s "
@@ -279,13 +286,10 @@ def _describe(kind, T, L):
 
 
 def _odp_threshold(mc, x, gw, shape, protect_np, protect_dev):
-    """mu that prunes ODP_PRUNE of the unprotected tokens, from the library's own
-    routing weights at mu = 0 (w1/w0 per token)."""
+    """mu that prunes ODP_PRUNE of the prunable tokens: the library's quantile of
+    w1/w0 (mc_odp_threshold_host) over its own routing weights at mu = 0."""
     r = mc.route(x, gw, shape, 0.0, protect_dev)
-    w = r["w"].cpu().numpy().astype(np.float64)
-    ratio = w[:, 1] / w[:, 0]
-    free = ratio[protect_np == 0] if protect_np is not None else ratio
-    return float(np.quantile(free, ODP_PRUNE))
+    return mc.odp_threshold(r["w"], protect_np, ODP_PRUNE)
 
 
 def _traffic(kernel, workload):

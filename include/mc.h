@@ -6,6 +6,7 @@
  *   logits  = x Wg^T                                  (gate G of Eq. 1)
  *   (e0,e1) = top-2 experts, w = renormalised softmax  (Eq. 1)
  *   pruned  = !protect && w1/w0 < mu  -> w = (1, 0)    (Eq. 5, Sec. 2.3.2)
+ *   dropped = mask byte 2              -> w = (0, 0)    (Sec. 3.2, Fig. 9)
  *   y       = sum over kept slots of w * E_e(x)        (Eq. 1)
  *   E(x)    = W2 (silu(W1 x) * W3 x)                   (Mixtral SwiGLU expert)
  * with every expert's W1, W3, W2 quantised weight-only to that expert's bit width
@@ -120,15 +121,19 @@ int mc_pack_verify(const mc_shape *shape, const int8_t *bits_host, const void *p
 
 /* ------------------------------------------------------------------------ *
  * Routing: Eq. 1 gate + top-2 + renormalised softmax, Eq. 5 ODP, Sec. 2.3.2
- * protection, then the permutation of kept (token, slot) pairs by expert.
+ * protection, the Sec. 3.2 (Fig. 9) token drop, then the permutation of kept
+ * (token, slot) pairs by expert.
  *   x       bf16 [T, H]        gate_w  bf16 [E, H]
  *   mu      Eq. 5 threshold (finite, >= 0; 0 disables pruning; > 1 prunes every
  *           unprotected token)
- *   protect uint8 [T], nonzero = never prune; may be NULL
+ *   protect uint8 [T] token mask, may be NULL (all 0): 0 = prunable by Eq. 5,
+ *           2 = dropped (all of the token's experts masked: no pair, output 0),
+ *           any other value = protected (never pruned)
  * Outputs (device):
  *   topk_idx int32 [T, 2]  slot 0 = primary (larger weight), ties -> lower index
- *   topk_w   fp32  [T, 2]  renormalised weights; (1, 0) for a pruned token
- *   pruned   uint8 [T]
+ *   topk_w   fp32  [T, 2]  renormalised weights; (1, 0) for a pruned token,
+ *                          (0, 0) for a dropped one
+ *   pruned   uint8 [T]     0 kept, 1 secondary pruned, 2 token dropped
  *   expert_offsets int32 [E+1]  exclusive prefix counts of kept pairs
  *   perm     int32 [2T]   first expert_offsets[E] entries valid: 2*token + slot,
  *                          grouped by expert, ascending token within an expert
@@ -207,6 +212,32 @@ int mc_stack_forward(void *h, int T, const mc_shape *shape, int layers, const vo
                      const int8_t *bits_host, const void *const *packed_dev, const float *mu_host,
                      const uint8_t *protect, const void *gamma, float eps, void *workspace,
                      size_t ws_bytes, void *stream);
+
+/* ------------------------------------------------------------------------ *
+ * Token importance (Sec. 2.3.2, Eq. 6) and the protect mask of ODP.
+ *   t      bf16 [L, H]      the tokens entering the MoE block (the l1 norm of Eq. 6)
+ *   attn   fp32 [nh, L, L]  the block's attention probabilities, attn[h][i][j] =
+ *                           weight of query i on key j (causal: used for i >= j;
+ *                           entries must be finite and >= 0)
+ *   importance fp32 [L] out: I_j = ||t_j||_1 * (1/(L - j)) * sum_{i=j}^{L-1} Abar[i][j]
+ *                           (0-based j), Abar the mean over the heads: the mean
+ *                           attention key j receives from the queries that see it
+ *   protect_frac in [0, 1]: mask (uint8 [L] out, may be NULL) gets 1 for the
+ *                           ceil(protect_frac * L) tokens of largest importance
+ *                           (a product within 1e-6 of an integer counts as it)
+ *                           (ties to the lower index), 0 for the others -- the
+ *                           protect input of mc_route / mc_moe_forward.
+ * Deterministic (fixed summation order); asynchronous on `stream`.
+ * ------------------------------------------------------------------------ */
+int mc_token_importance(const void *t, const float *attn, int L, int H, int nh, float protect_frac,
+                        float *importance, uint8_t *mask, void *stream);
+
+/* The Eq. 5 threshold from calibration routing weights (Sec. 2.3.1: the median
+ * of w1/w0 over calibration data is q = 0.5): the q-quantile, linear between
+ * order statistics, of w1/w0 over the tokens whose mask byte is 0 (mask_host
+ * may be NULL) and whose primary weight is positive.  Host arrays: w_host
+ * fp32 [T, 2] as written by mc_route.  MC_ERR_INVALID_ARG when no token qualifies. */
+int mc_odp_threshold_host(const float *w_host, const uint8_t *mask_host, int T, double q, float *mu_out);
 
 /* Choose the expert path of mc_moe_forward: 0 = automatic (the GEMV below 512
  * kept-or-not pairs, 2T < 512, else the GEMM), 1 = the mma.sync grouped GEMV

@@ -15,6 +15,9 @@ function states the passage of the paper it follows:
 * ``expert``                    -- the Mixtral SwiGLU expert E_i of Eq. 1.
 * ``moe_layer``                 -- Eq. 1 with Eq. 5.
 * ``rmsnorm``                   -- the normalisation between stacked layers.
+* ``token_importance`` / ``select_top`` -- Sec. 2.3.2 Eq. 6 and the protect mask
+  of the most important tokens; ``odp_threshold`` -- the Eq. 5 threshold as a
+  quantile (the median in Sec. 2.3.1) of w1/w0 over calibration tokens.
 * ``stack``                     -- pre-norm residual layers h <- h + MoE(RMSNorm(h)),
   each result rounded to bf16 where the stacked workload stores bf16.
 
@@ -153,7 +156,9 @@ def gate_logits(x, wg) -> np.ndarray:
 
 
 def route(x, wg, mu: float, protect=None):
-    """Eq. 1 top-2 + renormalised softmax weights, Eq. 5 ODP, Sec. 2.3.2 protection.
+    """Eq. 1 top-2 + renormalised softmax weights, Eq. 5 ODP, Sec. 2.3.2 protection
+    and the Sec. 3.2 (Fig. 9) token drop: protect byte 0 = prunable, 2 = dropped
+    (weights (0, 0), no expert: pruned = 2), any other value = protected.
 
     Returns (idx int32 [T,2], w float32 [T,2], pruned uint8 [T]).
     """
@@ -238,3 +243,47 @@ def stack(x, gates, mats, mus, protect=None, eps: float = 1e-5, gamma=None):
         routes.append((idx, w, pr, xn))
     return h, routes
 
+
+
+def token_importance(t, attn, protect_frac: float):
+    """Sec. 2.3.2, Eq. 6, in fp64: I_j = ||t_j||_1 * (sum_{i=j}^{L-1} Abar[i, j]) / (L - j)
+    (0-based j; Abar = mean of the heads' attention probabilities attn[h, i, j],
+    query i, key j; the mean attention key j receives from the queries that see it),
+    and the protect mask of the ceil(protect_frac * L) most important tokens
+    (``select_top``; the product taken within 1e-6 of an integer as that integer).  t [L, H] (bf16 values), attn [nh, L, L].  Returns
+    (importance fp64 [L], mask uint8 [L])."""
+    t = np.asarray(t, np.float64)
+    A = np.asarray(attn, np.float64)
+    nh, L, _ = A.shape
+    Abar = A.sum(axis=0) / nh
+    imp = np.empty(L, np.float64)
+    for j in range(L):
+        imp[j] = np.abs(t[j]).sum() * Abar[j:, j].sum() / (L - j)
+    # ceil(frac * L), a product within 1e-6 of an integer counting as that integer
+    # (frac arrives as fp32: 0.3 * 10 must give 3)
+    n = int(np.ceil(float(np.float32(protect_frac)) * L - 1e-6))
+    return imp, select_top(imp, n)
+
+
+def select_top(imp, n: int):
+    """Mask of the n tokens of largest importance, ties to the lower index."""
+    imp = np.asarray(imp)
+    order = sorted(range(len(imp)), key=lambda j: (-imp[j], j))
+    mask = np.zeros(len(imp), np.uint8)
+    mask[order[:max(0, min(n, len(imp)))]] = 1
+    return mask
+
+
+def odp_threshold(w, mask=None, q: float = 0.5) -> float:
+    """Sec. 2.3.1: the Eq. 5 threshold as the q-quantile (0.5: the median the
+    paper uses) of w1/w0 over the tokens that can be pruned (mask 0) and have a
+    positive primary weight; linear between order statistics."""
+    w = np.asarray(w, np.float64)
+    keep = w[:, 0] > 0
+    if mask is not None:
+        keep &= np.asarray(mask) == 0
+    r = np.sort(w[keep, 1] / w[keep, 0])
+    pos = q * (len(r) - 1)
+    lo = int(np.floor(pos))
+    hi = min(lo + 1, len(r) - 1)
+    return float(r[lo] + (pos - lo) * (r[hi] - r[lo]))

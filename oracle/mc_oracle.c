@@ -7,7 +7,8 @@
  *   - the group-wise asymmetric weight dequantisation of Sec. 2.1 (Eq. 2's
  *     integer grid) and the 1-bit storage transform of Appendix A.2,
  *   - Online Dynamic Pruning, Sec. 2.3.1, Eq. 5, with the significant-token
- *     protection of Sec. 2.3.2,
+ *     protection of Sec. 2.3.2 and the less-significant-token drop of Sec. 3.2
+ *     (Fig. 9),
  *   - the SwiGLU expert feed-forward of Mixtral (the E_i of Eq. 1),
  *   - the weighted combine of Eq. 1.
  *
@@ -29,7 +30,10 @@
  *       top-2 and renormalised to sum to 1 (Mixtral's gate).
  *   R5  Top-2 ties are broken towards the lower expert index.  Selection is
  *       decided on the logits rounded to fp32 (the precision the GPU decides in).
- *   R6  A protected token (mask byte != 0) is never pruned (Sec. 2.3.2).
+ *   R6  Mask byte 1 (or any value other than 0 and 2): the token is protected and
+ *       never pruned (Sec. 2.3.2).  Mask byte 2: the token is dropped, all its
+ *       experts are masked (Sec. 3.2, Fig. 9): weights (0, 0), no expert
+ *       evaluated, its layer output is zero; pruned = 2 records it.
  *   R7  A 1-bit code is B~ = (sign(W)+1)/2 (Appendix A.2); it dequantises with the
  *       same formula using z = 1/2 and s = 2*alpha, giving w = +-alpha.
  *   R8  bits == 16 means the expert is not quantised: dense weights are used.
@@ -163,10 +167,12 @@ void mco_route(const float *x, const float *wg, int T, int H, int E, double mu,
         double p1 = exp(lt[e1] - mx) / z;
         double w0 = p0 / (p0 + p1);
         double w1 = p1 / (p0 + p1);
-        /* Eq. 5 (R3) unless protected (R6). */
-        int prot = protect ? (protect[t] != 0) : 0;
+        /* Eq. 5 (R3) unless protected; a dropped token keeps no expert (R6). */
+        const int drop = protect ? (protect[t] == 2) : 0;
+        const int prot = protect ? (protect[t] != 0 && !drop) : 0;
         int prune = (!prot) && (w1 / w0 < mu);
         if (prune) { w0 = 1.0; w1 = 0.0; }
+        if (drop) { w0 = 0.0; w1 = 0.0; prune = 2; }
         idx[2 * t + 0] = e0;
         idx[2 * t + 1] = e1;
         w[2 * t + 0] = (float)w0;
@@ -180,7 +186,8 @@ void mco_route(const float *x, const float *wg, int T, int H, int E, double mu,
  * The token -> expert correspondence of Eq. 1 as a permutation: every kept
  * (token, slot) pair, grouped by expert, ascending token inside an expert.
  * offsets[E+1] (exclusive prefix counts), perm[P] with entry = 2*token + slot.
- * Returns P.  A pruned token's slot 1 is not a pair.
+ * Returns P.  A pruned token's slot 1 is not a pair; a dropped token (pruned 2)
+ * has no pair.
  */
 int mco_permute(const int32_t *idx, const uint8_t *pruned, int T, int E,
                 int32_t *offsets, int32_t *perm)
@@ -190,7 +197,7 @@ int mco_permute(const int32_t *idx, const uint8_t *pruned, int T, int E,
     for (int e = 0; e < E; ++e) {
         for (int t = 0; t < T; ++t)
             for (int slot = 0; slot < 2; ++slot) {
-                if (slot == 1 && pruned[t]) continue;
+                if ((slot == 1 && pruned[t]) || pruned[t] == 2) continue;
                 if (idx[2 * t + slot] == e) perm[n++] = 2 * t + slot;
             }
         offsets[e + 1] = n;
@@ -220,7 +227,7 @@ void mco_moe_layer(const float *x, const float *wg, int T, int H, int E,
         double *yt = y + (size_t)i * H;
         for (int h = 0; h < H; ++h) yt[h] = 0.0;
         for (int slot = 0; slot < 2; ++slot) {
-            if (slot == 1 && pruned[t]) continue;
+            if ((slot == 1 && pruned[t]) || pruned[t] == 2) continue;
             int e = idx[2 * t + slot];
             mco_expert(&mats[3 * e + 0], &mats[3 * e + 1], &mats[3 * e + 2], xt, eo);
             double wt = (double)w[2 * t + slot];

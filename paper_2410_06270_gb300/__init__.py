@@ -71,6 +71,8 @@ def load():
         "mc_rmsnorm": (I, [P, P, I, I, F32, P, P]),
         "mc_add": (I, [P, P, Z, P, P]),
         "mc_selftest_umma": (I, [P, P, P, I, I, P, P]),
+        "mc_token_importance": (I, [P, P, I, I, I, F32, P, P, P]),
+        "mc_odp_threshold_host": (I, [P, P, I, ctypes.c_double, P]),
         "mc_profile_enable": (I, [I]),
         "mc_profile_select": (ctypes.c_uint, [ctypes.c_uint]),
         "mc_profile_read": (I, [P, P, I]),
@@ -207,7 +209,9 @@ def pack_verify(shape: Shape, bits, packed_dev) -> None:
 # ------------------------------------------------------------------ routing --
 
 def route(x, gate_w, shape: Shape, mu: float, protect=None):
-    """Eq. 1 top-2 + Eq. 5 ODP + permutation.  Returns a dict of device tensors."""
+    """Eq. 1 top-2 + Eq. 5 ODP + permutation.  protect: uint8 [T] token mask (0
+    prunable, 2 dropped, other values protected) or None.  Returns a dict of
+    device tensors."""
     import torch
     T = x.shape[0]
     dev = x.device
@@ -345,6 +349,44 @@ def add(a, b, out=None):
 # -------------------------------------------------------------- profiling --
 
 N_KERNELS = 10
+
+
+def token_importance(t, attn, protect_frac: float = 0.02, importance=None, mask=None, with_mask: bool = True):
+    """Eq. 6 token importance of the tokens t (bf16 [L, H]) from the block's
+    attention probabilities attn (fp32 [nh, L, L], query-major) and the protect
+    mask of the top ceil(protect_frac * L) tokens.  Returns (importance, mask)."""
+    import torch
+    L, H = t.shape
+    nh = attn.shape[0]
+    assert attn.dtype == torch.float32 and tuple(attn.shape) == (nh, L, L) and attn.is_contiguous()
+    if importance is None:
+        importance = torch.empty(L, dtype=torch.float32, device=t.device)
+    if with_mask and mask is None:
+        mask = torch.empty(L, dtype=torch.uint8, device=t.device)
+    _check(load().mc_token_importance(_ptr(t), _ptr(attn), L, H, nh, float(protect_frac), _ptr(importance),
+                                      _ptr(mask) if with_mask else None, _stream()))
+    return importance, mask
+
+
+def odp_threshold(w, mask=None, q: float = 0.5) -> float:
+    """Eq. 5 threshold mu: the q-quantile of w1/w0 over the tokens with mask 0
+    (w: routing weights [T, 2] from route(); host copies are taken)."""
+    wh = np.ascontiguousarray(_host(w), dtype=np.float32)
+    mh = None if mask is None else np.ascontiguousarray(_host(mask), dtype=np.uint8)
+    mu = ctypes.c_float()
+    _check(load().mc_odp_threshold_host(wh.ctypes.data, None if mh is None else mh.ctypes.data, wh.shape[0],
+                                        float(q), ctypes.byref(mu)))
+    return float(mu.value)
+
+
+def _host(a):
+    try:
+        import torch
+        if isinstance(a, torch.Tensor):
+            return a.detach().cpu().numpy()
+    except ImportError:
+        pass
+    return np.asarray(a)
 
 
 def profile_enable(on: bool = True) -> bool:

@@ -1,6 +1,7 @@
 // mc_route.cu -- the gate of Eq. 1, top-2 selection with renormalised softmax
-// weights, the ODP test of Eq. 5 with the token protection of Sec. 2.3.2, and the
-// permutation of kept (token, slot) pairs by expert.
+// weights, the ODP test of Eq. 5 with the token protection of Sec. 2.3.2 and the
+// token drop of Sec. 3.2 (Fig. 9: mask byte 2 masks all of a token's experts),
+// and the permutation of kept (token, slot) pairs by expert.
 //
 // route_kernel: one CTA of 16 warps per token; each thread takes 8 columns of
 //   a 4096-column round and issues all of the round's loads (x and the E gate
@@ -27,8 +28,9 @@ __device__ __forceinline__ void route_token(const RouteParams &p, int t)
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int H = p.H, E = p.E;
     const __nv_bfloat16 *xr = p.x + (size_t)t * H;
-    // the protection flag is needed only by thread 0's decision; load it now
-    const bool prot = threadIdx.x == 0 && p.protect != nullptr && p.protect[t] != 0;
+    // the mask byte is needed only by thread 0's decision; load it now
+    // (0: prunable, 2: dropped, anything else: protected)
+    const int mask = threadIdx.x == 0 && p.protect != nullptr ? p.protect[t] : 0;
     float acc[kMaxE];
 #pragma unroll
     for (int e = 0; e < kMaxE; ++e) acc[e] = 0.f;
@@ -96,16 +98,21 @@ __device__ __forceinline__ void route_token(const RouteParams &p, int t)
     const float d = b0 - b1;  // >= 0
     const float r = __expf(-d);     // = p1 / p0
     float w0 = 1.f / (1.f + r), w1 = r / (1.f + r);
-    const bool prune = !prot && (d > p.neg_log_mu);
+    const bool drop = mask == 2, prot = mask != 0 && !drop;
+    int prune = !prot && (d > p.neg_log_mu);
     if (prune) {
         w0 = 1.f;
         w1 = 0.f;
+    }
+    if (drop) {  // no expert: weights (0, 0), pruned = 2
+        w0 = w1 = 0.f;
+        prune = 2;
     }
     p.idx[2 * t] = e0;
     p.idx[2 * t + 1] = e1;
     p.w[2 * t] = w0;
     p.w[2 * t + 1] = w1;
-    p.pruned[t] = prune ? 1 : 0;
+    p.pruned[t] = (uint8_t)prune;
     if (p.idx_out) {
         p.idx_out[2 * t] = e0;
         p.idx_out[2 * t + 1] = e1;
@@ -114,7 +121,7 @@ __device__ __forceinline__ void route_token(const RouteParams &p, int t)
         p.w_out[2 * t] = w0;
         p.w_out[2 * t + 1] = w1;
     }
-    if (p.pruned_out) p.pruned_out[t] = prune ? 1 : 0;
+    if (p.pruned_out) p.pruned_out[t] = (uint8_t)prune;
 }
 
 __global__ void __launch_bounds__(kRouteThreads) route_kernel(RouteParams p)
@@ -134,11 +141,12 @@ __device__ __forceinline__ void permute_block(const PermuteParams &p)
     __shared__ int wcnt[32][kMaxE];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int NP = 2 * p.T;
-    // expert of pair i, -1 when ODP pruned it (both loads in flight together)
+    // expert of pair i, -1 when ODP pruned it or its token was dropped (both loads
+    // in flight together)
     auto pair_key = [&](int i) {
         const uint8_t pr = __ldcg(p.pruned + (i >> 1));
         const int e = __ldcg(p.idx + i);
-        return (i & 1) && pr ? -1 : e;
+        return ((i & 1) && pr) || pr == 2 ? -1 : e;
     };
     const int key0 = tid < NP ? pair_key(tid) : -1;  // the first pass's pair, kept for the placement
     if (tid < kMaxE) {

@@ -237,6 +237,23 @@ def importance_protect(x_bits, frac, seed):
     return protect
 
 
+def importance_mask(x_bits, protect_frac, drop_frac, seed):
+    """Token mask with the Sec. 3.2 (Fig. 9) drop: the top `protect_frac` of tokens
+    by the importance surrogate of `importance_protect` get 1 (protected), the
+    bottom `drop_frac` get 2 (all experts masked), ties to the lower index.  Input
+    generation only."""
+    x = bf16_bits_to_f32(x_bits)
+    score = np.abs(x).sum(axis=1, dtype=np.float64) * _rng(seed, 5).random(x.shape[0])
+    order = np.lexsort((np.arange(x.shape[0]), -score))  # score descending, index ascending
+    mask = np.zeros(x.shape[0], np.uint8)
+    n_p = int(np.ceil(protect_frac * x.shape[0]))
+    n_d = int(np.ceil(drop_frac * x.shape[0]))
+    mask[order[:n_p]] = 1
+    if n_d:
+        mask[order[-n_d:]] = 2
+    return mask
+
+
 def config_odp(T=256, seed=1238, bits_total=20, protect_frac=0.10):
     """Mixtral-8x7b-shaped layer for ODP: 256 tokens, 10% protected by the
     importance surrogate, bits with sum 20 / 16 / 13 (mean 2.5 / 2.0 / 1.6).  The

@@ -157,3 +157,20 @@ def test_workspace_size_grows_with_tokens(mc):
     s = mc.Shape(8, 4096, 14336, 128)
     a, b = mc.workspace_size(s, 16), mc.workspace_size(s, 4096)
     assert 0 < a < b
+
+
+def test_odp_threshold_host_matches_oracle():
+    """mc_odp_threshold_host (host code, no GPU) against the oracle's quantile of
+    w1/w0 over the prunable tokens."""
+    import oracle
+    import paper_2410_06270_gb300 as mc
+    rng = np.random.default_rng(70)
+    w0 = rng.uniform(0.5, 1.0, 200).astype(np.float32)
+    w = np.stack([w0, (1 - w0)], axis=1).astype(np.float32)
+    mask = np.zeros(200, np.uint8)
+    mask[::9] = 1
+    mask[3::17] = 2
+    for q in (0.0, 0.15, 0.5, 1.0):
+        assert mc.odp_threshold(w, mask, q) == pytest.approx(oracle.odp_threshold(w, mask, q), rel=1e-6)
+    with pytest.raises(mc.MCError):
+        mc.odp_threshold(w, np.ones(200, np.uint8), 0.5)

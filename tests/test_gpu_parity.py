@@ -44,7 +44,18 @@ def _check_routing(mc, L, idx, w, pr, offsets=None, perm=None):
 
 # -------------------------------------------------------------- routing ----
 
-@pytest.mark.parametrize("case", ["tiny", "odp", "odp_heavy", "many_tokens", "e16", "ragged_h"])
+def _with_drops(L, n, seed):
+    """Drop n unprotected tokens (mask byte 2, Sec. 3.2 Fig. 9); returns their indices."""
+    free = np.flatnonzero(L.protect == 0) if L.protect is not None else np.arange(L.T)
+    if L.protect is None:
+        L.protect = np.zeros(L.T, np.uint8)
+    dropped = np.random.default_rng(seed).choice(free, size=n, replace=False)
+    L.protect[dropped] = 2
+    return np.sort(dropped)
+
+
+@pytest.mark.parametrize("case", ["tiny", "odp", "odp_heavy", "many_tokens", "e16", "ragged_h", "drop_small",
+                                  "drop"])
 def test_route_bit_exact(mc, case):
     if case == "tiny":
         L = synth.config_tiny()
@@ -59,9 +70,14 @@ def test_route_bit_exact(mc, case):
                              experts=False)
     elif case == "e16":
         L = synth.make_layer(100, 384, 128, 16, 128, [2] * 16, 34, gate_std=0.1, mu=0.6, experts=False)
-    else:  # H = 384 is a multiple of 128 but not of 256
+    elif case == "ragged_h":  # H = 384 is a multiple of 128 but not of 256
         L = synth.make_layer(77, 384, 128, 8, 64, [2] * 8, 35, gate_std=0.1, mu=0.4, protect_frac=0.3,
                              experts=False)
+    else:  # token drop: T = 48 takes the single-launch routing, T = 200 the two-launch one
+        T = 48 if case == "drop_small" else 200
+        L = synth.make_layer(T, 256, 128, 8, 64, [2] * 8, 37, gate_std=0.15, mu=0.3, protect_frac=0.1,
+                             experts=False)
+        dropped = _with_drops(L, T // 8, 38)
     condition_routing(L, L.mu)
     x, g, p = to_dev(L)
     shape = mc.Shape(L.E, L.H, L.F, L.group)
@@ -69,7 +85,9 @@ def test_route_bit_exact(mc, case):
     torch.cuda.synchronize()
     _check_routing(mc, L, out["idx"], out["w"], out["pruned"], out["offsets"], out["perm"])
     if case != "tiny":
-        assert 0 < int(out["pruned"].sum()) < L.T
+        assert 0 < int((out["pruned"] == 1).sum()) < L.T
+    if case.startswith("drop"):
+        np.testing.assert_array_equal(np.flatnonzero(out["pruned"].cpu().numpy() == 2), dropped)
 
 
 def test_route_mu_zero_and_above_one(mc):
@@ -181,6 +199,25 @@ def test_forward_is_deterministic(mc):
     y2 = mc.moe_forward(x, g, shape, L.bits, packed)
     torch.cuda.synchronize()
     assert torch.equal(y1.view(torch.int16), y2.view(torch.int16))
+
+
+@pytest.mark.parametrize("T", [40, 300])
+def test_forward_token_drop(mc, T):
+    """Dropped tokens (mask byte 2) get a zero output and the rest match the
+    oracle; T = 40 takes the GEMV path, T = 300 the GEMM path."""
+    L = synth.make_layer(T, 256, 512, 8, 64, [3, 2, 2, 1, 3, 2, 2, 3], 84, gate_std=0.1, mu=0.3,
+                         protect_frac=0.1)
+    dropped = _with_drops(L, max(2, T // 20), 85)
+    condition_routing(L, L.mu)
+    shape, packed = _pack(mc, L)
+    x, g, p = to_dev(L)
+    y, r = mc.moe_forward(x, g, shape, L.bits, packed, L.mu, p, routing=True)
+    torch.cuda.synchronize()
+    _check_routing(mc, L, r["idx"], r["w"], r["pruned"])
+    got = y.float().cpu().numpy()
+    assert (got[dropped] == 0).all()
+    ref, *_ = oracle_layer(L, oracle_mats(L))
+    assert_close(got, ref, "token drop T=%d" % T)
 
 
 @pytest.mark.parametrize("T", [16, 300])

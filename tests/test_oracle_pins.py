@@ -118,6 +118,27 @@ def test_prune_set_is_ratio_below_mu():
     assert counts == sorted(counts)
 
 
+def test_dropped_tokens_keep_no_expert():
+    """Mask byte 2 drops the token (Sec. 3.2, Fig. 9): weights (0, 0), pruned = 2,
+    the same top-2 indices as without the drop, no pair in the permutation; the
+    other tokens route exactly as before."""
+    L = _rand_layer(T=40, E=8, bits=(1, 2, 3, 2, 1, 2, 3, 3), experts=False,
+                    gate_std=0.6, protect_frac=0.2)
+    base = oracle.route(L.x_f32(), L.gate_f32(), mu=0.5, protect=L.protect)
+    mask = L.protect.copy()
+    dropped = [3, 11, 25, int(np.flatnonzero(L.protect)[0])]  # a protected token can be dropped too
+    mask[dropped] = 2
+    idx, w, pr = oracle.route(L.x_f32(), L.gate_f32(), mu=0.5, protect=mask)
+    np.testing.assert_array_equal(idx, base[0])
+    keep = np.setdiff1d(np.arange(40), dropped)
+    np.testing.assert_array_equal(w[keep], base[1][keep])
+    np.testing.assert_array_equal(pr[keep], base[2][keep])
+    assert (pr[dropped] == 2).all() and (w[dropped] == 0).all()
+    offsets, perm = oracle.permute(idx, pr, 8)
+    assert not set(perm.tolist()) & {2 * t + s for t in dropped for s in range(2)}
+    assert offsets[-1] == 80 - int(pr.astype(int).sum())
+
+
 # ----------------------------------------------------------- permutation ----
 
 def test_permutation_brute_force():
@@ -267,6 +288,8 @@ def _brute_layer(L, mats, mu, protect):
         # routing weights are carried in fp32 between the gate and the combine
         wa = float(np.float32(p[t, a] / (p[t, a] + p[t, b])))
         wb = float(np.float32(p[t, b] / (p[t, a] + p[t, b])))
+        if protect is not None and protect[t] == 2:  # dropped token: no expert (Sec. 3.2)
+            continue
         prot = protect is not None and protect[t]
         if not prot and wb / wa < mu:
             y[t] = outs[a]
@@ -276,13 +299,16 @@ def _brute_layer(L, mats, mu, protect):
 
 
 @pytest.mark.parametrize("mu", [0.0, 0.8])
-def test_layer_brute_force_tiny(mu):
+@pytest.mark.parametrize("drop", [False, True])
+def test_layer_brute_force_tiny(mu, drop):
     L = _rand_layer(T=10, H=16, F=24, E=4, group=8, bits=(1, 2, 3, 2), seed=11,
                     gate_std=0.5, protect_frac=0.3)
+    if drop:  # two unprotected tokens dropped (Sec. 3.2, Fig. 9)
+        L.protect[np.flatnonzero(L.protect == 0)[[1, 4]]] = 2
     mats = _mats(L)
     y, idx, w, pr = oracle.moe_layer(L.x_f32(), L.gate_f32(), mats, mu, L.protect)
     if mu > 0:
-        assert 0 < pr.sum() < L.T  # the case exercises both branches
+        assert 0 < (pr == 1).sum() < L.T  # the case exercises both branches
     np.testing.assert_allclose(y, _brute_layer(L, mats, mu, L.protect), rtol=1e-9, atol=1e-12)
 
 
@@ -367,3 +393,89 @@ def test_stack_one_layer_is_residual_of_normalised_layer():
     want = torch.tensor(x + yb, dtype=torch.float32).to(torch.bfloat16).double().numpy()
     h, _ = oracle.stack(L.x_f32(), [g], _mats(L), [0.0])
     np.testing.assert_array_equal(h, want)
+
+
+# ---------------------------------------------------- token importance (N2) ---
+
+def _causal_softmax(nh, L, seed, temp=1.0):
+    rng = np.random.default_rng(seed)
+    s = rng.standard_normal((nh, L, L)) * temp
+    s = np.where(np.tril(np.ones((L, L), bool))[None], s, -np.inf)
+    e = np.exp(s - s.max(axis=2, keepdims=True))
+    return e / e.sum(axis=2, keepdims=True)
+
+
+def test_importance_uniform_causal_attention_is_harmonic():
+    """Every query spreads evenly over the keys it sees (A[i, j] = 1/(i+1), j <= i):
+    the attention key j receives is H_L - H_j (harmonic numbers), so Eq. 6 gives
+    I_j = ||t_j||_1 (H_L - H_j) / (L - j)."""
+    L, H = 37, 8
+    t = np.random.default_rng(40).standard_normal((L, H))
+    A = np.tril(np.ones((L, L))) / np.arange(1, L + 1)[:, None]
+    imp, _ = oracle.token_importance(t, A[None], 0.0)
+    harm = np.concatenate([[0.0], np.cumsum(1.0 / np.arange(1, L + 1))])
+    want = np.abs(t).sum(1) * (harm[L] - harm[:L]) / (L - np.arange(L))
+    np.testing.assert_allclose(imp, want, rtol=1e-12)
+
+
+def test_importance_one_hot_attention_and_ties():
+    """All queries attend to key 0 only: I_0 = ||t_0||_1, every other token 0; the
+    mask takes token 0, then the zero-importance tokens by ascending index."""
+    L = 10
+    t = np.random.default_rng(41).standard_normal((L, 4)) + 3.0
+    A = np.zeros((1, L, L))
+    A[0, :, 0] = 1.0
+    imp, mask = oracle.token_importance(t, A, 0.3)
+    np.testing.assert_allclose(imp, np.r_[np.abs(t[0]).sum(), np.zeros(L - 1)], rtol=1e-12)
+    assert mask.tolist() == [1, 1, 1] + [0] * (L - 3)
+
+
+def test_importance_is_linear_in_the_heads_and_uses_l1():
+    """Eq. 6 is linear in A and in the l1 norm: two heads give the mean of the
+    one-head importances; scaling a token scales its importance by |c|; the sign
+    of its entries does not matter."""
+    L, H = 20, 6
+    t = np.random.default_rng(42).standard_normal((L, H))
+    A = _causal_softmax(2, L, 43)
+    both, _ = oracle.token_importance(t, A, 0.0)
+    one = [oracle.token_importance(t, A[h:h + 1], 0.0)[0] for h in range(2)]
+    np.testing.assert_allclose(both, 0.5 * (one[0] + one[1]), rtol=1e-12)
+    t2 = t.copy()
+    t2[5] *= -3.0
+    imp2, _ = oracle.token_importance(t2, A, 0.0)
+    np.testing.assert_allclose(imp2[5], 3.0 * both[5], rtol=1e-12)
+    np.testing.assert_allclose(np.delete(imp2, 5), np.delete(both, 5), rtol=1e-12)
+
+
+def test_importance_mask_size_and_brute_force():
+    """The mask holds ceil(frac * L) tokens, each at least as important as any
+    unmasked one (lower index on ties), checked against an exhaustive count."""
+    L = 30
+    t = np.random.default_rng(44).standard_normal((L, 5))
+    A = _causal_softmax(3, L, 45)
+    for frac in (0.0, 0.02, 0.1, 0.5, 1.0):
+        imp, mask = oracle.token_importance(t, A, frac)
+        n = int(np.ceil(float(np.float32(frac)) * L - 1e-6))
+        assert mask.sum() == n
+        for j in range(L):
+            better = sum(1 for i in range(L) if imp[i] > imp[j] or (imp[i] == imp[j] and i < j))
+            assert mask[j] == (better < n)
+
+
+def test_odp_threshold_is_quantile_of_prunable_ratios():
+    """q = 0.5 is the median of w1/w0 over the prunable tokens (Sec. 2.3.1), the
+    quantile follows numpy's linear rule, protected / dropped tokens are left out,
+    and mu = the q-quantile prunes (strictly below it) about a q share."""
+    L = _rand_layer(T=101, E=8, bits=(1, 2, 3, 2, 1, 2, 3, 3), experts=False, gate_std=0.5)
+    idx, w, pr = oracle.route(L.x_f32(), L.gate_f32(), mu=0.0)
+    r = w[:, 1].astype(np.float64) / w[:, 0]
+    assert oracle.odp_threshold(w, None, 0.5) == pytest.approx(np.median(r), rel=1e-12)
+    for q in (0.0, 0.15, 0.9, 1.0):
+        assert oracle.odp_threshold(w, None, q) == pytest.approx(np.quantile(r, q), rel=1e-12)
+    mask = np.zeros(101, np.uint8)
+    mask[::3] = 1
+    mask[1::7] = 2
+    assert oracle.odp_threshold(w, mask, 0.5) == pytest.approx(np.median(r[mask == 0]), rel=1e-12)
+    mu = oracle.odp_threshold(w, None, 0.15)
+    _, _, pr = oracle.route(L.x_f32(), L.gate_f32(), mu=mu)
+    assert abs(pr.mean() - 0.15) <= 1.0 / 101 + 1e-12
