@@ -38,11 +38,14 @@ HBM_NOMINAL_GBS = 7900.0  # GB300 HBM3e nominal, reported beside the measured co
 WORKLOADS = {"decode16": ("decode", 16), "decode4": ("decode", 4), "decode1": ("decode", 1),
              "prefill4096": ("prefill", 4096),
              "odp256": ("odp", 256), "odp256_b16": ("odp", 256), "odp256_b13": ("odp", 256),
-             "odp256_drop": ("odp", 256),
+             "odp256_drop": ("odp", 256), "odp256_mask": ("odp", 256),
              "stack32": ("stack", 32)}
 STACK_LAYERS = 32
-ODP_BITS = {"odp256": 20, "odp256_b16": 16, "odp256_b13": 13, "odp256_drop": 20}
+ODP_BITS = {"odp256": 20, "odp256_b16": 16, "odp256_b13": 13, "odp256_drop": 20, "odp256_mask": 20}
 ODP_DROP = {"odp256_drop": 0.02}  # fraction of tokens whose experts are all masked (Sec. 3.2, Fig. 9)
+# workloads whose step first computes the protect mask from an attention map (Eq. 6):
+# heads of the synthetic causal attention, fraction of tokens protected
+MASK_HEADS, MASK_PROTECT = 32, 0.02
 ODP_PRUNE = 0.15  # fraction of unprotected tokens whose secondary expert the threshold drops
 
 
@@ -154,6 +157,11 @@ def cpu_baseline(L, budget_s=12.0, threads=None):
     mats = [[oracle.QMat(*L.mat_shape(m), L.group, int(L.bits[e]), L.codes[e][m], L.scale[e][m], L.zero[e][m])
              for m in range(3)] for e in range(L.E)]
     xf, gf = L.x_f32(), L.gate_f32()
+    t_mask = 0.0
+    if name_has_mask(L):  # the step's Eq. 6 mask, for all tokens (charged pro rata below)
+        t0 = time.perf_counter()
+        oracle.token_importance(xf, L.attn, MASK_PROTECT)
+        t_mask = time.perf_counter() - t0
     t0 = time.perf_counter()
     oracle.moe_layer(xf, gf, mats, L.mu, L.protect, tokens=[0])
     one = time.perf_counter() - t0
@@ -163,11 +171,12 @@ def cpu_baseline(L, budget_s=12.0, threads=None):
     t0 = time.perf_counter()
     with cf.ThreadPoolExecutor(min(n, cores)) as ex:
         list(ex.map(lambda t: oracle.moe_layer(xf, gf, mats, L.mu, L.protect, tokens=[t]), toks))
-    dt = time.perf_counter() - t0
+    dt = time.perf_counter() - t0 + t_mask * n / L.T
     return {"value": n / dt, "unit": "tokens/s", "cores": min(n, cores), "kind": "oracle",
-            "single_thread_value": 1.0 / one,
-            "sample": "%d of the workload's %d tokens (full layer per token, fp64, one token per thread); "
-                      "single_thread_value: token 0 alone on one thread" % (n, L.T)}
+            "single_thread_value": 1.0 / (one + t_mask / L.T),
+            "sample": "%d of the workload's %d tokens (full layer per token, fp64, one token per thread%s); "
+                      "single_thread_value: token 0 alone on one thread" % (
+                          n, L.T, "; plus the Eq. 6 mask of all tokens, charged n/T of its time" if t_mask else "")}
 
 
 def cpu_baseline_stack(L, gates, mus, budget_s=12.0, threads=None):
@@ -224,9 +233,10 @@ def run_reference(args):
         mus = _stack_mus_oracle(L, gates)
     if kind == "odp":
         import oracle
+        if name_has_mask(L):
+            L.protect = oracle.token_importance(L.x_f32(), L.attn, MASK_PROTECT)[1]
         _, w, _ = oracle.route(L.x_f32(), L.gate_f32(), 0.0, L.protect)
-        ratio = w[:, 1].astype(np.float64) / w[:, 0]
-        L.mu = float(np.quantile(ratio[L.protect == 0], ODP_PRUNE))
+        L.mu = oracle.odp_threshold(w, L.protect, ODP_PRUNE)
     steps = args.steps if args.steps else 3
     vals = []
     cb = None
@@ -260,6 +270,10 @@ def _workload(name):
         L = synth.config_odp(T=T, bits_total=ODP_BITS[name])
         if name in ODP_DROP:
             L.protect = synth.importance_mask(L.x, 0.10, ODP_DROP[name], 1238)
+    if name.endswith("_mask"):
+        # the step computes the protect mask from this attention map (Eq. 6)
+        L.mask_step = True
+        L.attn = synth.causal_attention(MASK_HEADS, T, 1240)
     return kind, T, L
 
 
@@ -271,6 +285,13 @@ def _describe(kind, T, L):
                 "secondary expert of %d%% of unprotected tokens), %d%% of tokens protected, whole stack in one "
                 "CUDA graph" % (STACK_LAYERS, T, list(map(int, L.bits)), L.mean_bits(), round(100 * ODP_PRUNE),
                                 round(100 * float((L.protect == 1).mean()))))
+    if name_has_mask(L):
+        return ("mixtral-8x7b MoE layer %s, %d tokens, H 4096, F 14336, 8 experts, top-2, group 128, bits %s "
+                "(mean %.2f), the step computes the protect mask of the top %d%% tokens from a %d-head causal "
+                "attention map (Eq. 6) and runs the layer with ODP (mu %.4g: drops the secondary expert of %d%% of "
+                "unprotected tokens)%s" % (kind, T, list(map(int, L.bits)), L.mean_bits(), round(100 * MASK_PROTECT),
+                                           MASK_HEADS, L.mu, round(100 * ODP_PRUNE),
+                                           ", expert loads skewed ~4:1" if kind == "prefill" else ""))
     if kind == "odp":
         odp = "ODP on (mu %.4g: drops the secondary expert of %d%% of unprotected tokens), %d%% of tokens " \
               "protected by the importance surrogate" % (L.mu, round(100 * ODP_PRUNE),
@@ -283,6 +304,10 @@ def _describe(kind, T, L):
     return ("mixtral-8x7b MoE layer %s, %d tokens, H 4096, F 14336, 8 experts, top-2, group 128, bits %s "
             "(mean %.2f), %s%s" % (kind, T, list(map(int, L.bits)), L.mean_bits(), odp,
                                    ", expert loads skewed ~4:1" if kind == "prefill" else ""))
+
+
+def name_has_mask(L):
+    return getattr(L, "mask_step", False)
 
 
 def _odp_threshold(mc, x, gw, shape, protect_np, protect_dev):
@@ -361,13 +386,24 @@ def run(args):
     x = torch.from_numpy(L.x.view(np.int16).copy()).view(torch.bfloat16).to(dev)
     gw = torch.from_numpy(L.gate.view(np.int16).copy()).view(torch.bfloat16).to(dev)
     prot = None if L.protect is None else torch.from_numpy(L.protect.copy()).to(dev)
-    if kind == "odp":
+    attn = imp = None
+    if name_has_mask(L):
+        # the protect mask comes from the step itself (Eq. 6 on the attention map)
+        attn = torch.from_numpy(L.attn).to(dev)
+        imp = torch.empty(T, dtype=torch.float32, device=dev)
+        prot = torch.empty(T, dtype=torch.uint8, device=dev)
+        iws = torch.empty(mc.load().mc_token_importance_workspace_size(T), dtype=torch.uint8, device=dev)
+        mc.token_importance(x, attn, MASK_PROTECT, importance=imp, mask=prot, workspace=iws)
+        L.protect = prot.cpu().numpy()
+    if kind == "odp" or attn is not None:
         L.mu = _odp_threshold(mc, x, gw, shape, L.protect, prot)
     mu = float(L.mu)
     ws = mc.alloc_workspace(shape, T, dev)
     y = torch.empty_like(x)
 
     def step(i):
+        if attn is not None:
+            mc.token_importance(x, attn, MASK_PROTECT, importance=imp, mask=prot, workspace=iws)
         return mc.moe_forward(x, gw, shape, L.bits, packed[i % nsets], mu, prot, y=y, workspace=ws)
 
     # routing once, to know which experts a step touches and how many pairs it keeps (fixed inputs)

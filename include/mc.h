@@ -227,10 +227,14 @@ int mc_stack_forward(void *h, int T, const mc_shape *shape, int layers, const vo
  *                           (a product within 1e-6 of an integer counts as it)
  *                           (ties to the lower index), 0 for the others -- the
  *                           protect input of mc_route / mc_moe_forward.
- * Deterministic (fixed summation order); asynchronous on `stream`.
+ *   workspace: device scratch of at least mc_token_importance_workspace_size(L)
+ *           bytes, 8-byte aligned (no initial contents needed).
+ * Deterministic: the column sums are accumulated in 2^-40 fixed point with
+ * integer atomics; asynchronous on `stream`.
  * ------------------------------------------------------------------------ */
+size_t mc_token_importance_workspace_size(int L);
 int mc_token_importance(const void *t, const float *attn, int L, int H, int nh, float protect_frac,
-                        float *importance, uint8_t *mask, void *stream);
+                        float *importance, uint8_t *mask, void *workspace, size_t ws_bytes, void *stream);
 
 /* The Eq. 5 threshold from calibration routing weights (Sec. 2.3.1: the median
  * of w1/w0 over calibration data is q = 0.5): the q-quantile, linear between
@@ -271,7 +275,8 @@ int mc_check_status(void *workspace, void *stream);
  * the launching stream (for benchmarks; off by default).  mc_profile_read
  * synchronises on the recorded events, writes the summed milliseconds and launch
  * counts of kernel ids 0 .. n-1 (names from mc_profile_name: route, permute,
- * gemv_w13, gemv_w2, combine, gemm_gather, gemm_w13, gemm_w2, rmsnorm, glu) and
+ * gemv_w13, gemv_w2, combine, gemm_gather, gemm_w13, gemm_w2, rmsnorm, glu,
+ * importance) and
  * clears the records.  Inside stream capture the events become event nodes of
  * the graph: every replay records them again, and each mc_profile_read reports
  * the latest replay and keeps those records until mc_profile_clear. */

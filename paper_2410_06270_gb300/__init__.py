@@ -71,7 +71,8 @@ def load():
         "mc_rmsnorm": (I, [P, P, I, I, F32, P, P]),
         "mc_add": (I, [P, P, Z, P, P]),
         "mc_selftest_umma": (I, [P, P, P, I, I, P, P]),
-        "mc_token_importance": (I, [P, P, I, I, I, F32, P, P, P]),
+        "mc_token_importance_workspace_size": (Z, [I]),
+        "mc_token_importance": (I, [P, P, I, I, I, F32, P, P, P, Z, P]),
         "mc_odp_threshold_host": (I, [P, P, I, ctypes.c_double, P]),
         "mc_profile_enable": (I, [I]),
         "mc_profile_select": (ctypes.c_uint, [ctypes.c_uint]),
@@ -348,10 +349,11 @@ def add(a, b, out=None):
 
 # -------------------------------------------------------------- profiling --
 
-N_KERNELS = 10
+N_KERNELS = 11
 
 
-def token_importance(t, attn, protect_frac: float = 0.02, importance=None, mask=None, with_mask: bool = True):
+def token_importance(t, attn, protect_frac: float = 0.02, importance=None, mask=None, with_mask: bool = True,
+                     workspace=None):
     """Eq. 6 token importance of the tokens t (bf16 [L, H]) from the block's
     attention probabilities attn (fp32 [nh, L, L], query-major) and the protect
     mask of the top ceil(protect_frac * L) tokens.  Returns (importance, mask)."""
@@ -363,8 +365,12 @@ def token_importance(t, attn, protect_frac: float = 0.02, importance=None, mask=
         importance = torch.empty(L, dtype=torch.float32, device=t.device)
     if with_mask and mask is None:
         mask = torch.empty(L, dtype=torch.uint8, device=t.device)
+    if workspace is None:
+        workspace = torch.empty(max(1, load().mc_token_importance_workspace_size(L)), dtype=torch.uint8,
+                                device=t.device)
     _check(load().mc_token_importance(_ptr(t), _ptr(attn), L, H, nh, float(protect_frac), _ptr(importance),
-                                      _ptr(mask) if with_mask else None, _stream()))
+                                      _ptr(mask) if with_mask else None, _ptr(workspace), workspace.numel(),
+                                      _stream()))
     return importance, mask
 
 

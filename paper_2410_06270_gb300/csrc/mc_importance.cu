@@ -6,12 +6,12 @@
 //   Abar = the mean over the nh heads of the attention probabilities attn[h][i][j]
 //          (query i, key j; a causal map, so key j is seen by queries i >= j)
 //
-// colsum_kernel: one CTA per 32 key columns, 32 row lanes x 32 columns: lane r
-//   adds rows i = j0 + r, j0 + r + 32, ... (i >= j) of every head in order, reading
-//   128 contiguous bytes of a row per warp; the CTA adds its 32 row lanes in order,
-//   so the result does not depend on scheduling.
-// importance_kernel: one warp per token: the l1 norm of t_j, times the column mean
-//   (the column sums are staged in the importance buffer itself).
+// colsum_kernel: one CTA per (32 key columns, head, 256-row chunk), 32 columns
+//   x 8 row lanes, reading 128 contiguous bytes of a row per warp; each CTA adds
+//   its partial column sums to a fixed-point (2^-40) int64 accumulator with
+//   integer atomics, which commute, so the result does not depend on the order
+//   the CTAs run in (the partial of a CTA is a fixed sequence of fp32 adds).
+// importance_kernel: one warp per token: the l1 norm of t_j, times the column mean.
 // select_kernel: one CTA: radix select of the n-th largest importance (8 bits per
 //   pass over the float bit patterns, which order like the values for
 //   non-negative floats), then the mask: every token above that value and, among
@@ -25,35 +25,48 @@
 
 #include "mc_host.h"
 #include "mc_kernels.h"
+#include "mc_profile.h"
 
 namespace mc {
 
-constexpr int kColTile = 32;
+constexpr int kColTile = 32, kRowChunk = 256, kRowLanes = 8;
+constexpr double kFix = 1099511627776.0;  // 2^40: fixed-point scale of the column sums
 
-__global__ void __launch_bounds__(1024) colsum_kernel(const float *attn, int L, int nh, float *colsum)
+__global__ void zero_kernel(unsigned long long *acc, int L)
 {
-    __shared__ float part[32][kColTile + 1];
+    pdl_trigger();
+    pdl_wait();
+    const int j = blockIdx.x * blockDim.x + threadIdx.x;
+    if (j < L) acc[j] = 0ull;
+}
+
+__global__ void __launch_bounds__(kColTile * kRowLanes) colsum_kernel(const float *attn, int L, unsigned long long *acc)
+{
+    __shared__ float part[kRowLanes][kColTile + 1];
     pdl_trigger();
     pdl_wait();
     const int c = threadIdx.x & 31, r = threadIdx.x >> 5;
-    const int j0 = blockIdx.x * kColTile, j = j0 + c;
-    float acc = 0.f;
+    const int j0 = blockIdx.x * kColTile, j = j0 + c, h = blockIdx.y;
+    const int i0 = max(j0, blockIdx.z * kRowChunk), i1 = min(L, (blockIdx.z + 1) * kRowChunk);
+    if (i0 >= i1) return;  // the chunk lies above the tile's diagonal (whole CTA)
+    const float *a = attn + (size_t)h * L * L;
+    float s = 0.f;
     if (j < L)
-        for (int h = 0; h < nh; ++h) {
-            const float *a = attn + (size_t)h * L * L;
-            for (int i = j0 + r; i < L; i += 32)
-                if (i >= j) acc += a[(size_t)i * L + j];
-        }
-    part[r][c] = acc;
+#pragma unroll 4
+        for (int i = i0 + r; i < i1; i += kRowLanes)
+            if (i >= j) s += a[(size_t)i * L + j];
+    part[r][c] = s;
     __syncthreads();
     if (r == 0 && j < L) {
-        float s = 0.f;
-        for (int q = 0; q < 32; ++q) s += part[q][c];
-        colsum[j] = s;
+        float t = 0.f;
+#pragma unroll
+        for (int q = 0; q < kRowLanes; ++q) t += part[q][c];
+        atomicAdd(acc + j, (unsigned long long)llrint((double)t * kFix));
     }
 }
 
-__global__ void __launch_bounds__(256) importance_kernel(const __nv_bfloat16 *t, int L, int H, int nh, float *imp)
+__global__ void __launch_bounds__(256) importance_kernel(const __nv_bfloat16 *t, int L, int H, int nh,
+                                                         const unsigned long long *acc, float *imp)
 {
     pdl_trigger();
     pdl_wait();
@@ -63,7 +76,7 @@ __global__ void __launch_bounds__(256) importance_kernel(const __nv_bfloat16 *t,
     float l1 = 0.f;
     for (int h = lane; h < H; h += 32) l1 += fabsf(__bfloat162float(row[h]));
     for (int m = 16; m >= 1; m >>= 1) l1 += __shfl_xor_sync(0xffffffffu, l1, m);
-    if (lane == 0) imp[j] = l1 * (imp[j] / ((float)nh * (float)(L - j)));
+    if (lane == 0) imp[j] = (float)((double)l1 * ((double)acc[j] / kFix) / ((double)nh * (double)(L - j)));
 }
 
 __global__ void __launch_bounds__(1024) select_kernel(const float *imp, int L, int n, uint8_t *mask)
@@ -142,28 +155,47 @@ using namespace mc;
 
 extern "C" {
 
+size_t mc_token_importance_workspace_size(int L) { return L <= 0 ? 0 : (((size_t)L * 8 + 255) & ~(size_t)255); }
+
 int mc_token_importance(const void *t, const float *attn, int L, int H, int nh, float protect_frac,
-                        float *importance, uint8_t *mask, void *stream)
+                        float *importance, uint8_t *mask, void *workspace, size_t ws_bytes, void *stream)
 {
     clear_error();
-    if (L < 0 || H <= 0 || nh <= 0 || !(protect_frac >= 0.f && protect_frac <= 1.f))
+    if (L < 0 || H <= 0 || nh <= 0 || nh > 65535 || !(protect_frac >= 0.f && protect_frac <= 1.f))
         return set_error(MC_ERR_INVALID_ARG, "L=%d H=%d nh=%d protect_frac=%g", L, H, nh, (double)protect_frac);
     if (L == 0) return MC_OK;
-    if (!t || !attn || !importance) return set_error(MC_ERR_INVALID_ARG, "NULL pointer argument");
-    if ((double)nh * L * L > 9.0e18 / 4) return set_error(MC_ERR_INVALID_ARG, "attention map too large");
+    if (!t || !attn || !importance || !workspace) return set_error(MC_ERR_INVALID_ARG, "NULL pointer argument");
+    if (ws_bytes < mc_token_importance_workspace_size(L))
+        return set_error(MC_ERR_INVALID_ARG, "workspace has %zu bytes, needs %zu", ws_bytes,
+                         mc_token_importance_workspace_size(L));
+    if ((double)nh * L * L > 9.0e18 / 4 || (double)nh * L > 2.0e9 * kRowChunk)
+        return set_error(MC_ERR_INVALID_ARG, "attention map too large");
     cudaStream_t st = (cudaStream_t)stream;
-    cudaError_t err = launch_k(colsum_kernel, dim3((L + kColTile - 1) / kColTile), dim3(1024), 0, st, attn, L, nh,
-                               importance);
-    if (err == cudaSuccess)
+    unsigned long long *acc = (unsigned long long *)workspace;
+    const dim3 grid((L + kColTile - 1) / kColTile, nh, (L + kRowChunk - 1) / kRowChunk);
+    profile_begin(kKImportance, st);
+    cudaError_t err = launch_k(zero_kernel, dim3((L + 255) / 256), dim3(256), 0, st, acc, L);
+    profile_end(kKImportance, st);
+    if (err == cudaSuccess) {
+        profile_begin(kKImportance, st);
+        err = launch_k(colsum_kernel, grid, dim3(kColTile * kRowLanes), 0, st, attn, L, acc);
+        profile_end(kKImportance, st);
+    }
+    if (err == cudaSuccess) {
+        profile_begin(kKImportance, st);
         err = launch_k(importance_kernel, dim3((L + 7) / 8), dim3(256), 0, st, (const __nv_bfloat16 *)t, L, H, nh,
-                       importance);
+                       (const unsigned long long *)acc, importance);
+        profile_end(kKImportance, st);
+    }
     if (err == cudaSuccess && mask) {
         // ceil(frac * L); a product within 1e-6 of an integer counts as that integer
         const int n = (int)ceil((double)protect_frac * L - 1e-6);
+        profile_begin(kKImportance, st);
         if (n <= 0 || n >= L)
             err = launch_k(fill_kernel, dim3((L + 255) / 256), dim3(256), 0, st, mask, L, (uint8_t)(n > 0));
         else
             err = launch_k(select_kernel, dim3(1), dim3(1024), 0, st, (const float *)importance, L, n, mask);
+        profile_end(kKImportance, st);
     }
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "importance launch: %s", cudaGetErrorString(err));
     return MC_OK;

@@ -16,6 +16,7 @@ enum KernelId {
     kKGemmW2,
     kKRmsnorm,
     kKGlu,
+    kKImportance,
     kKCount
 };
 

@@ -284,3 +284,18 @@ def config_prefill(T=4096, seed=1237, bits_total=20, skew=(3.0, 0.9)):
     """Mixtral-8x7b-shaped prefill layer with skewed expert loads, ODP off."""
     bits = bit_table(seed, 8, bits_total)
     return make_layer(T, MIXTRAL_H, MIXTRAL_F, MIXTRAL_E, 128, bits, seed, skew=skew)
+
+
+def causal_attention(nh, L, seed, temp=1.0):
+    """Seeded synthetic attention probabilities fp32 [nh, L, L] (query i, key j):
+    a causal softmax of standard normal scores times `temp`, one head at a time.
+    Input generation for the token-importance step (Eq. 6)."""
+    rng = _rng(seed, 6)
+    out = np.empty((nh, L, L), np.float32)
+    tri = np.tril(np.ones((L, L), bool))
+    for h in range(nh):
+        s = rng.standard_normal((L, L)) * temp
+        s = np.where(tri, s, -np.inf)
+        e = np.exp(s - s.max(axis=1, keepdims=True))
+        out[h] = e / e.sum(axis=1, keepdims=True)
+    return out
