@@ -36,6 +36,7 @@ import synth  # noqa: E402
 METRIC = "Mixed-bit MoE-layer tokens/s; % HBM roofline (decode), % TC peak (prefill)"
 HBM_NOMINAL_GBS = 7900.0  # GB300 HBM3e nominal, reported beside the measured copy peak
 WORKLOADS = {"decode16": ("decode", 16), "decode4": ("decode", 4), "decode1": ("decode", 1),
+             "decode16_8x22b": ("decode", 16),
              "prefill4096": ("prefill", 4096),
              "odp256": ("odp", 256), "odp256_b16": ("odp", 256), "odp256_b13": ("odp", 256),
              "odp256_drop": ("odp", 256), "odp256_mask": ("odp", 256),
@@ -261,7 +262,7 @@ def run_reference(args):
 def _workload(name):
     kind, T = WORKLOADS[name]
     if kind == "decode":
-        L = synth.config_decode(T=T)
+        L = synth.config_decode_22b(T=T) if name.endswith("8x22b") else synth.config_decode(T=T)
     elif kind == "prefill":
         L = synth.config_prefill(T=T)
     elif kind == "stack":
@@ -301,8 +302,9 @@ def _describe(kind, T, L):
                 100 * float((L.protect == 2).mean()))
     else:
         odp = "ODP off"
-    return ("mixtral-8x7b MoE layer %s, %d tokens, H 4096, F 14336, 8 experts, top-2, group 128, bits %s "
-            "(mean %.2f), %s%s" % (kind, T, list(map(int, L.bits)), L.mean_bits(), odp,
+    model = "mixtral-8x22b" if L.H == synth.MIXTRAL22_H else "mixtral-8x7b"
+    return ("%s MoE layer %s, %d tokens, H %d, F %d, 8 experts, top-2, group 128, bits %s "
+            "(mean %.2f), %s%s" % (model, kind, T, L.H, L.F, list(map(int, L.bits)), L.mean_bits(), odp,
                                    ", expert loads skewed ~4:1" if kind == "prefill" else ""))
 
 

@@ -28,6 +28,9 @@ import numpy as np
 MIXTRAL_H = 4096
 MIXTRAL_F = 14336
 MIXTRAL_E = 8
+# Mixtral-8x22b (Tab. model): H 6144, 8 experts; F is not in the paper: 16384
+MIXTRAL22_H = 6144
+MIXTRAL22_F = 16384
 
 
 # ----------------------------------------------------------------- formats --
@@ -278,6 +281,13 @@ def config_stack(T=32, layers=32, seed=1239, bits_total=20, protect_frac=0.10, H
     L.protect = importance_protect(L.x, protect_frac, seed)
     gates = [gaussian_bf16(seed, (6, l), (E, H), gate_std) for l in range(layers)]
     return L, gates
+
+
+def config_decode_22b(T=16, seed=1241, bits_total=20):
+    """Mixtral-8x22b-shaped decode layer: H 6144, F 16384, 8 experts, group 128,
+    bits from {1,2,3} with sum 20 (mean 2.5), ODP off."""
+    bits = bit_table(seed, 8, bits_total)
+    return make_layer(T, MIXTRAL22_H, MIXTRAL22_F, MIXTRAL_E, 128, bits, seed)
 
 
 def config_prefill(T=4096, seed=1237, bits_total=20, skew=(3.0, 0.9)):

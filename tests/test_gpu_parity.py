@@ -191,6 +191,12 @@ def test_forward_mixtral_decode(mc, T):
     _forward_and_check(mc, L, tokens=tokens)
 
 
+def test_forward_mixtral_8x22b_decode(mc):
+    """Mixtral-8x22b-shaped decode layer (H 6144, F 16384, group 128, mean 2.5
+    bits), outputs on sampled tokens, routing on all tokens."""
+    _forward_and_check(mc, synth.config_decode_22b(T=16), tokens=[0, 9, 15])
+
+
 def test_forward_is_deterministic(mc):
     L = synth.make_layer(16, 256, 512, 8, 64, [3, 2, 2, 1, 3, 2, 2, 3], 80, gate_std=0.1)
     shape, packed = _pack(mc, L)
