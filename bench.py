@@ -36,7 +36,7 @@ import synth  # noqa: E402
 METRIC = "Mixed-bit MoE-layer tokens/s; % HBM roofline (decode), % TC peak (prefill)"
 HBM_NOMINAL_GBS = 7900.0  # GB300 HBM3e nominal, reported beside the measured copy peak
 WORKLOADS = {"decode16": ("decode", 16), "decode4": ("decode", 4), "decode1": ("decode", 1),
-             "decode16_8x22b": ("decode", 16),
+             "decode16_8x22b": ("decode", 16), "decode16_fp16": ("decode", 16),
              "prefill4096": ("prefill", 4096),
              "odp256": ("odp", 256), "odp256_b16": ("odp", 256), "odp256_b13": ("odp", 256),
              "odp256_drop": ("odp", 256), "odp256_mask": ("odp", 256),
@@ -142,7 +142,8 @@ def job_throughput(world, units_per_rank, steps, ms):
 def _algorithmic_bytes(shape, bits, touched, T, H):
     """Packed weight bytes of the touched experts (codes + fp16 scale/zero) plus
     the gate, activations and output.  Returns (total, w13 part)."""
-    per_mat = lambda b: H * shape.F * b / 8 + H * shape.F / shape.group * 4
+    # 16-bit (unquantised) experts carry no scale / zero
+    per_mat = lambda b: H * shape.F * b / 8 + (0 if b == 16 else H * shape.F / shape.group * 4)
     w13 = sum(2 * per_mat(int(bits[e])) for e in touched)
     w2 = sum(per_mat(int(bits[e])) for e in touched)
     other = shape.E * H * 2 + 2 * T * H * 2
@@ -262,7 +263,8 @@ def run_reference(args):
 def _workload(name):
     kind, T = WORKLOADS[name]
     if kind == "decode":
-        L = synth.config_decode_22b(T=T) if name.endswith("8x22b") else synth.config_decode(T=T)
+        L = synth.config_decode_22b(T=T) if name.endswith("8x22b") else \
+            synth.config_decode_fp16(T=T) if name.endswith("fp16") else synth.config_decode(T=T)
     elif kind == "prefill":
         L = synth.config_prefill(T=T)
     elif kind == "stack":
@@ -303,6 +305,8 @@ def _describe(kind, T, L):
     else:
         odp = "ODP off"
     model = "mixtral-8x22b" if L.H == synth.MIXTRAL22_H else "mixtral-8x7b"
+    if int(L.bits[0]) == 16:
+        odp += ", experts unquantised (fp16 weights: the baseline of the mixed-bit layer)"
     return ("%s MoE layer %s, %d tokens, H %d, F %d, 8 experts, top-2, group 128, bits %s "
             "(mean %.2f), %s%s" % (model, kind, T, L.H, L.F, list(map(int, L.bits)), L.mean_bits(), odp,
                                    ", expert loads skewed ~4:1" if kind == "prefill" else ""))
@@ -511,7 +515,9 @@ def run(args):
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": steps,
         "warmup": args.warmup, "ms_per_step": ms / steps, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "f16 x {1,2,3}-bit codes, fp32 accumulate", "data": "synthetic",
+        "vs_baseline": None, "data": "synthetic",
+        "dtype": "f16 x f16 (unquantised experts), fp32 accumulate" if int(L.bits[0]) == 16 else
+                 "f16 x {1,2,3}-bit codes, fp32 accumulate",
         "config": {"workload": _describe(kind, T, L),
                    "global_batch": T * world, "parallelism": "replicas" if world > 1 else "single",
                    "l2": "inputs larger than L2: %d rotating copies of the %.0f MB packed weights"

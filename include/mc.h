@@ -44,7 +44,7 @@ extern "C" {
 enum {
     MC_OK = 0,
     MC_ERR_INVALID_ARG = -1, /* null/misaligned pointer, bad shape, bad mu, ... */
-    MC_ERR_UNSUPPORTED = -2, /* a bit width outside {1,2,3}, E > 16, ... */
+    MC_ERR_UNSUPPORTED = -2, /* a bit width outside {1,2,3,16}, E > 16, ... */
     MC_ERR_CUDA = -3,        /* a CUDA runtime call failed (message has the text) */
     MC_ERR_TIMEOUT = -4,     /* a bounded device wait expired (status word) */
     MC_ERR_BAD_PACK = -5,    /* packed buffer header does not match (magic/shape/bits) */
@@ -72,6 +72,9 @@ int mc_pack_format_version(void);
  *   codes  uint8 [rows*cols], one code per byte, value < 2^bits[e]
  *   scale  fp16 bit patterns [rows, cols/group]
  *   zero   fp16 bit patterns [rows, cols/group]
+ * bits[e] = 16 (the unquantised fp16 baseline; all experts of a layer or none):
+ * codes is the matrix itself as fp16 bit patterns (uint16 [rows*cols], passed
+ * through the uint8 pointer) and scale / zero are unused (may be NULL).
  * The packed layout is private to this library and versioned by a header at the
  * start of the buffer; only its total size is part of the ABI.
  * ------------------------------------------------------------------------ */
@@ -83,7 +86,8 @@ size_t mc_packed_size(const mc_shape *shape, const int8_t *bits_host);
 /* Pack canonical host arrays into a HOST buffer of mc_packed_size() bytes.  The
  * arrays are indexed [3*e + m].  Pure host code (no GPU needed).  Returns
  * MC_ERR_INVALID_ARG for a code >= 2^bits, a null array or a short buffer;
- * MC_ERR_UNSUPPORTED for a bit width outside {1,2,3}. */
+ * MC_ERR_UNSUPPORTED for a bit width outside {1,2,3,16} or 16-bit experts mixed
+ * with quantised ones. */
 int mc_pack_experts_host(const mc_shape *shape, const int8_t *bits_host,
                          const uint8_t *const *codes_host,
                          const uint16_t *const *scale_host,
@@ -100,8 +104,9 @@ int mc_pack_experts(const mc_shape *shape, const int8_t *bits_host,
 
 /* Inverse of the packing for one (expert, matrix), from a HOST packed buffer:
  * writes canonical codes [rows*cols] and fp16 scale/zero [rows, cols/group]
- * (scale_host / zero_host may be NULL).  Pure host code.  MC_ERR_BAD_PACK if
- * the header is not a valid packed buffer. */
+ * (scale_host / zero_host may be NULL); a 16-bit expert's fp16 weights go to
+ * codes_host as uint16 [rows*cols].  Pure host code.  MC_ERR_BAD_PACK if the
+ * header is not a valid packed buffer. */
 int mc_unpack_experts_host(const void *packed_host, size_t packed_bytes, int expert, int mat,
                            uint8_t *codes_host, uint16_t *scale_host, uint16_t *zero_host);
 

@@ -119,7 +119,7 @@ class _PtrArray:
 
     def __init__(self, arrs):
         self.arrs = arrs
-        self.arr = (ctypes.c_void_p * len(arrs))(*[a.ctypes.data for a in arrs])
+        self.arr = (ctypes.c_void_p * len(arrs))(*[None if a is None else a.ctypes.data for a in arrs])
 
     @property
     def as_parameter(self):
@@ -144,17 +144,23 @@ def packed_size(shape: Shape, bits) -> int:
     return n
 
 
-def _canon(codes, scales, zeros):
-    c = [np.ascontiguousarray(a, dtype=np.uint8) for a in codes]
-    s = [np.ascontiguousarray(np.asarray(a, dtype=np.float16)).view(np.uint16) for a in scales]
-    z = [np.ascontiguousarray(np.asarray(a, dtype=np.float16)).view(np.uint16) for a in zeros]
+def _canon(codes, scales, zeros, bits=None):
+    """Host arrays for the pack entry points: uint8 codes and fp16 scale / zero;
+    a 16-bit expert's codes are its fp16 weights and its scale / zero are None."""
+    dense = [bits is not None and int(bits[i // 3]) == 16 for i in range(len(codes))]
+    c = [np.ascontiguousarray(np.asarray(a, dtype=np.float16)).view(np.uint16) if d
+         else np.ascontiguousarray(a, dtype=np.uint8) for a, d in zip(codes, dense)]
+    s = [None if d else np.ascontiguousarray(np.asarray(a, dtype=np.float16)).view(np.uint16)
+         for a, d in zip(scales, dense)]
+    z = [None if d else np.ascontiguousarray(np.asarray(a, dtype=np.float16)).view(np.uint16)
+         for a, d in zip(zeros, dense)]
     return c, s, z
 
 
 def pack_experts_host(shape: Shape, bits, codes, scales, zeros) -> np.ndarray:
     """codes/scales/zeros: flat lists of 3*E arrays indexed [3*e + m]."""
     b = _bits(bits)
-    c, s, z = _canon(codes, scales, zeros)
+    c, s, z = _canon(codes, scales, zeros, b)
     n = packed_size(shape, b)
     out = np.empty(n, np.uint8)
     _check(load().mc_pack_experts_host(ctypes.byref(shape), b.ctypes.data, _ptr_array(c, None),
@@ -175,7 +181,7 @@ def pack_experts(shape: Shape, bits, codes, scales, zeros, device="cuda"):
     """Pack and upload; returns a uint8 device tensor (synchronous)."""
     import torch
     b = _bits(bits)
-    c, s, z = _canon(codes, scales, zeros)
+    c, s, z = _canon(codes, scales, zeros, b)
     n = packed_size(shape, b)
     dst = torch.empty(n, dtype=torch.uint8, device=device)
     _check(load().mc_pack_experts(ctypes.byref(shape), b.ctypes.data, _ptr_array(c, None), _ptr_array(s, None),

@@ -216,7 +216,11 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     // expert path: many pairs per expert -> tensor-core grouped GEMM (prefill),
     // few -> mma.sync grouped GEMV (decode); mc_set_path overrides
     int path = g_path;
-    if (path == 0) path = 2 * T >= kPrefillPairs ? 3 : 1;
+    // 16-bit (unquantised) experts have the mma.sync kernels only
+    const bool dense = bits_host[0] == 16;
+    if (path == 0) path = dense ? 1 : 2 * T >= kPrefillPairs ? 3 : 1;
+    if (dense && path != 1)
+        return set_error(MC_ERR_UNSUPPORTED, "16-bit experts run on the mma.sync path only (path %d requested)", path);
 
     RouteParams rp{};
     memset(&rp, 0, sizeof rp);

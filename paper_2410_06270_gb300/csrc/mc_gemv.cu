@@ -58,16 +58,20 @@ static_assert(256 + sizeof(RingShared) <= 1024, "ring header");
 
 constexpr int kVecMax = kVecFragBytes + 8 * 2 * kTabFloats * 4;  // vec_bytes(64), the largest
 
-__host__ __device__ inline int slot_bytes(int group)
+// Column steps per ring stage: kKPS for quantised experts; one for 16-bit experts,
+// whose two supertiles per step are already 64 KB.
+__host__ __device__ inline int stage_steps(bool dense) { return dense ? 1 : kKPS; }
+__host__ __device__ inline int slot_bytes(int group, bool dense)
 {
-    return kKPS * 2 * supertile_bytes(3, group) + 2 * kKPS * kVecMax;
+    const int kps = stage_steps(dense);
+    return kps * 2 * supertile_bytes(dense ? 16 : 3, group) + 2 * kps * kVecMax;
 }
 constexpr int kHsBytes = kChunk * kTileK * 2;           // h tile [16][128] fp16 (two of them)
 constexpr int kXbufBytes = kTPW == 1 ? 8 * 32 * 8 * 4 : 0;  // W3 results handed to the W1 warps
 
-__host__ __device__ inline size_t gemv_smem(int nslots, int group)
+__host__ __device__ inline size_t gemv_smem(int nslots, int group, bool dense)
 {
-    return kRingOff + (size_t)nslots * slot_bytes(group) + 2 * kHsBytes + kXbufBytes + 8 * 32 * sizeof(uint2);
+    return kRingOff + (size_t)nslots * slot_bytes(group, dense) + 2 * kHsBytes + kXbufBytes + 8 * 32 * sizeof(uint2);
 }
 
 // Bounded wait that gives up as soon as another thread of the CTA aborted.
@@ -345,6 +349,37 @@ __device__ __forceinline__ void step_tiles(const uint8_t *const (&tile)[NTL], co
     }
 }
 
+// One 128-column step of 16-bit (unquantised fp16) tiles: the A fragments are
+// loaded as stored (one 16-byte load per k-step) and multiplied straight into y;
+// there is no quantisation group to fold.
+template <int NT, int NTL>
+__device__ __forceinline__ void step_dense(const uint8_t *const (&tile)[NTL], const uint8_t *vec0,
+                                           const uint8_t *vec1, int lane, float (&y)[NTL][NT][4])
+{
+#pragma unroll
+    for (int qd = 0; qd < 4; ++qd) {
+        uint4 a[NTL][2];
+#pragma unroll
+        for (int u = 0; u < NTL; ++u) {
+            const uint4 *t4 = reinterpret_cast<const uint4 *>(tile[u] + 128 * lane) + 2 * qd;
+            a[u][0] = t4[0];
+            a[u][1] = t4[1];
+        }
+        uint4 bq[NT];
+#pragma unroll
+        for (int j = 0; j < NT; ++j) bq[j] = reinterpret_cast<const uint4 *>(j ? vec1 : vec0)[qd * 32 + lane];
+#pragma unroll
+        for (int kk = 0; kk < 2; ++kk)
+#pragma unroll
+            for (int j = 0; j < NT; ++j) {
+                const uint32_t b0 = kk ? bq[j].z : bq[j].x, b1 = kk ? bq[j].w : bq[j].y;
+#pragma unroll
+                for (int u = 0; u < NTL; ++u)
+                    mma_acc(y[u][j], reinterpret_cast<const uint32_t *>(&a[u][kk]), b0, b1);
+            }
+    }
+}
+
 struct Item {
     int k, u;          // chunk, unit
     ChunkInfo ci;
@@ -409,6 +444,7 @@ __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, 
                                          __half *hs2, int &items, int &cbar_uses)
 {
     constexpr int group = kTileK / GPT;
+    constexpr int KPS = BITS == 16 ? 1 : kKPS;  // stage_steps
     const int STB = supertile_bytes(BITS, group), TB = tile_bytes(BITS, group);
     const int pw = W13 ? 2 : w2_pair_width(I.blkA >> 1, nrb);
     const int step_bytes = pw * STB;
@@ -422,19 +458,22 @@ __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, 
         for (int j = 0; j < NT; ++j)
 #pragma unroll
             for (int c = 0; c < 4; ++c) y[u][j][c] = 0.f;
-    for (int i = 0; i < I.nkt; i += kKPS) {
+    for (int i = 0; i < I.nkt; i += KPS) {
         if (i > 0 && !wait_or_abort(&R.full[slot], phase, p, sh)) return false;
         const uint8_t *base = R.base + (size_t)slot * R.SB;
         const int kc = sh->slot_kc[slot];
-        const uint8_t *v0 = base + R.vec_off0, *v1 = v0 + kKPS * R.VB;
+        const uint8_t *v0 = base + R.vec_off0, *v1 = v0 + KPS * R.VB;
 #pragma unroll
-        for (int kk = 0; kk < kKPS; ++kk)
+        for (int kk = 0; kk < KPS; ++kk)
             if (kk < kc) {
                 const uint8_t *st = base + kk * step_bytes;
                 const uint8_t *t[kTPW];
 #pragma unroll
                 for (int u = 0; u < kTPW; ++u) t[u] = st + off[u];
-                step_tiles<NT, BITS, GPT, kTPW>(t, v0 + kk * R.VB, v1 + kk * R.VB, lane, y);
+                if constexpr (BITS == 16)
+                    step_dense<NT, kTPW>(t, v0 + kk * R.VB, v1 + kk * R.VB, lane, y);
+                else
+                    step_tiles<NT, BITS, GPT, kTPW>(t, v0 + kk * R.VB, v1 + kk * R.VB, lane, y);
             }
         __syncwarp();
         if (lane == 0) mbar_arrive(&R.empty[slot]);
@@ -504,7 +543,7 @@ __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, 
     return true;
 }
 
-template <bool W13, int GPT>
+template <bool W13, int GPT, bool DENSE>
 __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
 {
     extern __shared__ __align__(1024) uint8_t smem[];
@@ -513,8 +552,9 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
     RingShared *sh = reinterpret_cast<RingShared *>(smem + 256);
     uint8_t *ring = smem + kRingOff;
     const int S = p.nslots, group = p.group;
-    const int SB = slot_bytes(group), VB = vec_bytes(group);
-    const int vec_off0 = kKPS * 2 * supertile_bytes(3, group);
+    constexpr int KPS = DENSE ? 1 : kKPS;  // stage_steps(DENSE)
+    const int SB = slot_bytes(group, DENSE), VB = vec_bytes(group);
+    const int vec_off0 = KPS * 2 * supertile_bytes(DENSE ? 16 : 3, group);
     __half *hs2 = reinterpret_cast<__half *>(smem + kRingOff + (size_t)S * SB);
     float *xbuf = reinterpret_cast<float *>(smem + kRingOff + (size_t)S * SB + 2 * kHsBytes);
     uint2 *afr = reinterpret_cast<uint2 *>(smem + kRingOff + (size_t)S * SB + 2 * kHsBytes + kXbufBytes);
@@ -565,7 +605,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
                 ChunkInfo next_ci = ci;
                 bool have_ci = false;
                 const Item I = decode_item<W13>(p, item, U, ci);
-                const int nst = (I.nkt + kKPS - 1) / kKPS, claim_at = nst > 1 ? nst - 2 : 0;
+                const int nst = (I.nkt + KPS - 1) / KPS, claim_at = nst > 1 ? nst - 2 : 0;
                 const int bits = I.ci.bits, NT = I.ci.nv > 8 ? 2 : 1;
                 const int e = I.ci.e;
                 const int STB = supertile_bytes(bits, group);
@@ -573,7 +613,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
                 const int pw = W13 ? 2 : w2_pair_width(I.blkA >> 1, nrb);
                 const uint8_t *wsrc =
                     p.packed + p.mat_off[e][W13 ? 0 : 2] + supertile_off(W13 ? 0 : 2, I.blkA, I.kt0, KTm, nrb, STB);
-                for (int i = 0, st = 0; i < I.nkt; i += kKPS, ++it, ++st) {
+                for (int i = 0, st = 0; i < I.nkt; i += KPS, ++it, ++st) {
                     const int slot = pslot;
                     if (it >= S && !wait_or_abort(&empty[slot], pphase ^ 1u, p, sh)) {
                         ok = false;
@@ -583,7 +623,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
                         pslot = 0;
                         pphase ^= 1u;
                     }
-                    const int kc = min(kKPS, I.nkt - i);
+                    const int kc = min(KPS, I.nkt - i);
                     sh->slot_item[slot] = item;
                     sh->slot_ci[slot] = I.ci;
                     sh->slot_kc[slot] = kc;
@@ -592,7 +632,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
                     mbar_arrive_expect_tx(&full[slot], wb + NT * vb);
                     bulk_g2s_stream(dst, wsrc + (size_t)i * pw * STB, wb, &full[slot], pol);
                     for (int j = 0; j < NT; ++j)
-                        bulk_g2s(dst + vec_off0 + j * kKPS * VB, vbase + vec_off(I.k, j, I.kt0 + i, KTm, group), vb,
+                        bulk_g2s(dst + vec_off0 + j * KPS * VB, vbase + vec_off(I.k, j, I.kt0 + i, KTm, group), vb,
                                  &full[slot]);
                     sh->issued = it + 1;
                     if (st == claim_at) {
@@ -633,7 +673,9 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
             bool ok;
 #define MC_RUN(NT_, B_) \
     run_item<W13, NT_, B_, GPT>(p, sh, R, I, nrb, x, tl, lane, slot, phase, xbuf, hs2, items, cbar_uses)
-            switch (sel) {
+            if constexpr (DENSE) {
+                ok = I.ci.nv > 8 ? MC_RUN(2, 16) : MC_RUN(1, 16);
+            } else switch (sel) {
             case 0: ok = MC_RUN(1, 1); break;
             case 1: ok = MC_RUN(2, 1); break;
             case 2: ok = MC_RUN(1, 2); break;
@@ -709,13 +751,17 @@ int launch_gemv(ExpertParams ep, cudaStream_t st)
     if (err == cudaSuccess) err = cudaDeviceGetAttribute(&maxsm, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
     if (err == cudaSuccess) err = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "device query: %s", cudaGetErrorString(err));
-    int nslots = (int)((maxsm - gemv_smem(0, ep.group)) / slot_bytes(ep.group));
+    // 16-bit experts are all or none of a layer (check_bits)
+    const bool dense = ep.bits[0] == 16;
+    int nslots = (int)((maxsm - gemv_smem(0, ep.group, dense)) / slot_bytes(ep.group, dense));
     nslots = nslots > kMaxSlots ? kMaxSlots : nslots;
     if (nslots < 2) return set_error(MC_ERR_UNSUPPORTED, "not enough shared memory for the GEMV ring");
     ep.nslots = nslots;
-    const size_t sm = gemv_smem(nslots, ep.group);
-    auto k13 = ep.group == 64 ? gemv_kernel<true, 2> : gemv_kernel<true, 1>;
-    auto k2 = ep.group == 64 ? gemv_kernel<false, 2> : gemv_kernel<false, 1>;
+    const size_t sm = gemv_smem(nslots, ep.group, dense);
+    auto k13 = dense ? (ep.group == 64 ? gemv_kernel<true, 2, true> : gemv_kernel<true, 1, true>)
+                     : (ep.group == 64 ? gemv_kernel<true, 2, false> : gemv_kernel<true, 1, false>);
+    auto k2 = dense ? (ep.group == 64 ? gemv_kernel<false, 2, true> : gemv_kernel<false, 1, true>)
+                    : (ep.group == 64 ? gemv_kernel<false, 2, false> : gemv_kernel<false, 1, false>);
     err = cudaFuncSetAttribute(k13, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (err == cudaSuccess) err = cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(err));

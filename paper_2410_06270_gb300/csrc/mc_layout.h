@@ -35,6 +35,10 @@
 //   b = 1: [32 lanes x 8 B]    b = 2: [32 lanes x 16 B]
 //   b = 3: [32 lanes x 16 B: words 0..3][32 lanes x 8 B: words 4, 5]
 // Meta bytes of a tile: [group-in-tile][g8 = 0..7][s(r0), z(r0), s(r1), z(r1)] fp16.
+// 16-bit (unquantised) experts, b = 16: the tile holds the fp16 weights themselves,
+// lane-major, 128 bytes per lane = its 32 pairs in order j (pair j = the two
+// columns above, as one half2): a k-step's four A-fragment registers are one
+// 16-byte load.  No meta.
 //
 // Decoding without shifts per field: a field at mantissa bit f of an fp16 whose
 // exponent field is set to 15 + E reads as 2^E + q * 2^(E + f - 10); choosing
@@ -75,7 +79,7 @@ static_assert(sizeof(PackHeader) <= kHeaderBytes, "header");
 
 MC_HD int tile_code_bytes(int bits) { return 256 * bits; }
 MC_HD int tile_meta_bytes(int group) { return 64 * (kTileK / group); }
-MC_HD int tile_bytes(int bits, int group) { return tile_code_bytes(bits) + tile_meta_bytes(group); }
+MC_HD int tile_bytes(int bits, int group) { return tile_code_bytes(bits) + (bits == 16 ? 0 : tile_meta_bytes(group)); }
 MC_HD int supertile_bytes(int bits, int group) { return kTilesPerBlock * tile_bytes(bits, group); }
 MC_HD uint64_t mat_bytes(int rows, int cols, int bits, int group)
 {

@@ -99,6 +99,8 @@ int mc_unpack_experts(const mc_shape *shape, const int8_t *bits_host, const void
     if (!packed_dev || !codes_dev) return set_error(MC_ERR_INVALID_ARG, "NULL pointer argument");
     if (expert < 0 || expert >= shape->E || mat < 0 || mat > 2)
         return set_error(MC_ERR_INVALID_ARG, "expert %d / matrix %d out of range", expert, mat);
+    if (bits_host[expert] == 16)
+        return set_error(MC_ERR_UNSUPPORTED, "16-bit experts hold no codes (mc_unpack_experts_host reads them)");
     uint64_t off[kMaxE][3], total;
     layout_offsets(shape, bits_host, off, &total);
     const int rows = mat < 2 ? shape->F : shape->H, cols = mat < 2 ? shape->H : shape->F;

@@ -46,9 +46,17 @@ int check_bits(const mc_shape *s, const int8_t *bits)
     int rc = check_shape(s);
     if (rc) return rc;
     if (!bits) return set_error(MC_ERR_INVALID_ARG, "bits table is NULL");
-    for (int e = 0; e < s->E; ++e)
+    int n16 = 0;
+    for (int e = 0; e < s->E; ++e) {
+        if (bits[e] == 16) {
+            ++n16;
+            continue;
+        }
         if (bits[e] < 1 || bits[e] > 3)
-            return set_error(MC_ERR_UNSUPPORTED, "bits[%d]=%d: only 1, 2 or 3 bits are supported", e, bits[e]);
+            return set_error(MC_ERR_UNSUPPORTED, "bits[%d]=%d: only 1, 2, 3 or 16 bits are supported", e, bits[e]);
+    }
+    if (n16 && n16 != s->E)
+        return set_error(MC_ERR_UNSUPPORTED, "16-bit experts cannot be mixed with quantised ones");
     return MC_OK;
 }
 
@@ -69,9 +77,49 @@ void layout_offsets(const mc_shape *s, const int8_t *bits, uint64_t off[kMaxE][3
 
 // Pack one matrix [rows, cols] into its tile stream.  Returns false on a code
 // that does not fit in `bits`.
+static void pack_dense(int m, int rows, int cols, const uint16_t *w, uint8_t *dst, int rb_lo, int rb_hi)
+{
+    const int KT = cols / kTileK, nrb = rows / kBlockRows;
+    for (int rb = rb_lo; rb < rb_hi; ++rb)
+        for (int kt = 0; kt < KT; ++kt) {
+            uint16_t *tile = (uint16_t *)(dst + tile_off(m, rb, kt, KT, nrb, 16, kTileK));
+            const int R0 = rb * kTileRows, K0 = kt * kTileK;
+            for (int lane = 0; lane < 32; ++lane)
+                for (int j = 0; j < 32; ++j) {
+                    int row, col;
+                    pair_pos(lane, j, row, col);
+                    const uint16_t *src = w + (size_t)(R0 + row) * cols + K0 + col;
+                    tile[lane * 64 + 2 * j] = src[0];
+                    tile[lane * 64 + 2 * j + 1] = src[1];
+                }
+        }
+}
+
+static void unpack_dense(int m, int rows, int cols, const uint8_t *src, uint16_t *w)
+{
+    const int KT = cols / kTileK, nrb = rows / kBlockRows;
+    for (int rb = 0; rb < rows / kTileRows; ++rb)
+        for (int kt = 0; kt < KT; ++kt) {
+            const uint16_t *tile = (const uint16_t *)(src + tile_off(m, rb, kt, KT, nrb, 16, kTileK));
+            const int R0 = rb * kTileRows, K0 = kt * kTileK;
+            for (int lane = 0; lane < 32; ++lane)
+                for (int j = 0; j < 32; ++j) {
+                    int row, col;
+                    pair_pos(lane, j, row, col);
+                    uint16_t *d = w + (size_t)(R0 + row) * cols + K0 + col;
+                    d[0] = tile[lane * 64 + 2 * j];
+                    d[1] = tile[lane * 64 + 2 * j + 1];
+                }
+        }
+}
+
 static bool pack_matrix(int m, int rows, int cols, int bits, int group, const uint8_t *codes,
                         const uint16_t *scale, const uint16_t *zero, uint8_t *dst, int rb_lo, int rb_hi)
 {
+    if (bits == 16) {
+        pack_dense(m, rows, cols, (const uint16_t *)codes, dst, rb_lo, rb_hi);
+        return true;
+    }
     const int KT = cols / kTileK, ng = cols / group, gpt = kTileK / group, nrb = rows / kBlockRows;
     const uint32_t lim = 1u << bits;
     for (int rb = rb_lo; rb < rb_hi; ++rb)
@@ -115,6 +163,10 @@ static bool pack_matrix(int m, int rows, int cols, int bits, int group, const ui
 static void unpack_matrix(int m, int rows, int cols, int bits, int group, const uint8_t *src,
                           uint8_t *codes, uint16_t *scale, uint16_t *zero)
 {
+    if (bits == 16) {
+        unpack_dense(m, rows, cols, src, (uint16_t *)codes);
+        return;
+    }
     const int KT = cols / kTileK, ng = cols / group, gpt = kTileK / group, nrb = rows / kBlockRows;
     for (int rb = 0; rb < rows / kTileRows; ++rb)
         for (int kt = 0; kt < KT; ++kt) {
@@ -180,7 +232,7 @@ int mc_pack_experts_host(const mc_shape *shape, const int8_t *bits_host,
         return set_error(MC_ERR_INVALID_ARG, "packed buffer has %zu bytes, needs %llu", packed_bytes,
                          (unsigned long long)total);
     for (int i = 0; i < 3 * shape->E; ++i)
-        if (!codes_host[i] || !scale_host[i] || !zero_host[i])
+        if (!codes_host[i] || (bits_host[i / 3] != 16 && (!scale_host[i] || !zero_host[i])))
             return set_error(MC_ERR_INVALID_ARG, "NULL array for expert %d matrix %d", i / 3, i % 3);
     uint8_t *base = (uint8_t *)packed_host;
     memset(base, 0, kHeaderBytes);

@@ -104,7 +104,12 @@ def gaussian_bf16(seed, stream, shape, std=1.0):
 
 
 def expert_matrix(seed, e, m, rows, cols, group, bits, zero_mode="integer"):
-    """Codes, fp16 scale, fp16 zero for matrix m (0=w1, 1=w3, 2=w2) of expert e."""
+    """Codes, fp16 scale, fp16 zero for matrix m (0=w1, 1=w3, 2=w2) of expert e;
+    for bits = 16 (the unquantised fp16 baseline) the fp16 weights ~ N(0, 0.02)
+    and no scale / zero."""
+    if bits == 16:
+        w = (_rng(seed, 3000 + e, m).standard_normal((rows, cols), dtype=np.float32) * np.float32(0.02))
+        return w.astype(np.float16), None, None
     r = _rng(seed, 1000 + e, m)
     n = rows * cols
     raw = np.frombuffer(r.bytes(n), dtype=np.uint8)
@@ -281,6 +286,12 @@ def config_stack(T=32, layers=32, seed=1239, bits_total=20, protect_frac=0.10, H
     L.protect = importance_protect(L.x, protect_frac, seed)
     gates = [gaussian_bf16(seed, (6, l), (E, H), gate_std) for l in range(layers)]
     return L, gates
+
+
+def config_decode_fp16(T=16, seed=1236):
+    """The decode layer of config_decode with every expert unquantised (fp16
+    weights, bits = 16): the baseline PMQ is compared with (Tab. 3's fp16)."""
+    return make_layer(T, MIXTRAL_H, MIXTRAL_F, MIXTRAL_E, 128, [16] * MIXTRAL_E, seed)
 
 
 def config_decode_22b(T=16, seed=1241, bits_total=20):

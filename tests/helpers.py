@@ -22,8 +22,11 @@ def flat(L, attr):
 
 
 def oracle_mats(L):
-    return [[oracle.QMat(*L.mat_shape(m), L.group, int(L.bits[e]), L.codes[e][m], L.scale[e][m], L.zero[e][m])
-             for m in range(3)] for e in range(L.E)]
+    def one(e, m):
+        if int(L.bits[e]) == 16:  # unquantised fp16 expert
+            return oracle.QMat(*L.mat_shape(m), L.group, 16, dense=np.asarray(L.codes[e][m], np.float32))
+        return oracle.QMat(*L.mat_shape(m), L.group, int(L.bits[e]), L.codes[e][m], L.scale[e][m], L.zero[e][m])
+    return [[one(e, m) for m in range(3)] for e in range(L.E)]
 
 
 def to_dev(L):

@@ -174,3 +174,29 @@ def test_odp_threshold_host_matches_oracle():
         assert mc.odp_threshold(w, mask, q) == pytest.approx(oracle.odp_threshold(w, mask, q), rel=1e-6)
     with pytest.raises(mc.MCError):
         mc.odp_threshold(w, np.ones(200, np.uint8), 0.5)
+
+
+def test_fp16_expert_pack_round_trip_host():
+    """16-bit experts: host pack then host unpack returns the fp16 weights; the
+    tile bytes follow the documented lane / pair order (pure host code)."""
+    import paper_2410_06270_gb300 as mc
+    E, H, F = 2, 256, 384
+    shape = mc.Shape(E, H, F, 128)
+    rng = np.random.default_rng(71)
+    mats = [rng.standard_normal((F, H) if m < 2 else (H, F)).astype(np.float16) for e in range(E) for m in range(3)]
+    packed = mc.pack_experts_host(shape, [16] * E, mats, [None] * (3 * E), [None] * (3 * E))
+    # header, then per expert the W1|W3 region and the W2 region, each 256-byte aligned
+    assert packed.nbytes == 4096 + sum(2 * F * H * 2 + H * F * 2 for e in range(E))
+    for e in range(E):
+        for m in range(3):
+            rows, cols = (F, H) if m < 2 else (H, F)
+            out = np.empty((rows, cols), np.uint16)
+            rc = mc.load().mc_unpack_experts_host(packed.ctypes.data, packed.nbytes, e, m, out.ctypes.data, None, None)
+            assert rc == 0
+            np.testing.assert_array_equal(out.view(np.float16), mats[3 * e + m])
+    # first tile of expert 0's W1: lane 5 (g8 = 1, t = 1), pair j = 6 (k-step 1, rho 2)
+    w1 = mats[0]
+    tile = packed[4096:4096 + 4096].view(np.uint16)
+    row, col = 1, 64 * 0 + 16 * 1 + 4 * 1 + 2 * 1
+    assert tile[5 * 64 + 2 * 6] == w1[row, col].view(np.uint16)
+    assert tile[5 * 64 + 2 * 6 + 1] == w1[row, col + 1].view(np.uint16)

@@ -367,3 +367,37 @@ def test_forward_both_expert_paths(mc, path, group):
     L = synth.make_layer(20, 384, 512, 8, group, [3, 2, 1, 3, 2, 2, 1, 3], 95 + group, gate_std=0.1, mu=0.4,
                          protect_frac=0.2, zero_mode="fractional")
     _forward_and_check(mc, L, path=path)
+
+
+# ------------------------------------------------- unquantised experts (N1) --
+
+@pytest.mark.parametrize("T", [5, 40])
+def test_forward_fp16_experts(mc, T):
+    """Every expert unquantised (bits 16: fp16 weights, no scale / zero), the
+    baseline of the mixed-bit layer: routing bit-exact, outputs against the
+    oracle's dense experts; T = 40 has 9..16-pair chunks; W2 with an odd number
+    of row blocks (H = 384)."""
+    L = synth.make_layer(T, 384, 512, 8, 128, [16] * 8, 86, gate_std=0.1, mu=0.3, protect_frac=0.2)
+    _forward_and_check(mc, L)
+
+
+def test_forward_fp16_experts_mixtral(mc):
+    """The Mixtral-8x7b decode layer with fp16 experts (the bench's baseline
+    workload), sampled tokens."""
+    _forward_and_check(mc, synth.config_decode_fp16(T=16), tokens=[0, 8, 15])
+
+
+def test_fp16_experts_refuse_other_paths_and_mixing(mc):
+    L = synth.make_layer(8, 256, 256, 8, 128, [16] * 8, 87, gate_std=0.1)
+    shape, packed = _pack(mc, L)
+    x, g, p = to_dev(L)
+    old = mc.set_path(3)
+    try:
+        with pytest.raises(mc.MCError) as ei:
+            mc.moe_forward(x, g, shape, L.bits, packed)
+        assert ei.value.code == mc.ERR_UNSUPPORTED
+    finally:
+        mc.set_path(old)
+    with pytest.raises(mc.MCError) as ei:
+        mc.packed_size(shape, [16] * 7 + [3])
+    assert ei.value.code == mc.ERR_UNSUPPORTED
