@@ -200,3 +200,10 @@ def test_fp16_expert_pack_round_trip_host():
     row, col = 1, 64 * 0 + 16 * 1 + 4 * 1 + 2 * 1
     assert tile[5 * 64 + 2 * 6] == w1[row, col].view(np.uint16)
     assert tile[5 * 64 + 2 * 6 + 1] == w1[row, col + 1].view(np.uint16)
+
+
+def test_fp16_experts_cannot_mix_with_quantised():
+    import paper_2410_06270_gb300 as mc
+    with pytest.raises(mc.MCError) as ei:
+        mc.packed_size(mc.Shape(8, 256, 256, 128), [16] * 7 + [3])
+    assert "cannot be mixed" in str(ei.value)
