@@ -248,6 +248,29 @@ int mc_token_importance(const void *t, const float *attn, int L, int H, int nh, 
  * fp32 [T, 2] as written by mc_route.  MC_ERR_INVALID_ARG when no token qualifies. */
 int mc_odp_threshold_host(const float *w_host, const uint8_t *mask_host, int T, double q, float *mu_out);
 
+/* ------------------------------------------------------------------------ *
+ * PMQ bit allocation (Sec. 2.2), host code run once per layer before
+ * quantisation.
+ * Expert significance from a calibration run's routing (Sec. 2.2.1): host arrays
+ * idx int32 [T, 2], w fp32 [T, 2], pruned uint8 [T] (may be NULL) as written by
+ * mc_route; phi[e] = n_e / N (activations of expert e per calibration token) and
+ * wact[e] = (sum of its routing weights) / N, N = T; a pruned secondary or a
+ * dropped token is not an activation.
+ * ------------------------------------------------------------------------ */
+int mc_expert_significance_host(const int32_t *idx, const float *w, const uint8_t *pruned, int T, int E,
+                                double *phi, double *wact);
+
+/* Eq. 4, solved exactly over all 3^E assignments: bits_out[i] in {1, 2, 3}
+ * minimising sum_i phi_i^alpha * wact_i^beta * eps[i][bits_i - 1]^gamma subject
+ * to sum_i bits_i = bits_total (n * k of Eq. 4), at least one 3-bit and one 2-bit
+ * expert.  eps [E][3]: the F-norm of the layer output error with only expert i
+ * quantised to 1, 2, 3 bits (Sec. 2.2.2), measured by the caller.  Ties go to
+ * the assignment met first when expert 0's width varies fastest.  E <= 16;
+ * MC_ERR_INVALID_ARG for an infeasible budget or a negative / non-finite input.
+ * objective_out (may be NULL) receives the minimum. */
+int mc_pmq_allocate(const double *phi, const double *wact, const double *eps, int E, int bits_total, double alpha,
+                    double beta, double gamma, int8_t *bits_out, double *objective_out);
+
 /* Choose the expert path of mc_moe_forward: 0 = automatic (the GEMV below 512
  * kept-or-not pairs, 2T < 512, else the GEMM), 1 = the mma.sync grouped GEMV
  * (decode), 2 = the tcgen05 grouped GEMV with chunks of 16 pairs, 3 = the

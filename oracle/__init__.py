@@ -18,6 +18,8 @@ function states the passage of the paper it follows:
 * ``token_importance`` / ``select_top`` -- Sec. 2.3.2 Eq. 6 and the protect mask
   of the most important tokens; ``odp_threshold`` -- the Eq. 5 threshold as a
   quantile (the median in Sec. 2.3.1) of w1/w0 over calibration tokens.
+* ``expert_significance`` / ``pmq_allocate`` -- Sec. 2.2.1 (phi, w) and the
+  Eq. 4 integer program by brute force.
 * ``stack``                     -- pre-norm residual layers h <- h + MoE(RMSNorm(h)),
   each result rounded to bf16 where the stacked workload stores bf16.
 
@@ -25,6 +27,8 @@ Parity status: every function is pinned by ``tests/test_oracle_pins.py`` (closed
 forms, library routines, brute force and invariants); none is "parity unpinned".
 """
 from __future__ import annotations
+
+import itertools
 
 import ctypes
 import os
@@ -287,3 +291,39 @@ def odp_threshold(w, mask=None, q: float = 0.5) -> float:
     lo = int(np.floor(pos))
     hi = min(lo + 1, len(r) - 1)
     return float(r[lo] + (pos - lo) * (r[hi] - r[lo]))
+
+
+def expert_significance(idx, w, pruned, E: int):
+    """Sec. 2.2.1: phi_i = n_i / N (activations of expert i per calibration token)
+    and w_i = (sum of its routing weights) / N, N = the number of tokens; a pruned
+    secondary (pruned 1) or a dropped token (pruned 2) is not an activation."""
+    idx = np.asarray(idx)
+    w = np.asarray(w, np.float64)
+    T = idx.shape[0]
+    pr = np.zeros(T, np.uint8) if pruned is None else np.asarray(pruned)
+    phi, wact = np.zeros(E), np.zeros(E)
+    for t in range(T):
+        for s in range(2):
+            if (s == 1 and pr[t]) or pr[t] == 2:
+                continue
+            phi[idx[t, s]] += 1
+            wact[idx[t, s]] += w[t, s]
+    return phi / T, wact / T
+
+
+def pmq_allocate(phi, wact, eps, bits_total: int, alpha=1.0, beta=1.0, gamma=2.0):
+    """Eq. 4 (Sec. 2.2.2) by brute force: every assignment x of {1, 2, 3} bits with
+    sum = bits_total, at least one 3-bit and one 2-bit expert, minimising
+    sum_i phi_i^alpha w_i^beta (eps_{i, x_i})^gamma.  Ties: the assignment met
+    first when expert 0's width varies fastest.  Returns (bits, objective) or None
+    when no assignment is feasible."""
+    E = len(phi)
+    best = None
+    for combo in itertools.product((1, 2, 3), repeat=E):
+        b = combo[::-1]  # expert 0 varies fastest
+        if sum(b) != bits_total or 3 not in b or 2 not in b:
+            continue
+        obj = sum(phi[i] ** alpha * wact[i] ** beta * float(eps[i][b[i] - 1]) ** gamma for i in range(E))
+        if best is None or obj < best[1]:
+            best = (np.array(b, np.int8), obj)
+    return best

@@ -74,6 +74,8 @@ def load():
         "mc_token_importance_workspace_size": (Z, [I]),
         "mc_token_importance": (I, [P, P, I, I, I, F32, P, P, P, Z, P]),
         "mc_odp_threshold_host": (I, [P, P, I, ctypes.c_double, P]),
+        "mc_expert_significance_host": (I, [P, P, P, I, I, P, P]),
+        "mc_pmq_allocate": (I, [P, P, P, I, I, ctypes.c_double, ctypes.c_double, ctypes.c_double, P, P]),
         "mc_profile_enable": (I, [I]),
         "mc_profile_select": (ctypes.c_uint, [ctypes.c_uint]),
         "mc_profile_read": (I, [P, P, I]),
@@ -389,6 +391,30 @@ def odp_threshold(w, mask=None, q: float = 0.5) -> float:
     _check(load().mc_odp_threshold_host(wh.ctypes.data, None if mh is None else mh.ctypes.data, wh.shape[0],
                                         float(q), ctypes.byref(mu)))
     return float(mu.value)
+
+
+def expert_significance(idx, w, pruned, E: int):
+    """Sec. 2.2.1: (phi, wact) per expert from routing outputs (host copies taken)."""
+    i = np.ascontiguousarray(_host(idx), dtype=np.int32)
+    ww = np.ascontiguousarray(_host(w), dtype=np.float32)
+    p = None if pruned is None else np.ascontiguousarray(_host(pruned), dtype=np.uint8)
+    phi, wact = np.empty(E), np.empty(E)
+    _check(load().mc_expert_significance_host(i.ctypes.data, ww.ctypes.data, None if p is None else p.ctypes.data,
+                                              i.shape[0], E, phi.ctypes.data, wact.ctypes.data))
+    return phi, wact
+
+
+def pmq_allocate(phi, wact, eps, bits_total: int, alpha: float = 1.0, beta: float = 1.0, gamma: float = 2.0):
+    """Eq. 4 bit allocation (exact).  eps [E, 3].  Returns (bits int8 [E], objective)."""
+    phi = np.ascontiguousarray(phi, dtype=np.float64)
+    wact = np.ascontiguousarray(wact, dtype=np.float64)
+    eps = np.ascontiguousarray(eps, dtype=np.float64)
+    E = phi.shape[0]
+    bits = np.empty(E, np.int8)
+    obj = ctypes.c_double()
+    _check(load().mc_pmq_allocate(phi.ctypes.data, wact.ctypes.data, eps.ctypes.data, E, int(bits_total),
+                                  float(alpha), float(beta), float(gamma), bits.ctypes.data, ctypes.byref(obj)))
+    return bits, float(obj.value)
 
 
 def _host(a):

@@ -207,3 +207,31 @@ def test_fp16_experts_cannot_mix_with_quantised():
     with pytest.raises(mc.MCError) as ei:
         mc.packed_size(mc.Shape(8, 256, 256, 128), [16] * 7 + [3])
     assert "cannot be mixed" in str(ei.value)
+
+
+def test_pmq_allocation_matches_oracle():
+    """mc_expert_significance_host and mc_pmq_allocate (host code) against the
+    oracle's counting and brute-force Eq. 4."""
+    import oracle
+    import paper_2410_06270_gb300 as mc
+    rng = np.random.default_rng(72)
+    T, E = 300, 8
+    idx = np.stack([rng.integers(0, E, T), rng.integers(0, E, T)], axis=1).astype(np.int32)
+    idx[:, 1] = (idx[:, 0] + 1 + rng.integers(0, E - 1, T)) % E
+    w0 = rng.uniform(0.5, 1.0, T)
+    w = np.stack([w0, 1 - w0], axis=1).astype(np.float32)
+    pr = (rng.random(T) < 0.15).astype(np.uint8)
+    pr[::37] = 2
+    phi, wact = mc.expert_significance(idx, w, pr, E)
+    ophi, owact = oracle.expert_significance(idx, w, pr, E)
+    np.testing.assert_allclose(phi, ophi, rtol=1e-12)
+    np.testing.assert_allclose(wact, owact, rtol=1e-6)
+    for total, gamma in ((20, 2.0), (16, 2.0), (13, 1.0)):
+        eps = np.sort(rng.uniform(0.1, 5.0, (E, 3)), axis=1)[:, ::-1]
+        bits, obj = mc.pmq_allocate(phi, wact, eps, total, 1.0, 1.0, gamma)
+        obits, oobj = oracle.pmq_allocate(phi, wact, eps, total, 1.0, 1.0, gamma)
+        np.testing.assert_array_equal(bits, obits)
+        assert obj == pytest.approx(oobj, rel=1e-12)
+        assert bits.sum() == total and (bits == 3).any() and (bits == 2).any()
+    with pytest.raises(mc.MCError):
+        mc.pmq_allocate(phi, wact, eps, 25)

@@ -479,3 +479,63 @@ def test_odp_threshold_is_quantile_of_prunable_ratios():
     mu = oracle.odp_threshold(w, None, 0.15)
     _, _, pr = oracle.route(L.x_f32(), L.gate_f32(), mu=mu)
     assert abs(pr.mean() - 0.15) <= 1.0 / 101 + 1e-12
+
+
+# ---------------------------------------------------- PMQ allocation (N3) ---
+
+def test_pmq_tiny_by_hand():
+    """E = 3, budget 6: only the 6 permutations of (1, 2, 3) are feasible (2,2,2
+    has no 3-bit expert); the objective of each written out by hand."""
+    phi, w = [0.5, 1.0, 0.5], [0.2, 0.6, 0.2]
+    eps = [[4.0, 2.0, 1.0], [3.0, 2.0, 0.5], [5.0, 1.0, 0.2]]
+    best, arg = None, None
+    for b in itertools.permutations((1, 2, 3)):
+        obj = sum(phi[i] * w[i] * eps[i][b[i] - 1] ** 2 for i in range(3))
+        if best is None or obj < best - 1e-15:
+            best, arg = obj, b
+    bits, obj = oracle.pmq_allocate(phi, w, eps, 6)
+    assert tuple(bits) == arg and obj == pytest.approx(best, rel=1e-12)
+
+
+def test_pmq_invariances_and_exchange():
+    """Scaling every eps by c > 0 keeps the allocation; with alpha = beta = 0 only
+    eps matters; of two experts with the same eps row (falling with the bit
+    width) the more significant one never gets fewer bits."""
+    rng = np.random.default_rng(46)
+    E = 6
+    phi, w = rng.uniform(0.1, 0.6, E), rng.uniform(0.05, 0.3, E)
+    eps = np.sort(rng.uniform(0.1, 5.0, (E, 3)), axis=1)[:, ::-1]  # 1 bit worst
+    b0, _ = oracle.pmq_allocate(phi, w, eps, 13)
+    b1, _ = oracle.pmq_allocate(phi, w, 3.7 * eps, 13)
+    np.testing.assert_array_equal(b0, b1)
+    b2, _ = oracle.pmq_allocate(np.ones(E), np.ones(E), eps, 13, alpha=0.0, beta=0.0)
+    b3, _ = oracle.pmq_allocate(phi, w, eps, 13, alpha=0.0, beta=0.0)
+    np.testing.assert_array_equal(b2, b3)
+    eps2 = eps.copy()
+    eps2[1] = eps2[0]
+    phi2 = phi.copy()
+    phi2[0], phi2[1] = 0.9, 0.2  # expert 0 more significant than expert 1
+    for total in (10, 12, 14):
+        b, _ = oracle.pmq_allocate(phi2, w * 0 + 0.2, eps2, total)
+        assert b[0] >= b[1]
+
+
+def test_pmq_infeasible_budget():
+    assert oracle.pmq_allocate([1, 1], [1, 1], [[1, 1, 1]] * 2, 6) is None  # (3,3) has no 2-bit expert
+    assert oracle.pmq_allocate([1, 1, 1], [1, 1, 1], [[1, 1, 1]] * 3, 10) is None  # > 3 bits each
+
+
+def test_expert_significance_sums():
+    """phi sums to the activations per token (2 - pruned secondaries - 2 x dropped,
+    over T) and w to the non-dropped share (each kept token's weights sum to 1)."""
+    L = _rand_layer(T=90, E=8, bits=(1, 2, 3, 2, 1, 2, 3, 3), experts=False, gate_std=0.5, protect_frac=0.1)
+    mask = L.protect.copy()
+    mask[[3, 30, 60]] = 2
+    idx, w, pr = oracle.route(L.x_f32(), L.gate_f32(), 0.5, mask)
+    phi, wact = oracle.expert_significance(idx, w, pr, 8)
+    n_pruned, n_drop = int((pr == 1).sum()), int((pr == 2).sum())
+    assert phi.sum() == pytest.approx((2 * 90 - n_pruned - 2 * n_drop) / 90, rel=1e-12)
+    assert wact.sum() == pytest.approx((90 - n_drop) / 90, rel=1e-6)
+    for e in range(8):  # brute force count
+        n = sum(1 for t in range(90) for s in range(2) if idx[t, s] == e and not ((s and pr[t]) or pr[t] == 2))
+        assert phi[e] == pytest.approx(n / 90, rel=1e-12)
