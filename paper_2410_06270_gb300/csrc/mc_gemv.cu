@@ -463,18 +463,26 @@ __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, 
         const uint8_t *base = R.base + (size_t)slot * R.SB;
         const int kc = sh->slot_kc[slot];
         const uint8_t *v0 = base + R.vec_off0, *v1 = v0 + KPS * R.VB;
+        auto step = [&](int kk) {
+            const uint8_t *st = base + kk * step_bytes;
+            const uint8_t *t[kTPW];
 #pragma unroll
-        for (int kk = 0; kk < KPS; ++kk)
-            if (kk < kc) {
-                const uint8_t *st = base + kk * step_bytes;
-                const uint8_t *t[kTPW];
+            for (int u = 0; u < kTPW; ++u) t[u] = st + off[u];
+            if constexpr (BITS == 16)
+                step_dense<NT, kTPW>(t, v0 + kk * R.VB, v1 + kk * R.VB, lane, y);
+            else
+                step_tiles<NT, BITS, GPT, kTPW>(t, v0 + kk * R.VB, v1 + kk * R.VB, lane, y);
+        };
+        if (GPT == 1 && kc == KPS) {
+            // a full stage as straight-line code, so consecutive steps' loads and
+            // decodes overlap (one group per tile keeps it within the registers)
 #pragma unroll
-                for (int u = 0; u < kTPW; ++u) t[u] = st + off[u];
-                if constexpr (BITS == 16)
-                    step_dense<NT, kTPW>(t, v0 + kk * R.VB, v1 + kk * R.VB, lane, y);
-                else
-                    step_tiles<NT, BITS, GPT, kTPW>(t, v0 + kk * R.VB, v1 + kk * R.VB, lane, y);
-            }
+            for (int kk = 0; kk < KPS; ++kk) step(kk);
+        } else {
+#pragma unroll
+            for (int kk = 0; kk < KPS; ++kk)
+                if (kk < kc) step(kk);
+        }
         __syncwarp();
         if (lane == 0) mbar_arrive(&R.empty[slot]);
         if (++slot == R.S) {
