@@ -196,8 +196,10 @@ __global__ void __launch_bounds__(256) frag_x_kernel(ExpertParams p)
     __shared__ uint2 afr[8 * 32];
     const int k = blockIdx.x, kt = blockIdx.y, KT = p.H / kTileK;
     build_tab_afrag(afr, threadIdx.x, 256);
-    pdl_trigger();
+    // trigger only after the routing launch has completed: the expert kernel that
+    // follows reads the routing outputs before its own wait
     pdl_wait();
+    pdl_trigger();
     // both loads in flight together (entry k < max_chunks exists even when unused)
     const int nchunks = *p.nchunks;
     const ChunkInfo ci = p.chunks[k];
@@ -583,27 +585,47 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
         fence_mbar_init();
     }
     if (W13) build_tab_afrag(afr, threadIdx.x, kGemvThreads);
-    pdl_wait();
     __syncthreads();
+
+    // The producer's first claim, the header check and an L2 prefetch of its first
+    // item's weights read only the routing outputs and the packed weights: the
+    // routing launch completed before the launch before this one triggered this
+    // kernel, so this overlaps that launch's end.  Everything after the wait may
+    // read what that launch wrote.
+    const bool producer = warp == kCW && lane == 0 && !(p.debug & kDebugNoProducer);
+    int *counter = &p.counters[W13 ? 0 : 1];
+    int item = 0, total = 0;
+    bool ok = true;
+    ChunkInfo ci{};
+    if (producer) {
+        const int nchunks = *p.nchunks;
+        item = atomicAdd(counter, 1);
+        ok = header_ok(p);
+        total = nchunks * U;
+        if (ok && item < total) {
+            ci = p.chunks[item / U];
+            const Item I = decode_item<W13>(p, item, U, ci);
+            const int STB = supertile_bytes(I.ci.bits, group);
+            const int pw = W13 ? 2 : w2_pair_width(I.blkA >> 1, nrb);
+            const uint8_t *wsrc =
+                p.packed + p.mat_off[I.ci.e][W13 ? 0 : 2] + supertile_off(W13 ? 0 : 2, I.blkA, I.kt0, KTm, nrb, STB);
+            const int nk = min(I.nkt, S * KPS);
+            for (int i = 0; i < nk; i += KPS)
+                bulk_prefetch_l2(wsrc + (size_t)i * pw * STB, (uint32_t)(min(KPS, nk - i) * pw * STB));
+        }
+    }
+    pdl_wait();
 
     if (warp == kCW) {
         // ---------------------------------------------------------- producer --
-        if (lane == 0 && !(p.debug & kDebugNoProducer)) {
+        if (producer) {
             const uint64_t pol = policy_evict_first();
-            int *counter = &p.counters[W13 ? 0 : 1];
-            // the item count, the first claim and the header check: one round trip
-            const int nchunks = *p.nchunks;
-            int item = atomicAdd(counter, 1);
-            bool ok = header_ok(p);
-            const int total = nchunks * U;
             int it = 0, pslot = 0;
             uint32_t pphase = 0;  // phase of the ring round being filled
             if (!ok) {
                 set_status(p.status, MC_ERR_BAD_PACK);
                 sh->abort = 1;
             }
-            ChunkInfo ci;
-            if (ok && item < total) ci = p.chunks[item / U];
             if (item >= total) pdl_trigger();
             while (ok && item < total) {
                 // the next item is claimed with this item's second-to-last stage and
