@@ -150,14 +150,22 @@ def _algorithmic_bytes(shape, bits, touched, T, H):
     return w13 + w2 + other, w13
 
 
+def _oracle_mats(oracle, L):
+    """The oracle's expert matrices of a synthetic layer (16-bit experts: dense fp16 weights)."""
+    def one(e, m):
+        if int(L.bits[e]) == 16:
+            return oracle.QMat(*L.mat_shape(m), L.group, 16, dense=np.asarray(L.codes[e][m], np.float32))
+        return oracle.QMat(*L.mat_shape(m), L.group, int(L.bits[e]), L.codes[e][m], L.scale[e][m], L.zero[e][m])
+    return [[one(e, m) for m in range(3)] for e in range(L.E)]
+
+
 def cpu_baseline(L, budget_s=12.0, threads=None):
     """Time the oracle, as it stands, on a bounded sample of the workload's tokens
     (one token per host thread)."""
     import concurrent.futures as cf
 
     import oracle
-    mats = [[oracle.QMat(*L.mat_shape(m), L.group, int(L.bits[e]), L.codes[e][m], L.scale[e][m], L.zero[e][m])
-             for m in range(3)] for e in range(L.E)]
+    mats = _oracle_mats(oracle, L)
     xf, gf = L.x_f32(), L.gate_f32()
     t_mask = 0.0
     if name_has_mask(L):  # the step's Eq. 6 mask, for all tokens (charged pro rata below)
@@ -187,8 +195,7 @@ def cpu_baseline_stack(L, gates, mus, budget_s=12.0, threads=None):
     import concurrent.futures as cf
 
     import oracle
-    mats = [[oracle.QMat(*L.mat_shape(m), L.group, int(L.bits[e]), L.codes[e][m], L.scale[e][m], L.zero[e][m])
-             for m in range(3)] for e in range(L.E)]
+    mats = _oracle_mats(oracle, L)
     gf = [synth.bf16_bits_to_f32(g) for g in gates]
     xf = L.x_f32()
     run = lambda t: oracle.stack(xf[t:t + 1], gf, mats, mus, L.protect[t:t + 1])
@@ -211,8 +218,7 @@ def _stack_mus_oracle(L, gates):
     """Per-layer thresholds from the oracle's own trajectory at mu = 0 (the
     reference arm's counterpart of the calibration in run_stack)."""
     import oracle
-    mats = [[oracle.QMat(*L.mat_shape(m), L.group, int(L.bits[e]), L.codes[e][m], L.scale[e][m], L.zero[e][m])
-             for m in range(3)] for e in range(L.E)]
+    mats = _oracle_mats(oracle, L)
     gf = [synth.bf16_bits_to_f32(g) for g in gates]
     xf = L.x_f32()
     mus = []
