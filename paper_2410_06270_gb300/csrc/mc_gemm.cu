@@ -218,6 +218,14 @@ __device__ __forceinline__ void tmem_st_16x256_x8(uint32_t taddr, const uint32_t
 }
 
 template <int GPT>
+__device__ __forceinline__ void convert_regs(const uint8_t *tile, int bits, int lane, uint32_t (&v)[32])
+{
+    if (bits == 1) convert_tile<1, GPT>(tile, lane, v);
+    else if (bits == 2) convert_tile<2, GPT>(tile, lane, v);
+    else convert_tile<3, GPT>(tile, lane, v);
+}
+
+template <int GPT>
 __device__ __forceinline__ void convert_store(const uint8_t *tile, int bits, int lane, uint32_t taddr)
 {
     uint32_t v[32];
@@ -396,13 +404,18 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
             if (!g_wait(&sh->full[slot], (it / kGSlots) & 1, p, sh)) break;
             const GStage st = sh->stage[slot];
             if (st.item < 0) break;
-            if (it >= 2 && !g_wait(&sh->aempty[b], ((it >> 1) - 1) & 1, p, sh)) break;
-            tc_fence_after();
             const int bits = st.ci.bits, STB = supertile_bytes(bits, group), TB = tile_bytes(bits, group);
             const int nstream = W13 ? 2 : w2_pair_width(st.u, nrb);
             const uint8_t *w = ring + (size_t)slot * kGStage + kImgBytes;
             const uint32_t abuf = tbase + 256u + 128u * (uint32_t)b;
-            for (int x = 0; x < nstream; ++x) {
+            // the first stream's tile is dequantised before the A buffer is free (the
+            // MMAs of two stages back may still read it); only its store waits
+            uint32_t v0[32];
+            convert_regs<GPT>(w + (2 * q + u2) * TB, bits, lane, v0);
+            if (it >= 2 && !g_wait(&sh->aempty[b], ((it >> 1) - 1) & 1, p, sh)) break;
+            tc_fence_after();
+            tmem_st_16x256_x8(abuf + ((uint32_t)(32 * q + 16 * u2) << 16), v0);
+            for (int x = 1; x < nstream; ++x) {
                 const uint8_t *tile = w + x * STB + (2 * q + u2) * TB;
                 const uint32_t taddr = abuf + 64u * (uint32_t)x + ((uint32_t)(32 * q + 16 * u2) << 16);
                 convert_store<GPT>(tile, bits, lane, taddr);
