@@ -230,6 +230,88 @@ __global__ void __launch_bounds__(1024) permute_kernel(PermuteParams p)
     permute_block(p);
 }
 
+// Placement of at most 128 pairs (T <= 64) by one warp, with no block barrier.
+// Pair i = 32k + lane sits in slice k.  Lane e (< E) keeps, per slice, the ballot
+// of the lanes whose pair goes to expert e; their population counts give the
+// expert's count, a warp scan over the lanes gives the offsets, and a pair's
+// place is its expert's start of the slice plus the lanes of that expert below
+// it in the slice.  Same result as permute_block.
+__device__ __forceinline__ void permute_warp(const PermuteParams &p)
+{
+    const unsigned full = 0xffffffffu, lt = (1u << (threadIdx.x & 31)) - 1;
+    const int lane = threadIdx.x & 31, NP = 2 * p.T, nk = (NP + 31) / 32, E = p.E;
+    int key[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int i = 32 * k + lane;
+        key[k] = -1;
+        if (i < NP) {
+            const uint8_t pr = __ldcg(p.pruned + (i >> 1));
+            const int e = __ldcg(p.idx + i);
+            key[k] = ((i & 1) && pr) || pr == 2 ? -1 : e;
+        }
+    }
+    unsigned mine[4] = {0u, 0u, 0u, 0u};  // lane e: ballot of expert e per slice
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+        if (k < nk)
+            for (int e = 0; e < E; ++e) {
+                const unsigned b = __ballot_sync(full, key[k] == e);
+                if (lane == e) mine[k] = b;
+            }
+    int cnt = 0, bits = 0;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) cnt += __popc(mine[k]);
+#pragma unroll
+    for (int f = 0; f < kMaxE; ++f)
+        if (f == lane) bits = p.bits[f];
+    int incl = cnt;  // inclusive scan of the counts over the lanes (experts)
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+        const int v = __shfl_up_sync(full, incl, d);
+        if (lane >= d) incl += v;
+    }
+    const int off = incl - cnt;
+    // the index of expert `lane`'s first work chunk in the order the expert
+    // kernels take them (more bits first, then by expert), and the chunk total
+    const int nch = (cnt + p.chunk - 1) / p.chunk;
+    int k0 = 0, nchunks = 0;
+    for (int f = 0; f < E; ++f) {
+        const int nf = __shfl_sync(full, nch, f), bf = __shfl_sync(full, bits, f);
+        nchunks += nf;
+        if (bf > bits || (bf == bits && f < lane)) k0 += nf;
+    }
+    if (lane < E) {
+        p.offsets[lane] = off;
+        if (lane == E - 1) p.offsets[E] = incl;
+        if (p.chunks)
+            for (int c = 0, k = k0; c < cnt; c += p.chunk, ++k) {
+                ChunkInfo ci;
+                ci.e = lane;
+                ci.pair_base = off + c;
+                ci.nv = min(p.chunk, cnt - c);
+                ci.bits = bits;
+                p.chunks[k] = ci;
+            }
+    }
+    if (lane == 0 && p.chunks) {
+        *p.nchunks = nchunks;
+        for (int i = 0; i < 4; ++i) p.counters[i] = 0;
+    }
+    int start = off;  // lane e: where expert e's pairs of the current slice begin
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+        if (k < nk) {
+            const int e = key[k], src = e >= 0 ? e : 0;
+            const int s0 = __shfl_sync(full, start, src);
+            const unsigned b = __shfl_sync(full, mine[k], src);
+            const int i = 32 * k + lane, pos = e >= 0 ? s0 + __popc(b & lt) : -1;
+            if (e >= 0) p.perm[pos] = i;
+            if (p.inv && i < NP) p.inv[i] = pos;
+            start += __popc(mine[k]);
+        }
+}
+
 // Routing of token blockIdx.x, then the last CTA to finish (counted on *done,
 // which it resets) places the pairs: one launch instead of two for small T.
 __global__ void __launch_bounds__(kRouteThreads) route_permute_kernel(RouteParams rp, PermuteParams pp, int32_t *done)
@@ -247,8 +329,8 @@ __global__ void __launch_bounds__(kRouteThreads) route_permute_kernel(RouteParam
         last = prev == (int)gridDim.x - 1;
     }
     __syncthreads();
-    if (!last) return;
-    permute_block(pp);
+    if (!last || threadIdx.x >= 32) return;
+    permute_warp(pp);  // T <= 64 here
     if (threadIdx.x == 0) *done = 0;
 }
 
