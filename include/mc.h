@@ -282,7 +282,11 @@ int mc_set_path(int path);
  * copies, so every consumer wait reaches its bound and the status word reports
  * MC_ERR_TIMEOUT (no fault, no hang); bit 1 launches every kernel without
  * programmatic dependent launch (by default each kernel's launch overlaps the
- * end of the one before it on the stream; results are the same either way).
+ * end of the one before it on the stream; results are the same either way); bit
+ * 2 makes mc_route take the single-launch routing mc_moe_forward uses for
+ * T <= 64 (the last routing CTA places the pairs), with its arrival count in a
+ * word owned by the library, so that tests can compare that placement with the
+ * two-launch one (calls with the bit set must not overlap in time on a device).
  * `timeout_ns` (0 = keep) bounds every device wait (default 1 s).
  * Process-wide. */
 int mc_set_debug(int flags, unsigned long long timeout_ns);

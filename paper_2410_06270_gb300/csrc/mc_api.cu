@@ -191,6 +191,11 @@ int mc_route(const void *x, const void *gate_w, int T, const mc_shape *shape, fl
     pp.offsets = expert_offsets;
     pp.perm = perm;
     pp.chunk = kChunk;
+    if (g_debug.load() & kDebugRouteFused) {
+        int32_t *done = route_done_word();
+        if (!done) return set_error(MC_ERR_CUDA, "routing arrival word not found");
+        return launch_route(rp, pp, (cudaStream_t)stream, done);
+    }
     return launch_route(rp, pp, (cudaStream_t)stream);
 }
 

@@ -98,6 +98,7 @@ struct ExpertParams {
 
 constexpr int kDebugNoProducer = 1;  // the copy producer never issues: waits expire
 constexpr int kDebugNoPdl = 2;       // launch without programmatic dependent launch
+constexpr int kDebugRouteFused = 4;  // mc_route takes the single-launch routing for T <= 64
 
 constexpr int kMaxKS = 8;  // column splits of the W2 GEMV pass, at most
 
@@ -141,5 +142,6 @@ size_t img_buffer_bytes(int max_blocks, int cols);
 int max_blocks_for(int T, int E);
 int launch_combine(const CombineParams &cp, cudaStream_t st);
 int max_chunks_for(int T, int E);
+int32_t *route_done_word();  // mc_route's arrival word for the single-launch routing
 
 }  // namespace mc

@@ -334,6 +334,17 @@ __global__ void __launch_bounds__(kRouteThreads) route_permute_kernel(RouteParam
     if (threadIdx.x == 0) *done = 0;
 }
 
+// The arrival count of mc_route's single-launch routing (kDebugRouteFused): one
+// word owned by the library, zero between launches (the last CTA resets it), so
+// such calls must not overlap in time on one device.
+__device__ int32_t g_route_done;
+
+int32_t *route_done_word()
+{
+    void *p = nullptr;
+    return cudaGetSymbolAddress(&p, g_route_done) == cudaSuccess ? (int32_t *)p : nullptr;
+}
+
 int max_chunks_for(int T, int E) { return (2 * T + kChunk - 1) / kChunk + E; }
 
 int launch_route(const RouteParams &rp, const PermuteParams &pp, cudaStream_t st, int32_t *done)

@@ -90,6 +90,35 @@ def test_route_bit_exact(mc, case):
         np.testing.assert_array_equal(np.flatnonzero(out["pruned"].cpu().numpy() == 2), dropped)
 
 
+@pytest.mark.parametrize("T", [1, 5, 17, 32, 33, 48, 64])
+def test_single_launch_routing_places_like_the_two_launch_one(mc, T):
+    """mc_moe_forward routes T <= 64 tokens in one launch whose last CTA places
+    the pairs with one warp (ballots per 32-pair slice, a warp scan over the
+    experts); debug bit 2 sends mc_route through that launch.  Offsets and the
+    stable permutation must equal the oracle's and the two-launch placement's,
+    with ODP pruning, protected tokens and dropped tokens in the batch."""
+    L = synth.make_layer(T, 256, 128, 8, 64, [2] * 8, 90 + T, gate_std=0.15, mu=0.4, protect_frac=0.2,
+                         experts=False)
+    if T >= 5:
+        _with_drops(L, max(1, T // 10), 91 + T)
+    condition_routing(L, L.mu)
+    x, g, p = to_dev(L)
+    shape = mc.Shape(L.E, L.H, L.F, L.group)
+    two = mc.route(x, g, shape, L.mu, p)
+    mc.set_debug(4, 0)
+    try:
+        for _ in range(3):  # the arrival word is back at zero after every call
+            one = mc.route(x, g, shape, L.mu, p)
+            torch.cuda.synchronize()
+            _check_routing(mc, L, one["idx"], one["w"], one["pruned"], one["offsets"], one["perm"])
+            for k in ("idx", "w", "pruned", "offsets"):
+                assert torch.equal(one[k], two[k]), k
+            n = int(two["offsets"][-1])
+            assert torch.equal(one["perm"][:n], two["perm"][:n])
+    finally:
+        mc.set_debug(0, 1_000_000_000)
+
+
 def test_route_mu_zero_and_above_one(mc):
     L = synth.make_layer(64, 256, 128, 8, 64, [2] * 8, 36, gate_std=0.2, protect_frac=0.25, experts=False)
     condition_routing(L, 0.0)
