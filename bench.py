@@ -486,7 +486,7 @@ def run(args):
     alg_bytes, w13_bytes = _algorithmic_bytes(shape, L.bits, touched, T, L.H)
     w13_flops = 4.0 * L.H * L.F * pairs          # W1 and W3: 2 x (2 H F) per kept pair
     layer_flops = 6.0 * L.H * L.F * pairs + 2.0 * L.H * L.E * T
-    rk = "gemv_w13" if 2 * T < 512 else "gemm_w13"  # the path mc_moe_forward picks
+    rk = "gemv_w13" if 2 * T < 240 else "gemm_w13"  # the path mc_moe_forward picks (kPrefillPairs)
 
     clocks = Clocks(local)
     clocks.start()

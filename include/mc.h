@@ -271,8 +271,8 @@ int mc_expert_significance_host(const int32_t *idx, const float *w, const uint8_
 int mc_pmq_allocate(const double *phi, const double *wact, const double *eps, int E, int bits_total, double alpha,
                     double beta, double gamma, int8_t *bits_out, double *objective_out);
 
-/* Choose the expert path of mc_moe_forward: 0 = automatic (the GEMV below 512
- * kept-or-not pairs, 2T < 512, else the GEMM), 1 = the mma.sync grouped GEMV
+/* Choose the expert path of mc_moe_forward: 0 = automatic (the GEMV below 240
+ * kept-or-not pairs, 2T < 240, else the GEMM), 1 = the mma.sync grouped GEMV
  * (decode), 2 = the tcgen05 grouped GEMV with chunks of 16 pairs, 3 = the
  * tcgen05 grouped GEMM with token blocks of 128 pairs (prefill).
  * Process-wide; returns the previous value. */

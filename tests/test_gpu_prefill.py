@@ -79,8 +79,8 @@ def test_prefill_sixteen_experts(mc):
 
 
 def test_automatic_switch_agrees_with_gemv(mc):
-    """T = 256 (512 pairs) takes the GEMM automatically; the GEMV path on the
-    same inputs agrees with it and with the oracle."""
+    """T = 256 (512 pairs; the GEMM from 240 pairs) takes the GEMM automatically;
+    the GEMV path on the same inputs agrees with it and with the oracle."""
     L = synth.make_layer(256, 256, 512, 8, 64, [3, 2, 2, 1, 3, 2, 2, 3], 350, gate_std=0.1, mu=0.3,
                          protect_frac=0.1)
     auto = _run(mc, L, 0)
