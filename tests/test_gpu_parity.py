@@ -255,6 +255,31 @@ def test_forward_token_drop(mc, T):
     assert_close(got, ref, "token drop T=%d" % T)
 
 
+@pytest.mark.parametrize("T,path", [(8, 1), (8, 2), (8, 3), (130, 0)])
+def test_forward_every_token_dropped(mc, T, path):
+    """The degenerate batch: every token dropped (mask byte 2).  No pair reaches
+    an expert, every expert kernel runs with zero work items, and the output is
+    exactly zero; on the GEMV, the tensor-memory GEMV and the GEMM paths (T = 130
+    takes the GEMM automatically)."""
+    L = synth.make_layer(T, 256, 512, 8, 64, [3, 2, 2, 1, 3, 2, 2, 3], 86, gate_std=0.1, mu=0.3)
+    L.protect = np.full(T, 2, np.uint8)
+    shape, packed = _pack(mc, L)
+    x, g, p = to_dev(L)
+    prev = mc.set_path(path)
+    try:
+        y = torch.full_like(x, 7.0)
+        y, r = mc.moe_forward(x, g, shape, L.bits, packed, L.mu, p, y=y, routing=True)
+        ws = mc.alloc_workspace(shape, T)
+        y2 = mc.moe_forward(x, g, shape, L.bits, packed, L.mu, p, workspace=ws)
+        mc.check_status(ws)
+        torch.cuda.synchronize()
+    finally:
+        mc.set_path(prev)
+    assert (r["pruned"] == 2).all()
+    assert (r["w"] == 0).all()
+    assert (y.float() == 0).all() and (y2.float() == 0).all()
+
+
 @pytest.mark.parametrize("T", [16, 300])
 def test_forward_same_without_programmatic_launch(mc, T):
     """Kernels launched without programmatic dependent launch (each one starts
