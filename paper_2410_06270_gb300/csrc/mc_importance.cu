@@ -16,6 +16,9 @@
 //   pass over the float bit patterns, which order like the values for
 //   non-negative floats), then the mask: every token above that value and, among
 //   the tokens equal to it, the lowest indices until n are chosen.
+// rank_select_kernel (L <= 1024): the same mask from each token's rank, the number
+//   of tokens with a larger bit pattern or an equal one at a lower index, counted
+//   over the importances held in shared memory (one pass, no histogram rounds).
 #include <math.h>
 #include <stdlib.h>
 #include <string.h>
@@ -141,6 +144,26 @@ __global__ void __launch_bounds__(1024) select_kernel(const float *imp, int L, i
     }
 }
 
+constexpr int kRankMaxL = 1024;
+
+__global__ void __launch_bounds__(1024) rank_select_kernel(const float *imp, int L, int n, uint8_t *mask)
+{
+    __shared__ unsigned key[kRankMaxL];
+    pdl_trigger();
+    pdl_wait();
+    for (int j = threadIdx.x; j < L; j += blockDim.x) key[j] = __float_as_uint(imp[j]);
+    __syncthreads();
+    for (int j = threadIdx.x; j < L; j += blockDim.x) {
+        const unsigned kj = key[j];
+        int r = 0;
+        for (int i = 0; i < L; ++i) {
+            const unsigned ki = key[i];  // the same word for every lane: a broadcast
+            r += ki > kj || (ki == kj && i < j);
+        }
+        mask[j] = r < n ? 1 : 0;
+    }
+}
+
 __global__ void fill_kernel(uint8_t *mask, int L, uint8_t v)
 {
     pdl_trigger();
@@ -193,6 +216,8 @@ int mc_token_importance(const void *t, const float *attn, int L, int H, int nh, 
         profile_begin(kKImportance, st);
         if (n <= 0 || n >= L)
             err = launch_k(fill_kernel, dim3((L + 255) / 256), dim3(256), 0, st, mask, L, (uint8_t)(n > 0));
+        else if (L <= kRankMaxL)
+            err = launch_k(rank_select_kernel, dim3(1), dim3(1024), 0, st, (const float *)importance, L, n, mask);
         else
             err = launch_k(select_kernel, dim3(1), dim3(1024), 0, st, (const float *)importance, L, n, mask);
         profile_end(kKImportance, st);

@@ -51,7 +51,8 @@ def _run(mc, L, H, nh, frac, seed, attn=None):
 
 
 @pytest.mark.parametrize("L,H,nh,frac", [(300, 256, 4, 0.02), (300, 256, 4, 0.1), (1, 128, 2, 0.5),
-                                         (33, 64, 1, 0.0), (33, 64, 1, 1.0), (2048, 128, 8, 0.02)])
+                                         (33, 64, 1, 0.0), (33, 64, 1, 1.0), (2048, 128, 8, 0.02),
+                                         (1024, 64, 2, 0.3), (1025, 64, 2, 0.3)])
 def test_importance_and_mask(mc, L, H, nh, frac):
     t64, A, imp, mask = _run(mc, L, H, nh, frac, 500 + L + nh)
     ref, ref_mask = oracle.token_importance(t64, A.astype(np.float64), frac)
