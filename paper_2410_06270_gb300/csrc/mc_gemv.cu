@@ -12,9 +12,8 @@
 //     [vector blocks of n-tile 0][of n-tile 1]      one copy each
 //   The packed layout interleaves the two streams step by step (mc_layout.h), so
 //   a stage is a few large copies: small copies cap the streaming bandwidth well
-//   below the HBM peak.  Consumer warps own 16-row tiles: kTPW = 2 gives eight
-//   warps with tile tl of BOTH streams (the B fragments and tables are loaded
-//   once for the two), kTPW = 1 sixteen warps with one tile each.  Code
+//   below the HBM peak.  Eight consumer warps own 16-row tile tl of BOTH streams
+//   (the B fragments and tables are loaded once for the two).  Code
 //   words become fp16 mma.sync A fragments with one LOP3 per register
 //   (mc_layout.h), and every quantisation group is accumulated from
 //       acc = -(O + z X) + sum_k (off_k + q_k) x_k = sum_k (q_k - z) x_k
@@ -33,10 +32,7 @@
 
 namespace mc {
 
-#ifndef MC_GEMV_TPW
-#define MC_GEMV_TPW 2
-#endif
-constexpr int kTPW = MC_GEMV_TPW;            // 16-row tiles per consumer warp (1 or 2)
+constexpr int kTPW = 2;                     // 16-row tiles per consumer warp: tile tl of both streams
 constexpr int kCW = 16 / kTPW;              // consumer warps
 constexpr int kGemvThreads = (kCW + 1) * 32;
 constexpr int kMaxSlots = 16;
@@ -67,11 +63,10 @@ __host__ __device__ inline int slot_bytes(int group, bool dense)
     return kps * 2 * supertile_bytes(dense ? 16 : 3, group) + 2 * kps * kVecMax;
 }
 constexpr int kHsBytes = kChunk * kTileK * 2;           // h tile [16][128] fp16 (two of them)
-constexpr int kXbufBytes = kTPW == 1 ? 8 * 32 * 8 * 4 : 0;  // W3 results handed to the W1 warps
 
 __host__ __device__ inline size_t gemv_smem(int nslots, int group, bool dense)
 {
-    return kRingOff + (size_t)nslots * slot_bytes(group, dense) + 2 * kHsBytes + kXbufBytes + 8 * 32 * sizeof(uint2);
+    return kRingOff + (size_t)nslots * slot_bytes(group, dense) + 2 * kHsBytes + 8 * 32 * sizeof(uint2);
 }
 
 // Bounded wait that gives up as soon as another thread of the CTA aborted.
@@ -433,17 +428,15 @@ __device__ __forceinline__ bool consumer_sync(const ExpertParams &p, RingShared 
 // One work item for one consumer warp: all its stages, then the epilogue.  The
 // first stage's full barrier has already been waited for; the ring position
 // (slot, phase) advances by one per stage.
-//   kTPW = 2: the warp owns tile tl of both streams.
-//   kTPW = 1: the warp owns tile tl of stream x.
+//   The warp owns tile tl of both streams.
 //   W13: h = silu(W1 x) * (W3 x) for the item's rows goes to the h tile
-//        (double-buffered by item parity; with one tile per warp the W3 results
-//        pass through xbuf first), then the consumer warps together write W2's
-//        vector blocks of this 128-row block.
+//        (double-buffered by item parity), then the consumer warps together
+//        write W2's vector blocks of this 128-row block.
 //   W2:  fp32 outputs of the split.
 template <bool W13, int NT, int BITS, int GPT>
 __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, const Ring &R, const Item &I, int nrb,
-                                         int x, int tl, int lane, int &slot, uint32_t &phase, float *xbuf,
-                                         __half *hs2, int &items, int &cbar_uses)
+                                         int tl, int lane, int &slot, uint32_t &phase, __half *hs2, int &items,
+                                         int &cbar_uses)
 {
     constexpr int group = kTileK / GPT;
     constexpr int KPS = BITS == 16 ? 1 : kKPS;  // stage_steps
@@ -452,7 +445,7 @@ __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, 
     const int step_bytes = pw * STB;
     // a lone W2 block (odd row-block count): stream B repeats stream A, unused
     const int offB = (pw == 2 ? STB : 0) + tl * TB;
-    const int off[2] = {kTPW == 2 ? tl * TB : (x ? offB : tl * TB), offB};
+    const int off[2] = {tl * TB, offB};
     float y[kTPW][NT][4];
 #pragma unroll
     for (int u = 0; u < kTPW; ++u)
@@ -496,34 +489,16 @@ __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, 
     if (W13) {
         __half *hs = hs2 + (items & 1) * (kChunk * kTileK);
         ++items;
-        float u[NT][4];
-        if (kTPW == 2) {
+        // y[0]: W1 x, y[1]: W3 x of the warp's rows
 #pragma unroll
-            for (int j = 0; j < NT; ++j)
+        for (int j = 0; j < NT; ++j)
 #pragma unroll
-                for (int c = 0; c < 4; ++c) u[j][c] = y[kTPW - 1][j][c];
-        } else {
-            float4 *xb = reinterpret_cast<float4 *>(xbuf + (tl * 32 + lane) * 8);
-            if (x == 1)
-#pragma unroll
-                for (int j = 0; j < NT; ++j) xb[j] = make_float4(y[0][j][0], y[0][j][1], y[0][j][2], y[0][j][3]);
-            if (!consumer_sync(p, sh, lane, cbar_uses)) return false;
-#pragma unroll
-            for (int j = 0; j < NT; ++j) {
-                const float4 v = xb[j];
-                u[j][0] = v.x; u[j][1] = v.y; u[j][2] = v.z; u[j][3] = v.w;
+            for (int c = 0; c < 4; ++c) {
+                const int n = 8 * j + t2 + (c & 1);
+                const int r = tl * 16 + g8 + 8 * (c >> 1);
+                const float hv = n < I.ci.nv ? silu(y[0][j][c]) * y[1][j][c] : 0.f;
+                hs[n * kTileK + r] = __float2half_rn(hv);
             }
-        }
-        if (kTPW == 2 || x == 0)
-#pragma unroll
-            for (int j = 0; j < NT; ++j)
-#pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    const int n = 8 * j + t2 + (c & 1);
-                    const int r = tl * 16 + g8 + 8 * (c >> 1);
-                    const float hv = n < I.ci.nv ? silu(y[0][j][c]) * u[j][c] : 0.f;
-                    hs[n * kTileK + r] = __float2half_rn(hv);
-                }
         // every warp finished the previous item's vector blocks before it got
         // here, so after this barrier the other h buffer is free again
         if (!consumer_sync(p, sh, lane, cbar_uses)) return false;
@@ -541,12 +516,8 @@ __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, 
                 const int r = tl * 16 + g8 + 8 * (c >> 1);
                 if (n < I.ci.nv) {
                     float *o = out + (size_t)(I.ci.pair_base + n) * p.H;
-                    if (kTPW == 2) {
-                        o[I.blkA * kBlockRows + r] = y[0][j][c];
-                        if (I.blkB >= 0) o[I.blkB * kBlockRows + r] = y[kTPW - 1][j][c];
-                    } else if (x == 0 || I.blkB >= 0) {
-                        o[(x ? I.blkB : I.blkA) * kBlockRows + r] = y[0][j][c];
-                    }
+                    o[I.blkA * kBlockRows + r] = y[0][j][c];
+                    if (I.blkB >= 0) o[I.blkB * kBlockRows + r] = y[1][j][c];
                 }
             }
     }
@@ -566,8 +537,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
     const int SB = slot_bytes(group, DENSE), VB = vec_bytes(group);
     const int vec_off0 = KPS * 2 * supertile_bytes(DENSE ? 16 : 3, group);
     __half *hs2 = reinterpret_cast<__half *>(smem + kRingOff + (size_t)S * SB);
-    float *xbuf = reinterpret_cast<float *>(smem + kRingOff + (size_t)S * SB + 2 * kHsBytes);
-    uint2 *afr = reinterpret_cast<uint2 *>(smem + kRingOff + (size_t)S * SB + 2 * kHsBytes + kXbufBytes);
+    uint2 *afr = reinterpret_cast<uint2 *>(smem + kRingOff + (size_t)S * SB + 2 * kHsBytes);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nrb = W13 ? p.F / kBlockRows : p.H / kBlockRows;  // 128-row blocks of the matrix
     const int U = W13 ? nrb : ((nrb + 1) / 2) * p.KS;
@@ -691,7 +661,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
     } else {
         // --------------------------------------------------------- consumers --
         const Ring R{full, empty, ring, S, SB, vec_off0, VB, afr};
-        const int x = kTPW == 2 ? 0 : warp >> 3, tl = warp & 7;
+        const int tl = warp;
         int slot = 0, items = 0, cbar_uses = 0;
         uint32_t phase = 0;
         while (true) {
@@ -702,7 +672,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
             const int sel = (I.ci.bits - 1) * 2 + (I.ci.nv > 8 ? 1 : 0);
             bool ok;
 #define MC_RUN(NT_, B_) \
-    run_item<W13, NT_, B_, GPT>(p, sh, R, I, nrb, x, tl, lane, slot, phase, xbuf, hs2, items, cbar_uses)
+    run_item<W13, NT_, B_, GPT>(p, sh, R, I, nrb, tl, lane, slot, phase, hs2, items, cbar_uses)
             if constexpr (DENSE) {
                 ok = I.ci.nv > 8 ? MC_RUN(2, 16) : MC_RUN(1, 16);
             } else switch (sel) {
