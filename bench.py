@@ -9,7 +9,8 @@ GEMV + SwiGLU, W2 GEMV, combine) on resident device inputs.  Packed weights
 rotate over several device copies so that no step finds its weights in L2.
 
   python bench.py [--gpus N] [--steps K] [--warmup W]
-                  [--workload decode16|decode1|decode4|prefill4096|odp256|odp256_b16|odp256_b13|stack32]
+                  [--workload decode16|decode1|decode4|decode16_8x22b|decode16_fp16|prefill4096|
+                              odp256|odp256_b16|odp256_b13|odp256_drop|odp256_mask|stack32]
   python bench.py --impl reference ...   (the CPU oracle on the host cores)
 
 Under torchrun every rank runs an independent replica (the layer does not need a
