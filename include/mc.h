@@ -154,10 +154,11 @@ int mc_route(const void *x, const void *gate_w, int T, const mc_shape *shape, fl
  *   x bf16 [T, H] (values must be finite and |x| <= 65504), gate_w bf16 [E, H],
  *   packed_dev: the buffer written by mc_pack_experts for (shape, bits_host),
  *   mu, protect as in mc_route, y bf16 [T, H] output.
- *   workspace: device scratch of at least mc_moe_workspace_size(shape, T) bytes,
- *   256-byte aligned, ZEROED before its first use (every call leaves the parts
- *   that need it at zero again); its first 4 bytes are the status word (see
- *   mc_check_status).
+ *   workspace: device scratch of mc_moe_workspace_size(shape, T_max) bytes for
+ *   some T_max >= T (one workspace serves every T up to the one it was sized
+ *   for), 256-byte aligned, ZEROED before its first use (every call leaves the
+ *   parts that need it at zero again; they sit at offsets that do not depend on
+ *   T); its first 4 bytes are the status word (see mc_check_status).
  *   topk_idx_out int32 [T,2], topk_w_out fp32 [T,2], pruned_out uint8 [T]: optional
  *   copies of the routing decisions (NULL to skip).
  * Never synchronises and never allocates; capturable in a CUDA graph.

@@ -92,7 +92,11 @@ static Workspace carve(const mc_shape *s, int T, void *base)
     w.max_chunks = max_chunks_for(T, s->E);
     const size_t P = 2 * (size_t)T, MC = (size_t)w.max_chunks;
     const size_t tb = (size_t)tab_bytes(s->group);
+    // The words that must be zero when a call starts (and that every call leaves
+    // at zero) come first, at offsets that do not depend on T, so one workspace
+    // serves calls with any T up to the T it was sized for.
     w.status = (int32_t *)take(256);
+    w.route_done = (int32_t *)take(4);
     w.idx = (int32_t *)take(P * 4);
     w.w = (float *)take(P * 4);
     w.pruned = (uint8_t *)take((size_t)T);
@@ -102,7 +106,6 @@ static Workspace carve(const mc_shape *s, int T, void *base)
     w.chunks = (ChunkInfo *)take(MC * sizeof(ChunkInfo));
     w.nchunks = (int32_t *)take(4);
     w.counters = (int32_t *)take(16);
-    w.route_done = (int32_t *)take(4);
     w.xfrag = (uint8_t *)take(MC * (s->H / kTileK) * kFragBytes);
     w.xtab = (float *)take(MC * (s->H / kTileK) * tb);
     w.hfrag = (uint8_t *)take(MC * (s->F / kTileK) * kFragBytes);

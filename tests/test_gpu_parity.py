@@ -255,6 +255,28 @@ def test_forward_token_drop(mc, T):
     assert_close(got, ref, "token drop T=%d" % T)
 
 
+def test_one_workspace_serves_every_token_count(mc):
+    """A workspace sized for 40 tokens serves calls with 1, 3, 16, 40 and again 1
+    and 3 tokens: the words a call counts on (the single-launch routing's arrival
+    count) sit at offsets that do not depend on T, so a call never finds another
+    T's data there.  Every output matches the oracle and, bit for bit, a call
+    with a fresh workspace of its own T."""
+    ws = mc.alloc_workspace(mc.Shape(8, 256, 512, 64), 40)
+    for T in (1, 3, 16, 40, 1, 3):
+        L = synth.make_layer(T, 256, 512, 8, 64, [3, 2, 2, 1, 3, 2, 2, 3], 87 + T, gate_std=0.1, mu=0.4,
+                             protect_frac=0.2)
+        condition_routing(L, L.mu)
+        shape, packed = _pack(mc, L)
+        x, g, p = to_dev(L)
+        y = mc.moe_forward(x, g, shape, L.bits, packed, L.mu, p, workspace=ws)
+        y_fresh = mc.moe_forward(x, g, shape, L.bits, packed, L.mu, p)
+        mc.check_status(ws)
+        torch.cuda.synchronize()
+        ref, *_ = oracle_layer(L, oracle_mats(L))
+        assert_close(y.float().cpu().numpy(), ref, "shared workspace T=%d" % T)
+        assert torch.equal(y, y_fresh), "shared vs fresh workspace, T=%d" % T
+
+
 @pytest.mark.parametrize("T,path", [(8, 1), (8, 2), (8, 3), (130, 0)])
 def test_forward_every_token_dropped(mc, T, path):
     """The degenerate batch: every token dropped (mask byte 2).  No pair reaches
