@@ -491,6 +491,11 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
                 bool bad = false;
 #pragma unroll
                 for (int n0 = 0; n0 < kGN; n0 += 16) {
+                    if (n0 >= gi.ci.nv) {  // no pair of the block in these columns: zero rows
+#pragma unroll
+                        for (int i = 0; i < 16; i += 2) hp[(n0 + i) / 2] = 0u;
+                        continue;
+                    }
                     uint32_t g[16], v[16];
                     tmem_ld_x16_nowait(tbase + lane_addr + (uint32_t)n0, g);
                     tmem_ld_x16_nowait(tbase + lane_addr + 128u + (uint32_t)n0, v);
@@ -517,7 +522,7 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
                 const int nstream = w2_pair_width(gi.u, nrb);
                 for (int x = 0; x < nstream; ++x) {
                     const int blk = 2 * gi.u + x;
-                    for (int n0 = 0; n0 < kGN; n0 += 16) {
+                    for (int n0 = 0; n0 < gi.ci.nv; n0 += 16) {
                         float v[16];
                         tmem_ld_x16(tbase + lane_addr + 128u * (uint32_t)x + (uint32_t)n0, v);
 #pragma unroll
