@@ -48,7 +48,8 @@ enum {
     MC_ERR_CUDA = -3,        /* a CUDA runtime call failed (message has the text) */
     MC_ERR_TIMEOUT = -4,     /* a bounded device wait expired (status word) */
     MC_ERR_BAD_PACK = -5,    /* packed buffer header does not match (magic/shape/bits) */
-    MC_ERR_RANGE = -6        /* an activation was non-finite or outside the fp16 range */
+    MC_ERR_RANGE = -6        /* an activation (x, or the SwiGLU product h that feeds W2) was
+                                non-finite or outside the fp16 range */
 };
 
 /* Layer shape.  E experts, hidden size H, SwiGLU width F, quantisation group
@@ -151,7 +152,9 @@ int mc_route(const void *x, const void *gate_w, int T, const mc_shape *shape, fl
 
 /* ------------------------------------------------------------------------ *
  * The whole layer (Eq. 1 with Eq. 5 on PMQ experts).
- *   x bf16 [T, H] (values must be finite and |x| <= 65504), gate_w bf16 [E, H],
+ *   x bf16 [T, H] (values must be finite and |x| <= 65504; the SwiGLU product
+ *   h = silu(W1 x) * (W3 x) that feeds W2 must be too, else the status word
+ *   reports MC_ERR_RANGE), gate_w bf16 [E, H],
  *   packed_dev: the buffer written by mc_pack_experts for (shape, bits_host),
  *   mu, protect as in mc_route, y bf16 [T, H] output.
  *   workspace: device scratch of mc_moe_workspace_size(shape, T_max) bytes for
@@ -188,10 +191,15 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
  *     scratch needs an initial value.
  *   Limit: the scratch must hold the call's buffers; a (shape, T) that needs
  *     more than 16 MiB returns MC_ERR_INVALID_ARG with the size in the message
- *     (at the Mixtral-8x7b shape, H 4096, F 14336, group 128, that is T > 52).
+ *     (at the Mixtral-8x7b shape, H 4096, F 14336, group 128, that is T > 96).
+ *     The W2 pass takes mc_moe_forward's column splits when their partial
+ *     outputs fit in the scratch, else a single split (same results).
  *   Set-up: the first call on a device, made with that device current, looks up
- *     the scratch's address once (cudaGetSymbolAddress); make that first call
- *     before any stream capture.
+ *     the scratch's address once (cudaGetSymbolAddress) and keeps it for the
+ *     life of the process; make that first call before any stream capture, and
+ *     do not call it on a device after cudaDeviceReset (a reset reloads the
+ *     library's device code, and the scratch may then sit elsewhere).
+ *   The mc_set_debug hooks (flags, wait bound) apply as for mc_moe_forward.
  *   Concurrency: every call on a device uses the same scratch, so calls whose
  *     kernels may overlap (other streams, other host threads) race and corrupt
  *     each other's results; order them (one stream, or events). */
@@ -272,11 +280,13 @@ int mc_expert_significance_host(const int32_t *idx, const float *w, const uint8_
 int mc_pmq_allocate(const double *phi, const double *wact, const double *eps, int E, int bits_total, double alpha,
                     double beta, double gamma, int8_t *bits_out, double *objective_out);
 
-/* Choose the expert path of mc_moe_forward: 0 = automatic (the GEMV below 240
- * kept-or-not pairs, 2T < 240, else the GEMM), 1 = the mma.sync grouped GEMV
- * (decode), 2 = the tcgen05 grouped GEMV with chunks of 16 pairs, 3 = the
- * tcgen05 grouped GEMM with token blocks of 128 pairs (prefill).
- * Process-wide; returns the previous value. */
+/* Test hook: choose the expert path of mc_moe_forward: 0 = automatic (the GEMV
+ * below 240 kept-or-not pairs, 2T < 240, else the GEMM), 1 = the mma.sync
+ * grouped GEMV with work chunks of 16 pairs (decode), 2 = the tcgen05 grouped
+ * GEMM with token blocks of 128 pairs (prefill).  Both paths compute the same
+ * layer; forcing one lets tests run both kernels at the same sizes.
+ * Process-wide (an atomic word read once per mc_moe_forward call); returns the
+ * previous value, or MC_ERR_INVALID_ARG (and no change) for another value. */
 int mc_set_path(int path);
 
 /* Test hook: `flags` bit 0 makes the expert kernels' weight producer issue no
@@ -308,8 +318,8 @@ int mc_check_status(void *workspace, void *stream);
  * the launching stream (for benchmarks; off by default).  mc_profile_read
  * synchronises on the recorded events, writes the summed milliseconds and launch
  * counts of kernel ids 0 .. n-1 (names from mc_profile_name: route, permute,
- * gemv_w13, gemv_w2, combine, gemm_gather, gemm_w13, gemm_w2, rmsnorm, glu,
- * importance) and
+ * gemv_w13, gemv_w2, combine, frag_x, gemm_w13, gemm_w2, rmsnorm, importance,
+ * x_img) and
  * clears the records.  Inside stream capture the events become event nodes of
  * the graph: every replay records them again, and each mc_profile_read reports
  * the latest replay and keeps those records until mc_profile_clear. */

@@ -331,7 +331,12 @@ def check_status(workspace) -> None:
 
 
 def set_path(path: int) -> int:
-    return load().mc_set_path(int(path))
+    """Force the expert path of moe_forward (PATH_AUTO, PATH_GEMV, PATH_GEMM);
+    returns the previous one."""
+    r = load().mc_set_path(int(path))
+    if r < 0:
+        _check(r)
+    return r
 
 
 def set_debug(flags: int, timeout_ns: int = 0) -> None:

@@ -13,7 +13,9 @@
 
 namespace mc {
 
-static std::atomic<int> g_path{0};
+// expert paths of mc_moe_forward (mc_set_path)
+constexpr int kPathAuto = 0, kPathGemv = 1, kPathGemm = 2;
+static std::atomic<int> g_path{kPathAuto};
 // pairs (2 T) from which mc_moe_forward's automatic choice is the prefill GEMM:
 // measured on the Mixtral-8x7b layer, the GEMV path (each weight tile decoded
 // once per 16-pair chunk) is faster up to ~96 tokens, the GEMM (once per
@@ -37,9 +39,9 @@ static inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 // chunks x 256-row block pairs x splits) fill the SMs' last wave best, the
 // smaller one on ties.
 
-static int max_ks(const mc_shape *s, int T) { return T > 64 ? 1 : kMaxKS; }
+int max_ks(const mc_shape *s, int T) { return T > 64 ? 1 : kMaxKS; }
 
-static int choose_ks(const mc_shape *s, int T, int nsm)
+int choose_ks(const mc_shape *s, int T, int nsm)
 {
     const int nt = s->F / kTileK, npairs = (s->H / kBlockRows + 1) / 2;
     const int chunks = 2 * T < s->E ? 2 * T : s->E;  // pairs land on distinct experts at small T
@@ -66,11 +68,6 @@ struct Workspace {
     ChunkInfo *chunks;
     int32_t *nchunks, *counters;
     int32_t *route_done;  // zero between calls: single-launch routing for small T
-    uint8_t *xfrag;
-    float *xtab;
-    uint8_t *hfrag;
-    float *htab;
-    float *gu;
     uint8_t *xvec, *hvec;
     uint8_t *ximg, *himg;
     float *opart;
@@ -91,7 +88,6 @@ static Workspace carve(const mc_shape *s, int T, void *base)
     w.KS = max_ks(s, T);  // room for the largest split count the forward may pick
     w.max_chunks = max_chunks_for(T, s->E);
     const size_t P = 2 * (size_t)T, MC = (size_t)w.max_chunks;
-    const size_t tb = (size_t)tab_bytes(s->group);
     // The words that must be zero when a call starts (and that every call leaves
     // at zero) come first, at offsets that do not depend on T, so one workspace
     // serves calls with any T up to the T it was sized for.
@@ -106,11 +102,6 @@ static Workspace carve(const mc_shape *s, int T, void *base)
     w.chunks = (ChunkInfo *)take(MC * sizeof(ChunkInfo));
     w.nchunks = (int32_t *)take(4);
     w.counters = (int32_t *)take(16);
-    w.xfrag = (uint8_t *)take(MC * (s->H / kTileK) * kFragBytes);
-    w.xtab = (float *)take(MC * (s->H / kTileK) * tb);
-    w.hfrag = (uint8_t *)take(MC * (s->F / kTileK) * kFragBytes);
-    w.htab = (float *)take(MC * (s->F / kTileK) * tb);
-    w.gu = (float *)take(MC * 2 * (size_t)s->F * kChunk * 4);
     w.xvec = (uint8_t *)take(MC * 2 * (s->H / kTileK) * (size_t)vec_bytes(s->group));
     w.hvec = (uint8_t *)take(MC * 2 * (s->F / kTileK) * (size_t)vec_bytes(s->group));
     w.max_blocks = max_blocks_for(T, s->E);
@@ -135,6 +126,8 @@ static float neg_log_mu(float mu)
 }
 
 bool pdl_enabled() { return !(g_debug.load() & kDebugNoPdl); }
+int debug_flags() { return g_debug.load(); }
+uint64_t wait_bound_ns() { return g_timeout_ns.load(); }
 
 }  // namespace mc
 
@@ -144,6 +137,10 @@ extern "C" {
 
 int mc_set_path(int path)
 {
+    if (path != kPathAuto && path != kPathGemv && path != kPathGemm) {
+        clear_error();
+        return set_error(MC_ERR_INVALID_ARG, "path %d: 0 (automatic), 1 (GEMV) or 2 (GEMM)", path);
+    }
     return g_path.exchange(path);
 }
 
@@ -229,8 +226,8 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     int path = g_path;
     // 16-bit (unquantised) experts have the mma.sync kernels only
     const bool dense = bits_host[0] == 16;
-    if (path == 0) path = dense ? 1 : 2 * T >= kPrefillPairs ? 3 : 1;
-    if (dense && path != 1)
+    if (path == kPathAuto) path = dense ? kPathGemv : 2 * T >= kPrefillPairs ? kPathGemm : kPathGemv;
+    if (dense && path != kPathGemv)
         return set_error(MC_ERR_UNSUPPORTED, "16-bit experts run on the mma.sync path only (path %d requested)", path);
 
     RouteParams rp{};
@@ -261,7 +258,7 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     pp.chunks = ws.chunks;
     pp.nchunks = ws.nchunks;
     pp.counters = ws.counters;
-    pp.chunk = path == 3 ? 128 : kChunk;
+    pp.chunk = path == kPathGemm ? 128 : kChunk;
     rc = launch_route(rp, pp, st, ws.route_done);
     if (rc) return rc;
 
@@ -280,11 +277,6 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     ep.counters = ws.counters;
     ep.x = (const __nv_bfloat16 *)x;
     ep.perm = ws.perm;
-    ep.xfrag = ws.xfrag;
-    ep.xtab = ws.xtab;
-    ep.hfrag = ws.hfrag;
-    ep.htab = ws.htab;
-    ep.gu = ws.gu;
     ep.xvec = ws.xvec;
     ep.hvec = ws.hvec;
     ep.ximg = ws.ximg;
@@ -294,13 +286,13 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     int nsm = 0, dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
         return set_error(MC_ERR_CUDA, "device query failed");
-    ep.KS = path == 3 ? 1 : choose_ks(shape, T, nsm);  // the GEMM's W2 pass covers all of F at once
+    ep.KS = path == kPathGemm ? 1 : choose_ks(shape, T, nsm);  // the GEMM's W2 pass covers all of F at once
     ep.Pmax = 2 * T;
     ep.max_chunks = ws.max_chunks;
     ep.status = ws.status;
     ep.timeout_ns = g_timeout_ns;
     ep.debug = g_debug;
-    rc = path == 3 ? launch_gemm(ep, st) : path == 2 ? launch_tc(ep, st) : launch_gemv(ep, st);
+    rc = path == kPathGemm ? launch_gemm(ep, st) : launch_gemv(ep, st);
     if (rc) return rc;
 
     CombineParams cp{};

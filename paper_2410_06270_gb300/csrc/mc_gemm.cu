@@ -580,9 +580,9 @@ int launch_gemm(ExpertParams ep, cudaStream_t st)
     if (err == cudaSuccess) err = cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGSmem);
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(err));
 
-    profile_begin(kKGemmGather, st);
+    profile_begin(kKXImg, st);
     err = launch_k(x_img_kernel, dim3(ep.max_blocks, ep.H / kTileK), dim3(256), 0, st, ep);
-    profile_end(kKGemmGather, st);
+    profile_end(kKXImg, st);
     if (err == cudaSuccess) {
         profile_begin(kKGemmW13, st);
         err = launch_k(k13, dim3(nsm), dim3(kGThreads), kGSmem, st, ep);

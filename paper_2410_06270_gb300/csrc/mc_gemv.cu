@@ -489,7 +489,9 @@ __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, 
     if (W13) {
         __half *hs = hs2 + (items & 1) * (kChunk * kTileK);
         ++items;
-        // y[0]: W1 x, y[1]: W3 x of the warp's rows
+        // y[0]: W1 x, y[1]: W3 x of the warp's rows; h is W2's fp16 input, so a
+        // value outside the fp16 range (or not finite) is reported, as for x
+        bool bad = false;
 #pragma unroll
         for (int j = 0; j < NT; ++j)
 #pragma unroll
@@ -497,8 +499,10 @@ __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, 
                 const int n = 8 * j + t2 + (c & 1);
                 const int r = tl * 16 + g8 + 8 * (c >> 1);
                 const float hv = n < I.ci.nv ? silu(y[0][j][c]) * y[1][j][c] : 0.f;
+                bad |= !(fabsf(hv) <= 65504.f);
                 hs[n * kTileK + r] = __float2half_rn(hv);
             }
+        if (bad) set_status(p.status, MC_ERR_RANGE);
         // every warp finished the previous item's vector blocks before it got
         // here, so after this barrier the other h buffer is free again
         if (!consumer_sync(p, sh, lane, cbar_uses)) return false;
@@ -766,9 +770,9 @@ int launch_gemv(ExpertParams ep, cudaStream_t st)
     if (err == cudaSuccess) err = cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(err));
 
-    profile_begin(kKGemmGather, st);
+    profile_begin(kKFragX, st);
     err = launch_k(frag_x_kernel, dim3(ep.max_chunks, ep.H / kTileK), dim3(256), 0, st, ep);
-    profile_end(kKGemmGather, st);
+    profile_end(kKFragX, st);
     if (err == cudaSuccess) {
         profile_begin(kKGemvW13, st);
         err = launch_k(k13, dim3(nsm), dim3(kGemvThreads), sm, st, ep);

@@ -76,11 +76,6 @@ struct ExpertParams {
     int32_t *counters;
     const __nv_bfloat16 *x;  // [T, H]
     const int32_t *perm;     // [P]
-    uint8_t *xfrag;          // [max_chunks][H/128] kFragBytes
-    float *xtab;             // [max_chunks][H/128] tab_bytes
-    uint8_t *hfrag;          // [max_chunks][F/128] kFragBytes
-    float *htab;             // [max_chunks][F/128] tab_bytes
-    float *gu;               // [max_chunks][2][F][16] W1 / W3 results (tensor-core path)
     uint8_t *xvec;           // [max_chunks][2][H/128] vector blocks of x (mma.sync path)
     uint8_t *hvec;           // [max_chunks][2][F/128] vector blocks of h (mma.sync path)
     uint8_t *ximg;           // [max_blocks][H/128] 32 KB activation images (prefill path)
@@ -136,12 +131,19 @@ inline cudaError_t launch_k(void (*kernel)(P...), dim3 grid, dim3 block, size_t 
 // T <= 64 (left at zero), or NULL for two launches.
 int launch_route(const RouteParams &rp, const PermuteParams &pp, cudaStream_t st, int32_t *done = nullptr);
 int launch_gemv(ExpertParams ep, cudaStream_t st);   // mma.sync path
-int launch_tc(ExpertParams ep, cudaStream_t st);     // tcgen05 path
 int launch_gemm(ExpertParams ep, cudaStream_t st);   // prefill path (tcgen05 grouped GEMM)
 size_t img_buffer_bytes(int max_blocks, int cols);
 int max_blocks_for(int T, int E);
 int launch_combine(const CombineParams &cp, cudaStream_t st);
 int max_chunks_for(int T, int E);
 int32_t *route_done_word();  // mc_route's arrival word for the single-launch routing
+// Column splits of the W2 GEMV pass: the most a workspace for T tokens holds, and
+// the count a forward picks (the one whose work items fill the SMs' last wave
+// best, among the divisors of F/128 that leave every item >= 8 column steps).
+int max_ks(const mc_shape *s, int T);
+int choose_ks(const mc_shape *s, int T, int nsm);
+// The test hooks of mc_set_debug: its flags and the bound on device waits.
+int debug_flags();
+uint64_t wait_bound_ns();
 
 }  // namespace mc

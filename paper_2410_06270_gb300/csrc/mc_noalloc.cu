@@ -56,7 +56,8 @@ struct StaticWs {
     size_t total;
 };
 
-static StaticWs carve_static(const mc_shape *s, int T, uint8_t *base)
+// KS: column splits of the W2 pass (the fp32 partial outputs hold KS copies).
+static StaticWs carve_static(const mc_shape *s, int T, int KS, uint8_t *base)
 {
     StaticWs w;
     size_t off = 0;
@@ -65,14 +66,7 @@ static StaticWs carve_static(const mc_shape *s, int T, uint8_t *base)
         off = (off + bytes + 255) & ~(size_t)255;
         return r;
     };
-    // column splits of the W2 pass: the rule mc_moe_forward uses
-    w.KS = 1;
-    if (T <= 64)
-        for (int ks : {4, 2})
-            if ((s->F / kTileK) % ks == 0) {
-                w.KS = ks;
-                break;
-            }
+    w.KS = KS;
     w.max_chunks = max_chunks_for(T, s->E);
     const size_t P = 2 * (size_t)T, MC = (size_t)w.max_chunks, VB = (size_t)vec_bytes(s->group);
     w.status = (int32_t *)take(256);
@@ -111,7 +105,17 @@ extern "C" int mc_moe_forward_static(const void *x, const void *gate_w, int T, c
     if (!aligned(x, 16) || !aligned(gate_w, 16) || !aligned(y, 16) || !aligned(packed_dev, 256) ||
         (status_dev && !aligned(status_dev, 4)))
         return set_error(MC_ERR_INVALID_ARG, "x, gate_w, y need 16-byte and packed_dev 256-byte alignment");
-    const size_t need = carve_static(shape, T, nullptr).total;
+    // W2 column splits: mc_moe_forward's choice when its partial outputs fit in
+    // the scratch, else a single split (the limit below is the single split's)
+    int dev = 0, nsm = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return set_error(MC_ERR_CUDA, "device query failed");
+    int KS = choose_ks(shape, T, nsm);
+    size_t need = carve_static(shape, T, KS, nullptr).total;
+    if (need > kStaticScratchBytes && KS > 1) {
+        KS = 1;
+        need = carve_static(shape, T, KS, nullptr).total;
+    }
     if (need > kStaticScratchBytes)
         return set_error(MC_ERR_INVALID_ARG,
                          "T=%d needs %zu bytes of scratch, more than the %zu-byte static scratch of "
@@ -119,7 +123,7 @@ extern "C" int mc_moe_forward_static(const void *x, const void *gate_w, int T, c
                          T, need, kStaticScratchBytes);
     void *base = nullptr;
     if ((rc = static_scratch(&base))) return rc;
-    const StaticWs ws = carve_static(shape, T, (uint8_t *)base);
+    const StaticWs ws = carve_static(shape, T, KS, (uint8_t *)base);
     cudaStream_t st = (cudaStream_t)stream;
     int32_t *status = status_dev ? status_dev : ws.status;
     if (!status_dev) {
@@ -177,7 +181,8 @@ extern "C" int mc_moe_forward_static(const void *x, const void *gate_w, int T, c
     ep.Pmax = 2 * T;
     ep.max_chunks = ws.max_chunks;
     ep.status = status;
-    ep.timeout_ns = 1000000000ull;
+    ep.timeout_ns = wait_bound_ns();  // the mc_set_debug hooks apply here as well
+    ep.debug = debug_flags();
     if ((rc = launch_gemv(ep, st))) return rc;
 
     CombineParams cp{};

@@ -20,7 +20,7 @@ std::vector<Rec> g_recs;
 std::vector<cudaEvent_t> g_pool;
 cudaEvent_t g_pending[kKCount];
 const char *g_names[kKCount] = {"route", "permute", "gemv_w13", "gemv_w2", "combine",
-                                "gemm_gather", "gemm_w13", "gemm_w2", "rmsnorm", "glu", "importance"};
+                                "frag_x", "gemm_w13", "gemm_w2", "rmsnorm", "importance", "x_img"};
 
 // An event record on st; inside stream capture it becomes an event node of the
 // graph, so every replay of the graph records it again.

@@ -11,12 +11,12 @@ enum KernelId {
     kKGemvW13,
     kKGemvW2,
     kKCombine,
-    kKGemmGather,
+    kKFragX,      // decode path: activations -> vector blocks
     kKGemmW13,
     kKGemmW2,
     kKRmsnorm,
-    kKGlu,
     kKImportance,
+    kKXImg,       // prefill path: activations -> SW128 images
     kKCount
 };
 

@@ -83,3 +83,26 @@ def assert_close(got, ref, what=""):
     print("[parity] %s rel_fro=%.3e max_abs/max=%.3e" % (what, rel, mx))
     assert rel <= REL_FRO and mx <= MAX_ABS, "%s rel_fro=%.3e max_abs/max=%.3e" % (what, rel, mx)
     return rel, mx
+
+
+def boundary_tokens(L, mu=None, blocks=(16, 128)):
+    """Tokens whose outputs cover the edges of the expert kernels' work units at a
+    full shape: for every expert, the first and the last pair of its first and of
+    its last (ragged) block of `block` pairs, for each block size the kernels use
+    (16-pair GEMV chunks, 128-pair GEMM token blocks).  The pairs come from the
+    oracle's routing and permutation (pairs grouped by expert, ascending token).
+    Every sampled token's output spans all W1|W3 row blocks and every W2 row
+    block and column split."""
+    mu = L.mu if mu is None else mu
+    idx, _, pr = oracle.route(L.x_f32(), L.gate_f32(), mu, L.protect)
+    off, perm = oracle.permute(idx, pr, L.E)
+    toks = set()
+    for e in range(L.E):
+        a, b = int(off[e]), int(off[e + 1])
+        if a == b:
+            continue
+        for blk in blocks:
+            last = a + ((b - 1 - a) // blk) * blk  # first pair of the last block
+            for q in (a, min(a + blk, b) - 1, last, b - 1):
+                toks.add(int(perm[q]) >> 1)
+    return sorted(toks)

@@ -235,3 +235,18 @@ def test_pmq_allocation_matches_oracle():
         assert bits.sum() == total and (bits == 3).any() and (bits == 2).any()
     with pytest.raises(mc.MCError):
         mc.pmq_allocate(phi, wact, eps, 25)
+
+
+def test_set_path_accepts_only_the_two_paths(mc):
+    """mc_set_path: 0 (automatic), 1 (GEMV), 2 (GEMM); any other value is
+    rejected and leaves the choice unchanged (host code only)."""
+    prev = mc.set_path(mc.PATH_GEMV)
+    try:
+        for bad in (-1, 3, 7):
+            with pytest.raises(mc.MCError) as ei:
+                mc.set_path(bad)
+            assert ei.value.code == mc.ERR_INVALID_ARG
+        assert mc.set_path(mc.PATH_GEMM) == mc.PATH_GEMV
+        assert mc.set_path(mc.PATH_AUTO) == mc.PATH_GEMM
+    finally:
+        mc.set_path(prev)

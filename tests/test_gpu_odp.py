@@ -3,13 +3,14 @@
 secondary expert of ~15% of the unprotected tokens (Eq. 5, Sec. 2.3.2), at the
 three bit budgets (sum 20 / 16 / 13).  Routing, prune flags and the permutation
 bit-exact on all tokens; outputs on sampled tokens (protected, pruned and kept
-ones) against the oracle, on the automatic (GEMM) path and on the GEMV path."""
+ones, and the edges of every expert's work chunks and token blocks) against the
+oracle, on the automatic (GEMM) path and on the GEMV path."""
 import numpy as np
 import pytest
 
 import oracle
 import synth
-from helpers import assert_close, condition_routing, flat, oracle_layer, oracle_mats, to_dev
+from helpers import assert_close, boundary_tokens, condition_routing, flat, oracle_layer, oracle_mats, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -49,7 +50,9 @@ def test_odp_layer(mc, bits_total):
     prot = np.nonzero(L.protect)[0]
     kept = np.nonzero((opr == 0) & (L.protect == 0))[0]
     assert 0.05 * L.T < len(pruned) < 0.25 * L.T
-    tokens = sorted(set(pruned[:2].tolist() + prot[:2].tolist() + kept[:2].tolist()))
+    # protected, pruned and kept tokens, and the edges of every expert's 16-pair
+    # GEMV chunks and 128-pair GEMM token blocks (from the oracle's permutation)
+    tokens = sorted(set(pruned[:2].tolist() + prot[:2].tolist() + kept[:2].tolist() + boundary_tokens(L)))
     mats = oracle_mats(L)
     ref, *_ = oracle_layer(L, mats, tokens)
     for path in (0, 1):

@@ -1,14 +1,17 @@
 """GPU parity of the stacked workload: pre-norm residual MoE layers
 (h <- h + MoE_l(RMSNorm(h)), per-layer gates and ODP thresholds, protected
-tokens) through mc_stack_forward against the oracle's stack; and the stack
-captured into one CUDA graph equal, bit for bit, to the eager call (at the
-Mixtral-8x7b shape too)."""
+tokens) through mc_stack_forward against the oracle's stack; the Mixtral-8x7b
+stack of 32 layers against the oracle layer by layer with teacher forcing; and
+the stack captured into one CUDA graph equal, bit for bit, to the eager call (at
+the Mixtral-8x7b shape too)."""
+import os
+
 import numpy as np
 import pytest
 
 import oracle
 import synth
-from helpers import assert_close, flat, oracle_mats
+from helpers import assert_close, errors, flat, oracle_mats
 
 pytestmark = pytest.mark.gpu
 
@@ -126,3 +129,103 @@ def test_stack_same_without_programmatic_launch(mc):
     torch.cuda.synchronize()
     mc.check_status(ws)
     assert torch.equal(h_on.view(torch.int16), h_off.view(torch.int16))
+
+
+def test_stack_mixtral_teacher_forced(mc):
+    """The stack workload at the Mixtral-8x7b shape (32 layers, 32 tokens, H 4096,
+    F 14336, bits sum 20, ODP on with per-layer mu dropping the secondary expert
+    of 15% of the unprotected tokens, 10% of tokens protected), checked layer by
+    layer with teacher forcing: the oracle's layer l consumes the GPU's own bf16
+    input to layer l (its RMSNorm output), so that every layer is compared on
+    the same inputs however far the trajectories drift apart.
+      - The layer-by-layer calls (mc_rmsnorm, mc_moe_forward, mc_add) reproduce
+        mc_stack_forward bit for bit, so these are the stack's own layers.
+      - Routing (top-2, weights, prune flags) against the oracle on every token
+        whose fp64 logits lie more than 1e-4 from a top-2 tie or from the ODP
+        threshold; the others are reported and excluded.
+      - Every layer's output y_l on two tokens per layer (64 in all, every token
+        twice), within the output tolerance.
+      - The end-to-end drift of the whole stack against the oracle's own
+        trajectory on two tokens is printed, not gated (Eq. 1 per layer; the
+        paper's Mixtral models have 32 MoE layers)."""
+    import concurrent.futures as cf
+    layers, T = 32, 32
+    L, gates = synth.config_stack(T=T, layers=layers)
+    shape = mc.Shape(L.E, L.H, L.F, L.group)
+    packed = mc.pack_experts(shape, L.bits, flat(L, "codes"), flat(L, "scale"), flat(L, "zero"))
+    gw = [_dev_bf16(g) for g in gates]
+    gamma = torch.ones((layers, L.H), dtype=torch.bfloat16, device="cuda")
+    prot = torch.from_numpy(L.protect.copy()).cuda()
+    ws = mc.alloc_workspace(shape, T)
+    # layer by layer, with the stack's per-layer thresholds from its own trajectory
+    h = _dev_bf16(L.x)
+    mus, xns, ys, routes = [], [], [], []
+    for l in range(layers):
+        xn = mc.rmsnorm(h, gamma[l])
+        r0 = mc.route(xn, gw[l], shape, 0.0, prot)
+        w0 = r0["w"].cpu().numpy().astype(np.float64)
+        mus.append(float(np.quantile((w0[:, 1] / w0[:, 0])[L.protect == 0], 0.15)))
+        y, r = mc.moe_forward(xn, gw[l], shape, L.bits, packed, mus[-1], prot, workspace=ws, routing=True)
+        mc.check_status(ws)
+        h = mc.add(h, y)
+        xns.append(xn.view(torch.int16).cpu().numpy().view(np.uint16))
+        ys.append(y.float().cpu().numpy().astype(np.float64))
+        routes.append((r["idx"].cpu().numpy(), r["w"].cpu().numpy(), r["pruned"].cpu().numpy()))
+    # the same layers through mc_stack_forward, bit for bit
+    args = mc.StackArgs(gw, [L.bits] * layers, [packed] * layers, mus)
+    hs = _dev_bf16(L.x)
+    mc.stack_forward(hs, shape, args, gamma, mc.stack_workspace(shape, T), prot)
+    torch.cuda.synchronize()
+    assert torch.equal(hs.view(torch.int16), h.view(torch.int16))
+
+    mats = oracle_mats(L)
+    gates_f = [synth.bf16_bits_to_f32(g) for g in gates]
+    excluded, jobs = 0, []
+    for l in range(layers):
+        xf = synth.bf16_bits_to_f32(xns[l])
+        lg = oracle.gate_logits(xf, gates_f[l])
+        srt = -np.sort(-lg, axis=1)
+        clear = (srt[:, 0] - srt[:, 1] > 1e-4) & (srt[:, 1] - srt[:, 2] > 1e-4) & \
+                (np.abs((srt[:, 0] - srt[:, 1]) + np.log(mus[l])) > 1e-4)
+        excluded += int((~clear).sum())
+        oidx, ow, opr = oracle.route(xf, gates_f[l], mus[l], L.protect)
+        gidx, gwt, gpr = routes[l]
+        np.testing.assert_array_equal(gidx[clear], oidx[clear], err_msg="layer %d top-2" % l)
+        np.testing.assert_array_equal(gpr[clear], opr[clear], err_msg="layer %d prune flags" % l)
+        np.testing.assert_allclose(gwt[clear], ow[clear], rtol=2e-6, atol=2e-6, err_msg="layer %d weights" % l)
+        assert 0 < int((opr == 1).sum()) and int((opr[L.protect == 1] == 1).sum()) == 0
+        toks = [t for t in ((2 * l) % T, (2 * l + 1) % T) if clear[t]]
+        jobs += [(l, t, xf) for t in toks]
+    print("[stack32] routing compared on %d of %d token-layers (%d within 1e-4 of a tie or the threshold)" % (
+        layers * T - excluded, layers * T, excluded))
+    assert excluded <= layers * T // 20
+
+    def one(job):
+        l, t, xf = job
+        yo, *_ = oracle.moe_layer(xf, gates_f[l], mats, mus[l], L.protect, tokens=[t])
+        return yo[0]
+
+    with cf.ThreadPoolExecutor(os.cpu_count() or 4) as ex:
+        refs = list(ex.map(one, jobs))
+    for l in range(layers):
+        sel = [i for i, j in enumerate(jobs) if j[0] == l]
+        if sel:
+            got = np.stack([ys[l][jobs[i][1]] for i in sel])
+            assert_close(got, np.stack([refs[i] for i in sel]), "stack32 layer %d (teacher forced)" % l)
+    got_all = np.concatenate([ys[jobs[i][0]][jobs[i][1]][None] for i in range(len(jobs))])
+    rel, mx = errors(got_all, np.stack(refs))
+    print("[stack32] all %d sampled layer outputs: rel_fro=%.3e max_abs/max=%.3e" % (len(jobs), rel, mx))
+
+    # end-to-end drift of the whole stack on two tokens (reported only)
+    drift_toks = [0, T - 1]
+
+    def traj(t):
+        return oracle.stack(L.x_f32()[t:t + 1], gates_f, mats, mus, L.protect[t:t + 1])[0][0]
+
+    with cf.ThreadPoolExecutor(len(drift_toks)) as ex:
+        h_ref = np.stack(list(ex.map(traj, drift_toks)))
+    x0 = L.x_f32().astype(np.float64)[drift_toks]
+    h_got = h.float().cpu().numpy().astype(np.float64)[drift_toks]
+    rel, mx = errors(h_got - x0, h_ref - x0)
+    print("[stack32] end-to-end drift after %d layers on tokens %s: rel_fro=%.3e max_abs/max=%.3e (not gated)" % (
+        layers, drift_toks, rel, mx))
