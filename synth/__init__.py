@@ -12,15 +12,21 @@ below:
 * activations x ~ N(0, 1), rounded to bf16;
 * gate weight Wg ~ N(0, 0.02), rounded to bf16 (optionally tilted along a shared
   direction so that expert loads are skewed);
-* expert codes drawn uniformly in [0, 2**b - 1] per weight (b = the expert's bit
-  width), one fp16 scale per group with the magnitude a min-max quantiser gives
-  an N(0, 0.02) group, an fp16 zero that is an integer in the code range for
-  b >= 2 and 1/2 for b = 1 (the binary format of the paper's appendix);
-  ``zero_mode="fractional"`` draws arbitrary fp16 zeros instead;
+* expert weights N(0, 0.02) quantised per group by ``rtn_quantize`` (round to
+  nearest min-max for b = 2, 3; the sign rule of the paper's appendix for b = 1)
+  in the named single-layer configurations; or, for the small test layers, the
+  32-layer stack and the Mixtral-8x22b layer, codes drawn uniformly in
+  [0, 2**b - 1] per weight (b = the expert's bit width), one fp16 scale per group
+  with the magnitude a min-max quantiser gives an N(0, 0.02) group, an fp16 zero
+  that is an integer in the code range for b >= 2 and 1/2 for b = 1 (the binary
+  format of the paper's appendix); ``zero_mode="fractional"`` draws arbitrary
+  fp16 zeros instead;
 * protect masks choose a seeded subset of tokens.
 """
 from __future__ import annotations
 
+import concurrent.futures as cf
+import os
 from dataclasses import dataclass, field
 
 import numpy as np
@@ -135,6 +141,41 @@ def expert_matrix(seed, e, m, rows, cols, group, bits, zero_mode="integer"):
     return codes, scale, zero
 
 
+def expert_weights_f32(seed, e, m, rows, cols, std=0.02):
+    """The unquantised weights of matrix m (0=w1, 1=w3, 2=w2) of expert e:
+    N(0, std) float32 [rows, cols], from their own seeded stream."""
+    return _rng(seed, 4000 + e, m).standard_normal((rows, cols), dtype=np.float32) * np.float32(std)
+
+
+def rtn_quantize(w, bits, group):
+    """Quantiser of the synthetic expert weights (input generation: the paper
+    quantises with GPTQ, Sec. 2.2.2, which needs calibration data and trained
+    weights; this stands in for it), per group of `group` consecutive columns:
+      b = 2, 3  round-to-nearest min-max: s = fp16((max - min) / (2^b - 1)), 1 if
+                max = min; z = clip(rint(-min / s), 0, 2^b - 1), an integer stored
+                in fp16; q = clip(rint(w / s + z), 0, 2^b - 1), ties to even;
+      b = 1     the sign rule of App. A.2 with sign(0) = +1: q = (w >= 0), z = 1/2,
+                s = fp16(2 * mean |w|) of the group (App. A.2's scale is per matrix;
+                per group refines it in the same storage format).
+    Returns (codes uint8 [rows, cols], scale fp16 [rows, cols/group], zero fp16)."""
+    w = np.asarray(w, np.float32)
+    rows, cols = w.shape
+    ng = cols // group
+    wg = w.reshape(rows, ng, group)
+    if bits == 1:
+        scale = (np.float32(2.0) * np.abs(wg).mean(axis=2, dtype=np.float32)).astype(np.float16)
+        zero = np.full((rows, ng), 0.5, np.float16)
+        return (w >= 0).astype(np.uint8), scale, zero
+    levels = np.float32((1 << bits) - 1)
+    mn, mx = wg.min(axis=2), wg.max(axis=2)
+    scale = ((mx - mn) / levels).astype(np.float16)
+    scale[scale == 0] = np.float16(1.0)
+    s = scale.astype(np.float32)
+    z = np.clip(np.rint(-mn / s), 0, levels)
+    q = np.clip(np.rint(wg / s[:, :, None] + z[:, :, None]), 0, levels).astype(np.uint8)
+    return q.reshape(rows, cols), scale, z.astype(np.float16)
+
+
 def bit_table(seed, E, total, lo=1, hi=3):
     """A seeded per-expert bit table with the given sum, values in [lo, hi], with at
     least one 3-bit and one 2-bit expert (the constraints of the paper's Eq. 4)."""
@@ -147,12 +188,16 @@ def bit_table(seed, E, total, lo=1, hi=3):
 
 
 def make_layer(T, H, F, E, group, bits, seed, *, gate_std=0.02, mu=0.0,
-               protect_frac=0.0, zero_mode="integer", skew=None, experts=True):
+               protect_frac=0.0, zero_mode="integer", skew=None, experts=True, quant="direct"):
     """One layer of synthetic inputs.
 
     ``skew``: None, or (c, beta) -- x gets +c along a seeded unit direction u and
     gate row e gets +beta*(e - (E-1)/2)/((E-1)/2) * u, which tilts expert loads.
     ``experts=False`` skips the expert weights (routing-only tests).
+    ``quant``: "direct" draws the codes uniformly with scales and zeros of a
+    quantised N(0, 0.02) group's magnitude (``expert_matrix``); "rtn" draws the
+    weights N(0, 0.02) and quantises them (``rtn_quantize``).  The matrices are
+    generated on parallel host threads, each from its own seeded stream.
     """
     bits = np.asarray(bits, dtype=np.int8)
     assert bits.shape == (E,)
@@ -173,17 +218,21 @@ def make_layer(T, H, F, E, group, bits, seed, *, gate_std=0.02, mu=0.0,
     gate = f32_to_bf16_bits(gr)
     codes, scale, zero = [], [], []
     if experts:
+        def one(em):
+            e, m = em
+            rows, cols = (F, H) if m < 2 else (H, F)
+            if quant == "rtn" and int(bits[e]) != 16:
+                return rtn_quantize(expert_weights_f32(seed, e, m, rows, cols), int(bits[e]), group)
+            if quant not in ("direct", "rtn"):
+                raise ValueError(quant)
+            return expert_matrix(seed, e, m, rows, cols, group, int(bits[e]), zero_mode)
+        jobs = [(e, m) for e in range(E) for m in range(3)]
+        with cf.ThreadPoolExecutor(max(1, min(len(jobs), 8, os.cpu_count() or 1))) as ex:
+            mats = list(ex.map(one, jobs))
         for e in range(E):
-            ce, se, ze = [], [], []
-            for m in range(3):
-                rows, cols = (F, H) if m < 2 else (H, F)
-                c_, s_, z_ = expert_matrix(seed, e, m, rows, cols, group, int(bits[e]), zero_mode)
-                ce.append(c_)
-                se.append(s_)
-                ze.append(z_)
-            codes.append(ce)
-            scale.append(se)
-            zero.append(ze)
+            codes.append([mats[3 * e + m][0] for m in range(3)])
+            scale.append([mats[3 * e + m][1] for m in range(3)])
+            zero.append([mats[3 * e + m][2] for m in range(3)])
     protect = None
     if protect_frac > 0:
         r = _rng(seed, 4)
@@ -219,16 +268,18 @@ def dense_expert_weights(seed, e, H, F, std=0.02):
 
 def config_tiny(seed=1235):
     """Tiny single layer: H 256, F 512, 8 experts, 64 tokens, group 64,
-    bits [3,2,2,1,3,2,2,3], mu 0.3, 25% of tokens protected."""
+    bits [3,2,2,1,3,2,2,3], mu 0.3, 25% of tokens protected; expert weights
+    N(0, 0.02) quantised by ``rtn_quantize``."""
     return make_layer(64, 256, 512, 8, 64, [3, 2, 2, 1, 3, 2, 2, 3], seed,
-                      mu=0.3, protect_frac=0.25)
+                      mu=0.3, protect_frac=0.25, quant="rtn")
 
 
 def config_decode(T=16, seed=1236, bits_total=20):
     """Mixtral-8x7b-shaped decode layer: H 4096, F 14336, 8 experts, group 128,
-    bits from {1,2,3} with sum 20 (mean 2.5, nearest feasible to 2.54), ODP off."""
+    bits from {1,2,3} with sum 20 (mean 2.5, nearest feasible to 2.54), ODP off;
+    expert weights N(0, 0.02) quantised by ``rtn_quantize``."""
     bits = bit_table(seed, 8, bits_total)
-    return make_layer(T, MIXTRAL_H, MIXTRAL_F, MIXTRAL_E, 128, bits, seed)
+    return make_layer(T, MIXTRAL_H, MIXTRAL_F, MIXTRAL_E, 128, bits, seed, quant="rtn")
 
 
 def importance_protect(x_bits, frac, seed):
@@ -266,9 +317,10 @@ def config_odp(T=256, seed=1238, bits_total=20, protect_frac=0.10):
     """Mixtral-8x7b-shaped layer for ODP: 256 tokens, 10% protected by the
     importance surrogate, bits with sum 20 / 16 / 13 (mean 2.5 / 2.0 / 1.6).  The
     prune threshold mu is set by the caller from the layer's own routing (the
-    value that prunes ~15% of the unprotected tokens' secondary experts)."""
+    value that prunes ~15% of the unprotected tokens' secondary experts); expert
+    weights N(0, 0.02) quantised by ``rtn_quantize``."""
     bits = bit_table(seed, 8, bits_total)
-    L = make_layer(T, MIXTRAL_H, MIXTRAL_F, MIXTRAL_E, 128, bits, seed)
+    L = make_layer(T, MIXTRAL_H, MIXTRAL_F, MIXTRAL_E, 128, bits, seed, quant="rtn")
     L.protect = importance_protect(L.x, protect_frac, seed)
     return L
 
@@ -302,9 +354,10 @@ def config_decode_22b(T=16, seed=1241, bits_total=20):
 
 
 def config_prefill(T=4096, seed=1237, bits_total=20, skew=(3.0, 0.9)):
-    """Mixtral-8x7b-shaped prefill layer with skewed expert loads, ODP off."""
+    """Mixtral-8x7b-shaped prefill layer with skewed expert loads, ODP off; expert
+    weights N(0, 0.02) quantised by ``rtn_quantize``."""
     bits = bit_table(seed, 8, bits_total)
-    return make_layer(T, MIXTRAL_H, MIXTRAL_F, MIXTRAL_E, 128, bits, seed, skew=skew)
+    return make_layer(T, MIXTRAL_H, MIXTRAL_F, MIXTRAL_E, 128, bits, seed, skew=skew, quant="rtn")
 
 
 def causal_attention(nh, L, seed, temp=1.0):
