@@ -1,16 +1,28 @@
 """Benchmark of the MC compressed MoE layer (PMQ mixed-bit experts + ODP routing)
 on GB300.
 
-Default workload: one Mixtral-8x7b-shaped MoE layer in decode -- H 4096, SwiGLU F
-14336, 8 experts, top-2, 16 tokens, group 128, per-expert bits from {1,2,3}
-(sum 20, mean 2.5), ODP off -- the configuration the decode tokens/s metric is
-quoted on.  A step is one mc_moe_forward (gate, top-2, ODP, permutation, W1|W3
-GEMV + SwiGLU, W2 GEMV, combine) on resident device inputs.  Packed weights
-rotate over several device copies so that no step finds its weights in L2.
+Default run: the headline line is one Mixtral-8x7b-shaped MoE layer in decode --
+H 4096, SwiGLU F 14336, 8 experts, top-2, 16 tokens, group 128, per-expert bits
+from {1,2,3} (sum 20, mean 2.5), ODP off -- the configuration the decode
+tokens/s metric is quoted on; the same JSON line carries, under "workloads", the
+other configurations measured the same way: the prefill layer (4096 tokens,
+skewed expert loads), the ODP layer (256 tokens, 15% of secondaries pruned, 10%
+protected) at bit sums 20 / 16 / 13, and the 32-layer stack at 32 tokens.  A
+step is one pass of the whole layer (gate, top-2, ODP, permutation, W1|W3 +
+SwiGLU, W2, combine; the stack: 32 of them with RMSNorm and residual adds) as a
+CUDA graph replay on resident device inputs.  Packed weights rotate over several
+device copies so that no step finds its weights in L2.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W]
-                  [--workload decode16|decode1|decode4|decode16_8x22b|decode16_fp16|prefill4096|
-                              odp256|odp256_b16|odp256_b13|odp256_drop|odp256_mask|stack32]
+Timing: each workload replays K steps between CUDA events on the launching
+stream, synchronised on both sides, in rounds until at least a second of timed
+load has passed (so that the nvidia-smi sampler, started and read before the
+first round, sees the GPU under load); the reported K-step time is the median
+round.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+      NAME: all (default: decode16 + the sub-records above) or one of
+            decode16 decode1 decode4 decode16_8x22b decode16_fp16 prefill4096
+            odp256 odp256_b16 odp256_b13 odp256_drop odp256_mask stack32
   python bench.py --impl reference ...   (the CPU oracle on the host cores)
 
 Under torchrun every rank runs an independent replica (the layer does not need a
@@ -42,6 +54,10 @@ WORKLOADS = {"decode16": ("decode", 16), "decode4": ("decode", 4), "decode1": ("
              "odp256": ("odp", 256), "odp256_b16": ("odp", 256), "odp256_b13": ("odp", 256),
              "odp256_drop": ("odp", 256), "odp256_mask": ("odp", 256),
              "stack32": ("stack", 32)}
+# the default run: the headline workload, then the sub-records of the same line
+HEADLINE = "decode16"
+SUB_RECORDS = ("prefill4096", "odp256", "odp256_b16", "odp256_b13", "stack32")
+NO_CPU_BASELINE = {"odp256_b16": "odp256", "odp256_b13": "odp256"}  # same layer shape and routing
 STACK_LAYERS = 32
 ODP_BITS = {"odp256": 20, "odp256_b16": 16, "odp256_b13": 13, "odp256_drop": 20, "odp256_mask": 20}
 ODP_DROP = {"odp256_drop": 0.02}  # fraction of tokens whose experts are all masked (Sec. 3.2, Fig. 9)
@@ -49,36 +65,75 @@ ODP_DROP = {"odp256_drop": 0.02}  # fraction of tokens whose experts are all mas
 # heads of the synthetic causal attention, fraction of tokens protected
 MASK_HEADS, MASK_PROTECT = 32, 0.02
 ODP_PRUNE = 0.15  # fraction of unprotected tokens whose secondary expert the threshold drops
+MIN_TIMED_S = 1.0  # timed load per workload (rounds of K steps)
+CPU_BUDGET_S = 8.0  # host-core seconds of oracle work per workload's CPU baseline
 
 
 def _peaks():
+    """(HBM GB/s, bf16 TFLOP/s burst, bf16 TFLOP/s sustained, source)."""
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
             d = json.load(f)
-        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), "measured"
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), float(d["bf16_tflops_sustained"]), "measured"
     except Exception:
-        return 6800.0, 1900.0, "fallback"
+        return 6800.0, 1900.0, 1700.0, "fallback"
 
 
 class Clocks:
-    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+    """nvidia-smi sampling of SM clocks and throttle reasons, read by a thread as
+    the rows arrive (each row carries its own timestamp)."""
 
     Q = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap,utilization.gpu")
+    NAMES = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
 
     def __init__(self, index):
         self.index = index
         self.proc = None
-        self.out = None
+        self.rows = []
+        self.lock = threading.Lock()
+        self.thread = None
 
-    def start(self):
+    def _parse(self, line):
+        f = [x.strip() for x in line.split(",")]
+        if len(f) < 11:
+            return None
+        try:
+            ts = time.mktime(time.strptime(f[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+            ts += float("0." + f[0].split(".")[1]) if "." in f[0] else 0.0
+            util = float(f[10]) if f[10] not in ("[N/A]", "") else None
+            return (ts, float(f[2]), float(f[3]), [n for n, v in zip(self.NAMES, f[6:10])
+                                                   if v.lower().startswith("active")], util)
+        except (ValueError, IndexError):
+            return None
+
+    def _reader(self):
+        for line in self.proc.stdout:
+            r = self._parse(line)
+            if r is not None:
+                with self.lock:
+                    self.rows.append(r)
+
+    def start(self, wait_s=5.0):
+        """Start the sampler and return once its first row has arrived (or after
+        wait_s seconds)."""
         try:
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.Q,
                                           "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except Exception:
             self.proc = None
+            return False
+        self.thread = threading.Thread(target=self._reader, daemon=True)
+        self.thread.start()
+        t0 = time.time()
+        while time.time() - t0 < wait_s:
+            with self.lock:
+                if self.rows:
+                    return True
+            time.sleep(0.02)
+        return False
 
     def stop(self, window=None):
         """Median SM clock and the throttle reasons seen; samples restricted to
@@ -87,33 +142,24 @@ class Clocks:
             return None
         self.proc.terminate()
         try:
-            out, _ = self.proc.communicate(timeout=5)
+            self.proc.wait(timeout=5)
         except Exception:
             self.proc.kill()
-            out, _ = self.proc.communicate()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        rows = []
-        for line in out.strip().splitlines():
-            f = [x.strip() for x in line.split(",")]
-            if len(f) < 10:
-                continue
-            try:
-                ts = time.mktime(time.strptime(f[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
-                ts += float("0." + f[0].split(".")[1]) if "." in f[0] else 0.0
-                rows.append((ts, float(f[2]), float(f[3]), [n for n, v in zip(names, f[6:10])
-                                                            if v.lower().startswith("active")]))
-            except (ValueError, IndexError):
-                continue
+        if self.thread is not None:
+            self.thread.join(timeout=5)
+        with self.lock:
+            rows = list(self.rows)
         if not rows:
             return None
         where = "run"
         if window is not None:
-            inside = [r for r in rows if window[0] - 0.05 <= r[0] <= window[1] + 0.05]
+            inside = [r for r in rows if window[0] <= r[0] <= window[1]]
             if inside:
                 rows, where = inside, "timed region"
         reasons = sorted({n for r in rows for n in r[3]})
+        loaded = [r for r in rows if r[4] is not None and r[4] > 0]
         return {"sm_mhz": statistics.median(r[1] for r in rows), "sm_max_mhz": max(r[2] for r in rows),
-                "samples": len(rows), "window": where, "reasons": reasons}
+                "samples": len(rows), "samples_under_load": len(loaded), "window": where, "reasons": reasons}
 
 
 def _dist():
@@ -138,6 +184,36 @@ def job_throughput(world, units_per_rank, steps, ms):
     """Whole-job units per second: every rank processes units_per_rank per step;
     the job takes the slowest rank's `ms` for `steps` steps."""
     return world * units_per_rank * steps / (ms * 1e-3)
+
+
+def _timed_rounds(torch, replay, steps, stream, world, min_s=MIN_TIMED_S, max_rounds=5000):
+    """Rounds of exactly `steps` replays between CUDA events on `stream`,
+    synchronised (and, with several ranks, barriered) on both sides, repeated
+    until at least min_s seconds of rounds have passed.  Returns (median round
+    ms, every round's ms, (wall t0, wall t1))."""
+    import torch.distributed as dist
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    rounds = []
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    w0 = time.time()
+    i = 0
+    while True:
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(steps):
+            replay(i)
+            i += 1
+        e1.record(stream)
+        torch.cuda.synchronize()
+        rounds.append(e0.elapsed_time(e1))
+        if len(rounds) >= max_rounds or (len(rounds) >= 3 and time.time() - w0 >= min_s):
+            break
+    if world > 1:
+        dist.barrier()
+    w1 = time.time()
+    return statistics.median(rounds), rounds, (w0, w1)
 
 
 def _e2e_pipelined(torch, step, nsets, x, y, steps, stream):
@@ -194,6 +270,7 @@ def _e2e_pipelined(torch, step, nsets, x, y, steps, stream):
     stream.wait_stream(copy)
     e3.record(stream)
     torch.cuda.synchronize()
+    del graphs
     return e2.elapsed_time(e3)
 
 
@@ -217,7 +294,7 @@ def _oracle_mats(oracle, L):
     return [[one(e, m) for m in range(3)] for e in range(L.E)]
 
 
-def cpu_baseline(L, budget_s=12.0, threads=None):
+def cpu_baseline(L, budget_s=CPU_BUDGET_S, threads=None):
     """Time the oracle, as it stands, on a bounded sample of the workload's tokens
     (one token per host thread)."""
     import concurrent.futures as cf
@@ -247,56 +324,72 @@ def cpu_baseline(L, budget_s=12.0, threads=None):
                           n, L.T, "; plus the Eq. 6 mask of all tokens, charged n/T of its time" if t_mask else "")}
 
 
-def cpu_baseline_stack(L, gates, mus, budget_s=12.0, threads=None):
-    """The oracle's 32-layer stack on a bounded sample of the workload's tokens
-    (one token's whole trajectory per host thread)."""
+def _oracle_stack_mus(L, gates, mats, nl, threads=None):
+    """Per-layer thresholds of the first nl layers along the oracle's own
+    trajectory (untimed calibration of the reference arm): at each layer, the
+    ODP_PRUNE quantile of w1/w0 over the unprotected tokens' routing at mu = 0,
+    then every token through that layer with it (one token per thread)."""
+    import concurrent.futures as cf
+
+    import oracle
+    gf = [synth.bf16_bits_to_f32(g) for g in gates]
+    h = L.x_f32().astype(np.float64)
+    mus = []
+    for l in range(nl):
+        xn = oracle.bf16_round(np.stack([oracle.rmsnorm(h[t], np.ones(L.H, np.float32), 1e-5) for t in range(L.T)]))
+        _, w, _ = oracle.route(xn, gf[l], 0.0, L.protect)
+        ratio = w[:, 1].astype(np.float64) / w[:, 0]
+        mus.append(float(np.quantile(ratio[L.protect == 0], ODP_PRUNE)))
+        one = lambda t: oracle.stack(h[t:t + 1], [gf[l]], mats, [mus[-1]], L.protect[t:t + 1])[0][0]
+        with cf.ThreadPoolExecutor(threads or os.cpu_count() or 1) as ex:
+            h = np.stack(list(ex.map(one, range(L.T))))
+    return mus
+
+
+def cpu_baseline_stack(L, gates, mus=None, budget_s=CPU_BUDGET_S, threads=None):
+    """The oracle's stack on a bounded sample of the workload: one token per host
+    thread through the first `nl` of the stack's layers (nl sized to the budget;
+    every layer has the same shape), scaled to whole-stack tokens/s by nl / layers.
+    mus: the per-layer thresholds (None: calibrated along the oracle's own
+    trajectory for the layers it runs, untimed)."""
     import concurrent.futures as cf
 
     import oracle
     mats = _oracle_mats(oracle, L)
     gf = [synth.bf16_bits_to_f32(g) for g in gates]
     xf = L.x_f32()
-    run = lambda t: oracle.stack(xf[t:t + 1], gf, mats, mus, L.protect[t:t + 1])
+    layers = len(gates)
     cores = threads or (os.cpu_count() or 1)
     t0 = time.perf_counter()
-    run(0)
-    one = time.perf_counter() - t0
-    n = int(max(1, min(L.T, cores, round(budget_s / max(one, 1e-3) * cores / 2))))
+    oracle.stack(xf[:1], gf[:1], mats, [0.0], L.protect[:1])
+    one = time.perf_counter() - t0  # one token, one layer
+    n = int(max(1, min(L.T, cores)))
+    nl = int(max(1, min(layers, round(budget_s / max(one, 1e-3) / 2))))
+    if mus is None:  # calibrated once per workload object
+        mus = getattr(L, "oracle_mus", None)
+        if mus is None or len(mus) < nl:
+            mus = L.oracle_mus = _oracle_stack_mus(L, gates, mats, nl, threads)
+    run = lambda t: oracle.stack(xf[t:t + 1], gf[:nl], mats, list(mus[:nl]), L.protect[t:t + 1])
     t0 = time.perf_counter()
-    with cf.ThreadPoolExecutor(min(n, cores)) as ex:
+    with cf.ThreadPoolExecutor(n) as ex:
         list(ex.map(run, range(n)))
     dt = time.perf_counter() - t0
-    return {"value": n / dt, "unit": "tokens/s", "cores": min(n, cores), "kind": "oracle",
-            "single_thread_value": 1.0 / one,
-            "sample": "%d of the workload's %d tokens (all %d layers per token, fp64, one token per thread); "
-                      "single_thread_value: token 0 alone on one thread" % (n, L.T, len(gates))}
-
-
-def _stack_mus_oracle(L, gates):
-    """Per-layer thresholds from the oracle's own trajectory at mu = 0 (the
-    reference arm's counterpart of the calibration in run_stack)."""
-    import oracle
-    mats = _oracle_mats(oracle, L)
-    gf = [synth.bf16_bits_to_f32(g) for g in gates]
-    xf = L.x_f32()
-    mus = []
-    sample = list(range(min(L.T, 8)))
-    _, routes = oracle.stack(xf[sample], gf, mats, [0.0] * len(gates), L.protect[sample])
-    for (idx, w, pr, xn) in routes:
-        ratio = w[:, 1].astype(np.float64) / w[:, 0]
-        free = ratio[L.protect[sample] == 0]
-        mus.append(float(np.quantile(free if free.size else ratio, ODP_PRUNE)))
-    return mus
+    return {"value": n * nl / layers / dt, "unit": "tokens/s", "cores": n, "kind": "oracle",
+            "single_thread_value": 1.0 / (one * layers),
+            "sample": "%d of the workload's %d tokens, one token per thread through the first %d of its %d layers "
+                      "(fp64), scaled by %d/%d to whole-stack tokens/s; single_thread_value: token 0 through one "
+                      "layer alone on one thread, times %d" % (n, L.T, nl, layers, nl, layers, layers)}
 
 
 def run_reference(args):
     world, rank, _ = _dist()
     if rank != 0:
         return 0
-    kind, T, L = _workload(args.workload)
+    name = HEADLINE if args.workload == "all" else args.workload
+    kind, T, L = _workload(name)
     if kind == "stack":
         L, gates = L
-        mus = _stack_mus_oracle(L, gates)
+        mus = None  # calibrated along the oracle's own trajectory
     if kind == "odp":
         import oracle
         if name_has_mask(L):
@@ -434,18 +527,19 @@ def _graph_profile(mc, torch, step, nsets, kernels, rounds):
     return {name: (ms / max(n, 1), n / (rounds * nsets)) for name, (ms, n) in tot.items()}
 
 
-def run(args):
-    import torch
-    import torch.distributed as dist
+def _clock_note(cl):
+    if cl is None:
+        return None
+    cl = dict(cl)
+    cl["note"] = "nvidia-smi -lms 50 rows read as they arrive; sampler started (first row received) before the " \
+                 "first timed round; rows restricted to the timed rounds' wall-clock window"
+    return cl
 
-    import paper_2410_06270_gb300 as mc
 
-    world, rank, local = _dist()
-    torch.cuda.set_device(local)
-    if world > 1:
-        dist.init_process_group("nccl")
-    dev = torch.device("cuda", local)
-    kind, T, L = _workload(args.workload)
+def measure_layer(name, args, torch, mc, dev, local, world, cpu=True):
+    """One single-layer workload.  Returns the JSON record (the slowest rank's
+    times; value = whole-job tokens/s)."""
+    kind, T, L = _workload(name)
     steps = args.steps if args.steps else {"decode": 2000, "odp": 1000, "prefill": 100}[kind]
     shape = mc.Shape(L.E, L.H, L.F, L.group)
     flat = lambda a: [a[e][m] for e in range(L.E) for m in range(3)]
@@ -456,7 +550,7 @@ def run(args):
     x = torch.from_numpy(L.x.view(np.int16).copy()).view(torch.bfloat16).to(dev)
     gw = torch.from_numpy(L.gate.view(np.int16).copy()).view(torch.bfloat16).to(dev)
     prot = None if L.protect is None else torch.from_numpy(L.protect.copy()).to(dev)
-    attn = imp = None
+    attn = imp = iws = None
     if name_has_mask(L):
         # the protect mask comes from the step itself (Eq. 6 on the attention map)
         attn = torch.from_numpy(L.attn).to(dev)
@@ -482,15 +576,15 @@ def run(args):
     _, r = mc.moe_forward(x, gw, shape, L.bits, packed[0], mu, prot, y=y, workspace=ws, routing=True)
     mc.check_status(ws)
     idx = r["idx"].cpu().numpy()
-    pairs = int(2 * T - int(r["pruned"].sum().item()))
-    touched = sorted(set(idx.reshape(-1).tolist()))
+    pr = r["pruned"].cpu().numpy()
+    pairs = int(2 * T - int(np.minimum(pr, 1).sum()) - int((pr == 2).sum()))
+    keep = np.stack([pr != 2, pr == 0], axis=1)
+    touched = sorted(set(idx[keep].reshape(-1).tolist()))
     alg_bytes, w13_bytes = _algorithmic_bytes(shape, L.bits, touched, T, L.H)
     w13_flops = 4.0 * L.H * L.F * pairs          # W1 and W3: 2 x (2 H F) per kept pair
     layer_flops = 6.0 * L.H * L.F * pairs + 2.0 * L.H * L.E * T
     rk = "gemv_w13" if 2 * T < 240 else "gemm_w13"  # the path mc_moe_forward picks (kPrefillPairs)
 
-    clocks = Clocks(local)
-    clocks.start()
     for i in range(args.warmup):
         step(i)
     torch.cuda.synchronize()
@@ -508,64 +602,54 @@ def run(args):
     for i in range(args.warmup):
         graphs[i % nsets].replay()
     torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
-    # timed region: K graph replays
     stream = torch.cuda.current_stream()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    torch.cuda.synchronize()
-    t_wall0 = time.time()
-    e0.record(stream)
-    for i in range(steps):
-        graphs[i % nsets].replay()
-    e1.record(stream)
-    torch.cuda.synchronize()
-    t_wall1 = time.time()
-    ms = e0.elapsed_time(e1)
+    clocks = Clocks(local)
+    clocks.start()
+    ms, rounds, window = _timed_rounds(torch, lambda i: graphs[i % nsets].replay(), steps, stream, world)
+    cl = clocks.stop(window)
     mc.check_status(ws)
-    cl = clocks.stop((t_wall0, t_wall1))
     # the roofline kernel's launch duration: CUDA events around that kernel only,
     # captured as event nodes of a profiling copy of the step graphs (events inside
     # the timed graphs would serialise the launches they bracket); then the
     # per-kernel breakdown from a second profiling copy with every kernel bracketed
-    prof = _graph_profile(mc, torch, step, nsets, [rk], rounds=min(steps, 200))
-    breakdown = _graph_profile(mc, torch, step, nsets, None, rounds=min(steps, 50))
+    prof = _graph_profile(mc, torch, step, nsets, [rk], rounds=max(3, min(steps, 200)))
+    breakdown = _graph_profile(mc, torch, step, nsets, None, rounds=max(3, min(steps, 50)))
     ms_e2e = _e2e_pipelined(torch, step, nsets, x, y, steps, stream)
+    ms, ms_e2e, avg = max_over_ranks([ms, ms_e2e, prof.get(rk, (0.0, 0))[0]], dev)
+    del graphs
 
-    ms, ms_e2e = max_over_ranks([ms, ms_e2e], dev)
-    if world > 1:
-        dist.barrier()
-    if rank != 0:
-        if world > 1:
-            dist.destroy_process_group()
-        return 0
-
-    hbm, bf16, src = _peaks()
-    avg = prof.get(rk, (0.0, 0))[0]
+    hbm, bf16, bf16_sus, src = _peaks()
     value = job_throughput(world, T, steps, ms)
     e2e = job_throughput(world, T, steps, ms_e2e)
+    layer_s = ms * 1e-3 / steps
+    layer_gbs = alg_bytes / layer_s / 1e9
+    layer_tf = layer_flops / layer_s / 1e12
+    t_hbm, t_tc = alg_bytes / (hbm * 1e9), layer_flops / (bf16 * 1e12)
+    layer_roof = {"bytes": alg_bytes, "flops": layer_flops, "hbm_bound_us": t_hbm * 1e6, "tensor_bound_us": t_tc * 1e6,
+                  "binding": "hbm" if t_hbm >= t_tc else "tensor", "measured_us": layer_s * 1e6,
+                  "frac": max(t_hbm, t_tc) / layer_s, "gbs": layer_gbs, "hbm_frac": layer_gbs / hbm,
+                  "tflops": layer_tf, "tensor_frac_burst": layer_tf / bf16,
+                  "note": "whole-step roofline: max(algorithmic bytes / measured HBM peak, algorithmic flops / "
+                          "measured bf16 burst peak) / measured step time"}
     if rk == "gemv_w13":
         achieved = w13_bytes / (avg * 1e-3) / 1e9 if avg > 0 else None
-        layer_gbs = alg_bytes * steps / (ms * 1e-3) / 1e9
         roof = {"bound": "hbm", "kernel": rk, "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                "frac": (achieved / hbm) if achieved else None, "traffic": _traffic(rk, args.workload),
+                "frac": (achieved / hbm) if achieved else None, "traffic": _traffic(rk, name),
                 "peak_source": "%s (MEASURED_PEAKS.json hbm_gbs)" % src if src == "measured" else src,
                 "frac_of_nominal_7900": (achieved / HBM_NOMINAL_GBS) if achieved else None,
-                "algorithmic_bytes_per_launch": w13_bytes, "layer_gbs": layer_gbs, "layer_frac": layer_gbs / hbm}
+                "algorithmic_bytes_per_launch": w13_bytes, "kernel_us": avg * 1e3,
+                "layer_gbs": layer_gbs, "layer_frac": layer_gbs / hbm}
     else:
-        sustained = _peak_sustained() or bf16
         achieved = w13_flops / (avg * 1e-3) / 1e12 if avg > 0 else None
-        layer_tf = layer_flops * steps / (ms * 1e-3) / 1e12
-        roof = {"bound": "tensor", "kernel": rk, "achieved": achieved, "peak": sustained, "unit": "TFLOP/s",
-                "frac": (achieved / sustained) if achieved else None, "traffic": _traffic(rk, args.workload),
-                "peak_source": "%s (MEASURED_PEAKS.json bf16_tflops_sustained; fp16 has the bf16 rate)" % src
-                               if src == "measured" else src,
-                "frac_of_burst_peak": (achieved / bf16) if achieved else None,
-                "algorithmic_flops_per_launch": w13_flops, "layer_tflops": layer_tf,
-                "layer_frac": layer_tf / sustained, "kept_pairs": pairs,
-                "layer_gbs": alg_bytes * steps / (ms * 1e-3) / 1e9,
-                "layer_hbm_frac": alg_bytes * steps / (ms * 1e-3) / 1e9 / hbm}
-    line = {
+        roof = {"bound": "tensor", "kernel": rk, "achieved": achieved, "peak": bf16, "unit": "TFLOP/s",
+                "frac": (achieved / bf16) if achieved else None, "traffic": _traffic(rk, name),
+                "peak_source": "%s (MEASURED_PEAKS.json bf16_tflops: the burst peak, the kernel runs for "
+                               "milliseconds at most; fp16 has the bf16 rate)" % src if src == "measured" else src,
+                "peak_sustained": bf16_sus, "frac_of_sustained": (achieved / bf16_sus) if achieved else None,
+                "algorithmic_flops_per_launch": w13_flops, "kernel_us": avg * 1e3, "kept_pairs": pairs,
+                "layer_tflops": layer_tf, "layer_frac": layer_tf / bf16,
+                "layer_gbs": layer_gbs, "layer_hbm_frac": layer_gbs / hbm}
+    rec = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": steps,
         "warmup": args.warmup, "ms_per_step": ms / steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "data": "synthetic",
@@ -575,41 +659,36 @@ def run(args):
                    "global_batch": T * world, "parallelism": "replicas" if world > 1 else "single",
                    "l2": "inputs larger than L2: %d rotating copies of the %.0f MB packed weights"
                          % (nsets, packed_host.nbytes / 1e6),
-                   "touched_experts": len(touched)},
+                   "touched_experts": len(touched), "kept_pairs": pairs},
         "roofline": roof,
+        "layer_roofline": layer_roof,
+        "timing": {"rounds": len(rounds), "round_ms_median": ms, "round_ms_min": min(rounds),
+                   "round_ms_max": max(rounds), "timed_s": window[1] - window[0],
+                   "how": "rounds of exactly K CUDA graph replays between CUDA events on the launching stream, "
+                          "synchronised on both sides, until >= %.1f s; median round reported" % MIN_TIMED_S},
         "kernels_ms_per_step": {k: v[0] * v[1] for k, v in breakdown.items()},
-        "launch": "timed region = K replays of a CUDA graph of the step; roofline duration = mean of CUDA "
-                  "events around the kernel, captured as event nodes in profiling copies of the step graphs "
-                  "(%d replays)" % (nsets * min(steps, 200)),
+        "launch": "roofline kernel duration = mean of CUDA events around that kernel, captured as event nodes in "
+                  "profiling copies of the step graphs (%d replays); kernels_ms_per_step from copies with every "
+                  "kernel bracketed (each event node between two kernels removes their programmatic launch "
+                  "overlap, so the sum exceeds ms_per_step)" % (nsets * max(3, min(steps, 200))),
         "e2e": {"value": e2e, "unit": "tokens/s", "h2d_bytes_per_step": int(x.numel() * 2),
                 "d2h_bytes_per_step": int(y.numel() * 2),
                 "copies": "cudaMemcpyAsync from / to pinned host buffers every step, on a copy stream, two "
                           "device buffer pairs: step i+1's input and step i's output move while step i runs"},
         "gpu_launches": int(round(sum(n for _, n in breakdown.values()))) * steps,
-        "clocks": cl,
+        "clocks": _clock_note(cl),
     }
-    if not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(L)
-    print(json.dumps(line), flush=True)
-    if world > 1:
-        dist.destroy_process_group()
-    return 0
+    if cpu and not args.no_cpu_baseline:
+        rec["cpu_baseline"] = cpu_baseline(L)
+    del packed, ws, x, y
+    torch.cuda.empty_cache()
+    return rec
 
 
-def run_stack(args):
+def measure_stack(name, args, torch, mc, dev, local, world, cpu=True):
     """The 32-layer stack: one mc_stack_forward captured into a CUDA graph (with the
-    copy of the step's input into the residual stream), replayed K times."""
-    import torch
-    import torch.distributed as dist
-
-    import paper_2410_06270_gb300 as mc
-
-    world, rank, local = _dist()
-    torch.cuda.set_device(local)
-    if world > 1:
-        dist.init_process_group("nccl")
-    dev = torch.device("cuda", local)
-    kind, T, (L, gates) = _workload(args.workload)
+    copy of the step's input into the residual stream), replayed."""
+    kind, T, (L, gates) = _workload(name)
     layers = len(gates)
     steps = args.steps if args.steps else 100
     shape = mc.Shape(L.E, L.H, L.F, L.group)
@@ -622,7 +701,7 @@ def run_stack(args):
     prot = torch.from_numpy(L.protect.copy()).to(dev)
     gamma = torch.ones((layers, L.H), dtype=torch.bfloat16, device=dev)
     # per-layer thresholds from this layer's own routing along the stack's trajectory at mu = 0
-    mus, touched = [], []
+    mus, touched, pairs = [], [], 0
     h = x0.clone()
     wsl = mc.alloc_workspace(shape, T, dev)
     for l in range(layers):
@@ -631,9 +710,13 @@ def run_stack(args):
         w = r["w"].cpu().numpy().astype(np.float64)
         mus.append(float(np.quantile((w[:, 1] / w[:, 0])[L.protect == 0], ODP_PRUNE)))
         y, rr = mc.moe_forward(xn, gw[l], shape, L.bits, packs[l], mus[-1], prot, workspace=wsl, routing=True)
-        touched.append(sorted(set(rr["idx"].cpu().numpy().reshape(-1).tolist())))
+        pr = rr["pruned"].cpu().numpy()
+        keep = np.stack([pr != 2, pr == 0], axis=1)
+        touched.append(sorted(set(rr["idx"].cpu().numpy()[keep].reshape(-1).tolist())))
+        pairs += int(keep.sum())
         h = mc.add(h, y)
     mc.check_status(wsl)
+    del wsl
     args_s = mc.StackArgs(gw, [L.bits] * layers, packs, mus)
     ws = mc.stack_workspace(shape, T, dev)
     hs = x0.clone()
@@ -648,26 +731,17 @@ def run_stack(args):
             mc.stack_forward(hs, shape, args_s, gamma, ws, prot)
     torch.cuda.current_stream().wait_stream(cs)
     alg = sum(_algorithmic_bytes(shape, L.bits, t, T, L.H)[0] for t in touched)
+    flops = 6.0 * L.H * L.F * pairs + 2.0 * L.H * L.E * T * layers
 
-    clocks = Clocks(local)
-    clocks.start()
     for _ in range(args.warmup):
         graph.replay()
     torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
     stream = torch.cuda.current_stream()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    t_wall0 = time.time()
-    e0.record(stream)
-    for _ in range(steps):
-        graph.replay()
-    e1.record(stream)
-    torch.cuda.synchronize()
-    t_wall1 = time.time()
-    ms = e0.elapsed_time(e1)
+    clocks = Clocks(local)
+    clocks.start()
+    ms, rounds, window = _timed_rounds(torch, lambda i: graph.replay(), steps, stream, world)
+    cl = clocks.stop(window)
     mc.check_status(ws)
-    cl = clocks.stop((t_wall0, t_wall1))
     # per-kernel breakdown: one eager profiled call
     mc.profile_select(None)
     mc.profile_enable(True)
@@ -690,15 +764,11 @@ def run_stack(args):
     torch.cuda.synchronize()
     ms_e2e = e2.elapsed_time(e3)
     ms, ms_e2e = max_over_ranks([ms, ms_e2e], dev)
-    if world > 1:
-        dist.barrier()
-    if rank != 0:
-        if world > 1:
-            dist.destroy_process_group()
-        return 0
-    hbm, _, src = _peaks()
-    gbs = alg * steps / (ms * 1e-3) / 1e9
-    line = {
+    del graph
+    hbm, bf16, _, src = _peaks()
+    step_s = ms * 1e-3 / steps
+    gbs = alg / step_s / 1e9
+    rec = {
         "metric": METRIC, "value": job_throughput(world, T, steps, ms), "unit": "tokens/s", "n_gpus": world,
         "steps": steps, "warmup": args.warmup, "ms_per_step": ms / steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f16 x {1,2,3}-bit codes, fp32 accumulate",
@@ -707,55 +777,89 @@ def run_stack(args):
                    "parallelism": "replicas" if world > 1 else "single",
                    "l2": "inputs larger than L2: %d layers x %.0f MB packed weights, one device copy per layer"
                          % (layers, packed_host.nbytes / 1e6),
-                   "weights": "one seeded expert set shared by the layers (separate copies), per-layer gates"},
+                   "weights": "one seeded expert set shared by the layers (separate copies), per-layer gates",
+                   "kept_pairs": pairs},
         "roofline": {"bound": "hbm", "kernel": "stack step (CUDA graph: %d layers of rmsnorm, route, permute, "
                                                 "GEMV W1|W3, GEMV W2, combine, add)" % layers,
                      "achieved": gbs, "peak": hbm, "unit": "GB/s", "frac": gbs / hbm, "traffic": None,
                      "frac_of_nominal_7900": gbs / HBM_NOMINAL_GBS,
                      "peak_source": "%s (MEASURED_PEAKS.json hbm_gbs)" % src if src == "measured" else src,
-                     "algorithmic_bytes_per_step": alg},
+                     "algorithmic_bytes_per_step": alg, "tensor_frac_burst": flops / step_s / 1e12 / bf16},
+        "timing": {"rounds": len(rounds), "round_ms_median": ms, "round_ms_min": min(rounds),
+                   "round_ms_max": max(rounds), "timed_s": window[1] - window[0]},
         "kernels_ms_per_step": {k: v[0] for k, v in breakdown.items()},
         "e2e": {"value": job_throughput(world, T, steps, ms_e2e), "unit": "tokens/s",
                 "h2d_bytes_per_step": int(x0.numel() * 2), "d2h_bytes_per_step": int(hs.numel() * 2)},
         # the profiled kernels of one call plus one rmsnorm and one add launch per layer
         "gpu_launches": (_launches_per_step(breakdown, 1) + 2 * layers) * steps,
-        "clocks": cl,
+        "clocks": _clock_note(cl),
     }
-    if not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline_stack(L, gates, mus)
-    print(json.dumps(line), flush=True)
-    if world > 1:
-        dist.destroy_process_group()
-    return 0
+    if cpu and not args.no_cpu_baseline:
+        rec["cpu_baseline"] = cpu_baseline_stack(L, gates, mus)
+    del packs, ws, hs, x0
+    torch.cuda.empty_cache()
+    return rec
 
 
 def _launches_per_step(breakdown, n):
     return int(round(sum(c for _, c in breakdown.values()) / max(n, 1)))
 
 
-def _peak_sustained():
-    try:
-        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
-            return float(json.load(f)["bf16_tflops_sustained"])
-    except Exception:
-        return None
+def _measure(name, args, torch, mc, dev, local, world, cpu=True):
+    fn = measure_stack if WORKLOADS[name][0] == "stack" else measure_layer
+    return fn(name, args, torch, mc, dev, local, world, cpu=cpu)
+
+
+def run(args):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2410_06270_gb300 as mc
+
+    world, rank, local = _dist()
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+    if args.workload == "all":
+        line = _measure(HEADLINE, args, torch, mc, dev, local, world)
+        subs = {}
+        for name in SUB_RECORDS:
+            rec = _measure(name, args, torch, mc, dev, local, world, cpu=name not in NO_CPU_BASELINE)
+            if name in NO_CPU_BASELINE and "cpu_baseline" in subs.get(NO_CPU_BASELINE[name], {}):
+                rec["cpu_baseline"] = dict(subs[NO_CPU_BASELINE[name]]["cpu_baseline"],
+                                           sample="that of %s (same layer shape, routing and oracle work per "
+                                                  "token)" % NO_CPU_BASELINE[name])
+            for k in ("metric", "n_gpus", "steps", "warmup", "higher_is_better", "scaling", "vs_baseline", "data"):
+                rec.pop(k, None)
+            subs[name] = rec
+        line["workloads"] = subs
+        line["gpu_launches_all_workloads"] = line["gpu_launches"] + sum(r["gpu_launches"] for r in subs.values())
+    else:
+        line = _measure(args.workload, args, torch, mc, dev, local, world)
+    if world > 1:
+        dist.barrier()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
 
 
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=0, help="timed steps (default: 2000 decode, 100 prefill)")
+    ap.add_argument("--steps", type=int, default=0, help="timed steps per round (default: 2000 decode, 1000 ODP, "
+                                                         "100 prefill and stack)")
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="mc", choices=["mc", "reference"])
-    ap.add_argument("--workload", default="decode16", choices=sorted(WORKLOADS))
+    ap.add_argument("--workload", default="all", choices=["all"] + sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
     if args.impl == "reference":
         return run_reference(args)
-    if WORKLOADS[args.workload][0] == "stack":
-        return run_stack(args)
     return run(args)
 
 
