@@ -8,22 +8,31 @@
 //   with the columns of every K = 16 slice ordered like the A operand below.
 // gemm_kernel<W13>: persistent, one CTA per SM, warp-specialised:
 //   producer warp      claims items (a token block x a 128-row block of W1|W3,
-//                      or x a 256-row block pair of W2) from an atomic counter and
-//                      streams per 128-column step one ring stage
-//                      [activation image 32 KB][packed weights of both streams]
-//                      with cp.async.bulk;
-//   converter warps (8) turn the packed codes (the decode path's layout) into
-//                      fp16 (q - z) s and store them into tensor memory with
-//                      tcgen05.st 16x256b, whose thread -> (lane, column) order is
-//                      the mma fragment order the packed tiles are stored in;
-//   MMA thread         tcgen05.mma kind::f16, M = 128 rows, N = 128 pairs,
+//                      or x a 256-row block pair of W2)
+//                      from an atomic counter and streams per 128-column step
+//                      one ring stage [activation image][packed weights of both
+//                      streams] with cp.async.bulk (half the image for a block of
+//                      <= 64 pairs: the MMA reads rows 0..63 only);
+//   converter warps    two groups of four, taking alternate stages (ping-pong):
+//                      while one group converts its stage, the other's
+//                      tensor-memory stores and barrier waits proceed.  Each warp
+//                      turns its four 16-row tiles (two row tiles x two streams)
+//                      of packed codes (the decode path's layout) into fp16
+//                      (q - z) s and stores them into the group's A buffer in
+//                      tensor memory with tcgen05.st 16x256b, whose thread ->
+//                      (lane, column) order is the mma fragment order the packed
+//                      tiles are stored in;
+//   MMA warps (2)      one per weight stream: tcgen05.mma kind::f16, M = 128
+//                      rows, N = 128 pairs (64 for a block of <= 64 pairs),
 //                      K = 16, A from tensor memory, B from the image, fp32
-//                      accumulators in tensor memory (one per stream);
+//                      accumulators in tensor memory; a stage is issued once its
+//                      converter group has stored it (the group saw the copies
+//                      land), so the MMA warps wait on one barrier per stage;
 //   epilogue warps 4-7 W13: h = silu(W1 x) * (W3 x) -> fp16 image of W2's input
 //                      (the same image layout, one 128-column step per row block);
 //                      W2: fp32 outputs per pair.
 // Tensor memory (512 columns): accumulators of streams 0/1 at columns 0 / 128,
-// two A buffers of 2 x 64 columns at 256 / 384.
+// the two groups' A buffers of 2 x 64 columns at 256 / 384.
 #include "mc_host.h"
 #include "mc_kernels.h"
 #include "mc_profile.h"
@@ -39,12 +48,14 @@ constexpr int kGSlots = 4;
 constexpr int kGHdr = 1024;
 constexpr int kGStaging = kImgBytes;               // epilogue staging of one h image
 constexpr size_t kGSmem = kGHdr + (size_t)kGSlots * kGStage + kGStaging;
-// warps 0-3 and 8-11 convert (warp w: tensor-memory lanes 32 (w % 4) + 16 (w / 8)
-// .. +15, one 16-row tile per stream), 4-7 run the epilogue, 12 produces, 13 issues MMAs
-constexpr int kGEpi0 = 4, kGProd = 12, kGMma = 13, kGConv = 8;
-constexpr int kGThreads = 14 * 32;
+// warps 0-3 / 8-11: converter groups 0 / 1 (warp w: tensor-memory lanes 32 (w % 4)
+// .. +31, tiles 2 (w % 4) and 2 (w % 4) + 1 of each stream); 4-7 epilogue;
+// 12 producer; 13 / 14 issue the MMAs of stream 0 / 1
+constexpr int kGEpi0 = 4, kGProd = 12, kGMma = 13, kGMmaN = 2, kGConvGroup = 4;
+constexpr int kGThreads = 15 * 32;
 constexpr int kGRuns = kMaxE;
 constexpr int kGItemRing = 8;
+constexpr int kGNarrow = 64;                       // blocks of <= 64 pairs: N = 64 MMAs
 static_assert(kGStage % 1024 == 0, "stage alignment");
 
 // Byte offset of (pair row n, column c of the 128-column step) in an image: two
@@ -62,11 +73,12 @@ __host__ __device__ __forceinline__ uint32_t img_off(int n, int c)
 struct GStage {
     int item, kt, first, last;  // item id, column step, first / last step of the item
     int k, u;                   // token block, unit (row block or row-block pair)
+    int narrow;                 // the block has <= 64 pairs
     ChunkInfo ci;
 };
 
 struct GItem {
-    int k, u;
+    int k, u;  // token block, unit
     ChunkInfo ci;
 };
 
@@ -77,7 +89,7 @@ struct GShared {
     uint32_t tmem_base;
     volatile int abort;
     volatile int issued;
-    volatile int end_items;  // items this CTA's MMA thread completed, set once it saw the end marker
+    volatile int end_items;  // items this CTA's MMA warps completed, set once they saw the end marker
     int nruns;
     int run_first[kGRuns], run_nb[kGRuns], run_base[kGRuns + 1];
     GStage stage[kGSlots];
@@ -225,16 +237,6 @@ __device__ __forceinline__ void convert_regs(const uint8_t *tile, int bits, int 
     else convert_tile<3, GPT>(tile, lane, v);
 }
 
-template <int GPT>
-__device__ __forceinline__ void convert_store(const uint8_t *tile, int bits, int lane, uint32_t taddr)
-{
-    uint32_t v[32];
-    if (bits == 1) convert_tile<1, GPT>(tile, lane, v);
-    else if (bits == 2) convert_tile<2, GPT>(tile, lane, v);
-    else convert_tile<3, GPT>(tile, lane, v);
-    tmem_st_16x256_x8(taddr, v);
-}
-
 // ------------------------------------------------------------- epilogue --
 
 __device__ __forceinline__ void tmem_ld_x16(uint32_t taddr, float (&v)[16])
@@ -271,6 +273,34 @@ __device__ __forceinline__ bool epi_sync(const ExpertParams &p, GShared *sh, int
 
 // ------------------------------------------------------------------ kernel --
 
+// One converter warp, one stage: its four tiles (tiles 2q, 2q+1 of each stream
+// present), dequantised and stored into A buffer `abuf`; the first store waits
+// until the MMAs that last read the buffer are done (need_wait).  False once the
+// CTA aborted.
+template <int GPT>
+__device__ __forceinline__ bool convert_stage(const uint8_t *w, int bits, int nstream, int STB, int TB, int q,
+                                              int lane, uint32_t abuf, bool need_wait, uint64_t *aempty,
+                                              uint32_t parity, const ExpertParams &p, GShared *sh)
+{
+    uint32_t va[32], vb[32];
+    // two register sets alternate, so that a tile's dequantisation overlaps the
+    // previous tile's store
+    convert_regs<GPT>(w + (2 * q) * TB, bits, lane, va);
+    if (need_wait && !g_wait(aempty, parity, p, sh)) return false;
+    tc_fence_after();
+    tmem_st_16x256_x8(abuf + ((uint32_t)(32 * q) << 16), va);
+    convert_regs<GPT>(w + (2 * q + 1) * TB, bits, lane, vb);
+    tmem_st_16x256_x8(abuf + ((uint32_t)(32 * q + 16) << 16), vb);
+    if (nstream > 1) {
+        convert_regs<GPT>(w + STB + (2 * q) * TB, bits, lane, va);
+        tmem_st_16x256_x8(abuf + 64u + ((uint32_t)(32 * q) << 16), va);
+        convert_regs<GPT>(w + STB + (2 * q + 1) * TB, bits, lane, vb);
+        tmem_st_16x256_x8(abuf + 64u + ((uint32_t)(32 * q + 16) << 16), vb);
+    }
+    tmem_st_wait();
+    return true;
+}
+
 template <bool W13, int GPT>
 __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
 {
@@ -281,24 +311,24 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int group = kTileK / GPT;
     const int nrb = W13 ? p.F / kBlockRows : p.H / kBlockRows;
-    const int U = W13 ? nrb : (nrb + 1) / 2;
     const int KTm = W13 ? p.H / kTileK : p.F / kTileK;  // column steps (K)
+    const int U = W13 ? nrb : (nrb + 1) / 2;            // units of a token block: row block (pair)
     const uint8_t *img_base = W13 ? p.ximg : p.himg;
 
     pdl_wait();
     if (threadIdx.x == 0) {
         for (int s = 0; s < kGSlots; ++s) {
             mbar_init(&sh->full[s], 1);
-            mbar_init(&sh->empty[s], 1 + kGConv);  // MMA commit + converter warps
+            mbar_init(&sh->empty[s], kGMmaN + kGConvGroup);  // MMA commits + the stage's converter group
         }
         for (int b = 0; b < 2; ++b) {
-            mbar_init(&sh->afull[b], kGConv);
-            mbar_init(&sh->aempty[b], 1);
+            mbar_init(&sh->afull[b], kGConvGroup);
+            mbar_init(&sh->aempty[b], kGMmaN);
         }
-        mbar_init(&sh->dfull, 1);
+        mbar_init(&sh->dfull, kGMmaN);
         mbar_init(&sh->dempty, 4);
         mbar_init(&sh->esync, 4);
-        mbar_init(&sh->drain, 1);
+        mbar_init(&sh->drain, kGMmaN);
         sh->abort = 0;
         sh->issued = 0;
         sh->end_items = 0x7fffffff;
@@ -360,6 +390,7 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
                 gi.ci = ci;
                 sh->items[nitem % kGItemRing] = gi;
                 ++nitem;
+                const int narrow = ci.nv <= kGNarrow;
                 const int STB = supertile_bytes(bits, group);
                 const int pw = W13 ? 2 : w2_pair_width(u, nrb);
                 const uint8_t *wsrc = p.packed + p.mat_off[e][W13 ? 0 : 2] +
@@ -378,79 +409,91 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
                     st.last = kt == KTm - 1;
                     st.k = k;
                     st.u = u;
+                    st.narrow = narrow;
                     st.ci = ci;
                     uint8_t *dst = ring + (size_t)slot * kGStage;
+                    const uint8_t *src = isrc + (size_t)kt * kImgBytes;
                     const uint32_t wb = (uint32_t)(pw * STB);
-                    mbar_arrive_expect_tx(&sh->full[slot], (uint32_t)kImgBytes + wb);
-                    bulk_g2s(dst, isrc + (size_t)kt * kImgBytes, kImgBytes, &sh->full[slot]);
+                    if (narrow) {
+                        // rows 0..63 of both 64-column atoms: the first 8 KB of each 16 KB
+                        mbar_arrive_expect_tx(&sh->full[slot], (uint32_t)(kImgBytes / 2) + wb);
+                        bulk_g2s(dst, src, kImgBytes / 4, &sh->full[slot]);
+                        bulk_g2s(dst + kImgBytes / 2, src + kImgBytes / 2, kImgBytes / 4, &sh->full[slot]);
+                    } else {
+                        mbar_arrive_expect_tx(&sh->full[slot], (uint32_t)kImgBytes + wb);
+                        bulk_g2s(dst, src, kImgBytes, &sh->full[slot]);
+                    }
                     bulk_g2s_stream(dst + kImgBytes, wsrc + (size_t)kt * pw * STB, wb, &sh->full[slot], pol);
                     sh->issued = it + 1;
                 }
             }
-            if (ok) {
+            // two end markers, one for each converter group (each takes every
+            // other stage)
+            for (int m = 0; ok && m < 2; ++m, ++it) {
                 const int slot = it % kGSlots;
-                if (it < kGSlots || g_wait(&sh->empty[slot], ((it / kGSlots) - 1) & 1, p, sh)) {
-                    sh->stage[slot].item = -1;
-                    mbar_arrive(&sh->full[slot]);
-                }
+                if (it >= kGSlots && !g_wait(&sh->empty[slot], ((it / kGSlots) - 1) & 1, p, sh)) break;
+                sh->stage[slot].item = -1;
+                mbar_arrive(&sh->full[slot]);
             }
         }
     } else if (warp < kGEpi0 || (warp >= 8 && warp < 12)) {
         // ---------------------------------------------------------- converters --
-        // tensor-memory lanes 32q + 16 u2 .. +15 = the rows of tile 2q + u2
-        const int q = warp & 3, u2 = warp >> 3;
-        for (int it = 0;; ++it) {
-            const int slot = it % kGSlots, b = it & 1;
+        // group cg takes stages cg, cg + 2, ... into A buffer cg; warp q of the
+        // group owns tensor-memory lanes 32q .. 32q + 31 (tiles 2q, 2q + 1)
+        const int q = warp & 3, cg = warp >> 3;
+        const uint32_t abuf = tbase + 256u + 128u * (uint32_t)cg;
+        for (int it = cg, n = 0;; it += 2, ++n) {
+            const int slot = it % kGSlots;
             if (!g_wait(&sh->full[slot], (it / kGSlots) & 1, p, sh)) break;
             const GStage st = sh->stage[slot];
-            if (st.item < 0) break;
+            if (st.item < 0) {
+                // the MMA warps wait on afull only: pass the end marker on, once
+                // the MMAs of the group's previous stage are done (so that afull
+                // never completes a phase before the MMA warps waited for the one
+                // before it)
+                if (n > 0 && !g_wait(&sh->aempty[cg], (uint32_t)((n - 1) & 1), p, sh)) break;
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sh->afull[cg]);
+                break;
+            }
             const int bits = st.ci.bits, STB = supertile_bytes(bits, group), TB = tile_bytes(bits, group);
             const int nstream = W13 ? 2 : w2_pair_width(st.u, nrb);
             const uint8_t *w = ring + (size_t)slot * kGStage + kImgBytes;
-            const uint32_t abuf = tbase + 256u + 128u * (uint32_t)b;
-            // the first stream's tile is dequantised before the A buffer is free (the
-            // MMAs of two stages back may still read it); only its store waits
-            uint32_t v0[32];
-            convert_regs<GPT>(w + (2 * q + u2) * TB, bits, lane, v0);
-            if (it >= 2 && !g_wait(&sh->aempty[b], ((it >> 1) - 1) & 1, p, sh)) break;
-            tc_fence_after();
-            tmem_st_16x256_x8(abuf + ((uint32_t)(32 * q + 16 * u2) << 16), v0);
-            for (int x = 1; x < nstream; ++x) {
-                const uint8_t *tile = w + x * STB + (2 * q + u2) * TB;
-                const uint32_t taddr = abuf + 64u * (uint32_t)x + ((uint32_t)(32 * q + 16 * u2) << 16);
-                convert_store<GPT>(tile, bits, lane, taddr);
-            }
-            tmem_st_wait();
+            if (!convert_stage<GPT>(w, bits, nstream, STB, TB, q, lane, abuf, n > 0, &sh->aempty[cg],
+                                    (uint32_t)((n - 1) & 1), p, sh))
+                break;
             tc_fence_before();
             __syncwarp();
             if (lane == 0) {
-                mbar_arrive(&sh->afull[b]);
+                mbar_arrive(&sh->afull[cg]);
                 mbar_arrive(&sh->empty[slot]);
             }
         }
-    } else if (warp == kGMma) {
+    } else if (warp >= kGMma && warp < kGMma + kGMmaN) {
         // ----------------------------------------------------------------- MMA --
+        const int mx = warp - kGMma;  // the weight stream this warp multiplies
         if (lane == 0) {
-            const uint32_t idesc = umma_idesc_f16(128, kGN);
             int nitem = 0;
             for (int it = 0;; ++it) {
                 const int slot = it % kGSlots, b = it & 1;
-                if (!g_wait(&sh->full[slot], (it / kGSlots) & 1, p, sh)) break;
+                // the stage's converter group arrives after it saw the copies land
+                if (!g_wait(&sh->afull[b], (it >> 1) & 1, p, sh)) break;
                 const GStage st = sh->stage[slot];
                 if (st.item < 0) break;
-                if (!g_wait(&sh->afull[b], (it >> 1) & 1, p, sh)) break;
                 if (st.first && nitem > 0 && !g_wait(&sh->dempty, (nitem - 1) & 1, p, sh)) break;
                 tc_fence_after();
                 const int nstream = W13 ? 2 : w2_pair_width(st.u, nrb);
-                const uint8_t *img = ring + (size_t)slot * kGStage;
-                const uint32_t abuf = tbase + 256u + 128u * (uint32_t)b;
-                for (int x = 0; x < nstream; ++x)
+                if (mx < nstream) {
+                    const uint32_t idesc = umma_idesc_f16(128, st.narrow ? kGNarrow : kGN);
+                    const uint8_t *img = ring + (size_t)slot * kGStage;
+                    const uint32_t abuf = tbase + 256u + 128u * (uint32_t)b + 64u * (uint32_t)mx;
 #pragma unroll
                     for (int s = 0; s < 8; ++s) {
                         const uint64_t bd = umma_desc_sw128(img + (s >> 2) * 16384 + (s & 3) * 32);
-                        umma_f16_ts(tbase + 128u * (uint32_t)x, abuf + 64u * (uint32_t)x + 8u * (uint32_t)s, bd,
-                                    idesc, !(st.first && s == 0));
+                        umma_f16_ts(tbase + 128u * (uint32_t)mx, abuf + 8u * (uint32_t)s, bd, idesc,
+                                    !(st.first && s == 0));
                     }
+                }
                 umma_commit(&sh->aempty[b]);
                 umma_commit(&sh->empty[slot]);
                 if (st.last) {
@@ -458,9 +501,9 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
                     ++nitem;
                 }
             }
-            // every MMA this thread issued has completed (and with it every commit
-            // to dfull) before the epilogue is told that no item follows and
-            // before TMEM is released
+            // every MMA of both warps has completed (and with it every commit to
+            // dfull) before the epilogue is told that no item follows and before
+            // TMEM is released
             umma_commit(&sh->drain);
             const uint64_t t0 = globaltimer_ns();
             while (!mbar_try_wait(&sh->drain, 0))
@@ -468,7 +511,7 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
             // the epilogue has taken the last item before dfull completes once more,
             // so that it never sees two completions of dfull in one wait
             if (nitem == 0 || g_wait(&sh->dempty, (nitem - 1) & 1, p, sh)) {
-                sh->end_items = nitem;
+                if (mx == 0) sh->end_items = nitem;
                 mbar_arrive(&sh->dfull);
             }
         }
@@ -518,8 +561,15 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
                     *reinterpret_cast<__half *>(staging + img_off(2 * i, row)) = __low2half(h);
                     *reinterpret_cast<__half *>(staging + img_off(2 * i + 1, row)) = __high2half(h);
                 }
+                // the image of W2's column step gi.u for token block gi.k
+                if (!epi_sync(p, sh, lane, uses)) break;
+                uint4 *dst = reinterpret_cast<uint4 *>(p.himg + ((size_t)gi.k * (p.F / kTileK) + gi.u) * kImgBytes);
+                const uint4 *src = reinterpret_cast<const uint4 *>(staging);
+                for (int i = tid; i < kImgBytes / 16; i += 128) dst[i] = src[i];
+                if (!epi_sync(p, sh, lane, uses)) break;
             } else {
                 const int nstream = w2_pair_width(gi.u, nrb);
+                float *out = p.opart;
                 for (int x = 0; x < nstream; ++x) {
                     const int blk = 2 * gi.u + x;
                     for (int n0 = 0; n0 < gi.ci.nv; n0 += 16) {
@@ -528,22 +578,12 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
 #pragma unroll
                         for (int i = 0; i < 16; ++i)
                             if (n0 + i < gi.ci.nv)
-                                p.opart[(size_t)(gi.ci.pair_base + n0 + i) * p.H + blk * kBlockRows + row] = v[i];
+                                out[(size_t)(gi.ci.pair_base + n0 + i) * p.H + blk * kBlockRows + row] = v[i];
                     }
                 }
-            }
-            if (!W13) {
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&sh->dempty);
-            }
-            if (W13) {
-                // the image of W2's column step gi.u for token block gi.k
-                if (!epi_sync(p, sh, lane, uses)) break;
-                uint4 *dst = reinterpret_cast<uint4 *>(p.himg + ((size_t)gi.k * (p.F / kTileK) + gi.u) * kImgBytes);
-                const uint4 *src = reinterpret_cast<const uint4 *>(staging);
-                for (int i = tid; i < kImgBytes / 16; i += 128) dst[i] = src[i];
-                if (!epi_sync(p, sh, lane, uses)) break;
             }
         }
     }
