@@ -372,7 +372,13 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
                 int r = 0;
                 while (r + 1 < sh->nruns && item >= sh->run_base[r + 1]) ++r;
                 const int local = item - sh->run_base[r], nbr = sh->run_nb[r];
-                const int u = local / nbr, k = sh->run_first[r] + local % nbr;
+                // W1,W3: the expert's token blocks vary fastest, so the CTAs that run
+                // at the same time share a row block's weights (and the blocks' x
+                // images stay in L2); W2: the 256-row block pairs vary fastest, so
+                // they share one block's h image while the expert's W2 weights stay
+                // in L2 from block to block
+                const int u = W13 ? local / nbr : local % U;
+                const int k = sh->run_first[r] + (W13 ? local % nbr : local / U);
                 const ChunkInfo ci = p.chunks[k];
                 const int e = ci.e, bits = ci.bits;
                 if (!((verified >> e) & 1u)) {
@@ -423,7 +429,11 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
                         mbar_arrive_expect_tx(&sh->full[slot], (uint32_t)kImgBytes + wb);
                         bulk_g2s(dst, src, kImgBytes, &sh->full[slot]);
                     }
-                    bulk_g2s_stream(dst + kImgBytes, wsrc + (size_t)kt * pw * STB, wb, &sh->full[slot], pol);
+                    // W1,W3 weights are read by the CTAs of one row block at about
+                    // the same time: evict-first; a W2 row-block pair's weights come
+                    // back for every token block of the expert: normal policy
+                    if (W13) bulk_g2s_stream(dst + kImgBytes, wsrc + (size_t)kt * pw * STB, wb, &sh->full[slot], pol);
+                    else bulk_g2s(dst + kImgBytes, wsrc + (size_t)kt * pw * STB, wb, &sh->full[slot]);
                     sh->issued = it + 1;
                 }
             }
