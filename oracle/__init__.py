@@ -19,7 +19,9 @@ function states the passage of the paper it follows:
   of the most important tokens; ``odp_threshold`` -- the Eq. 5 threshold as a
   quantile (the median in Sec. 2.3.1) of w1/w0 over calibration tokens.
 * ``expert_significance`` / ``pmq_allocate`` -- Sec. 2.2.1 (phi, w) and the
-  Eq. 4 integer program by brute force.
+  Eq. 4 integer program by brute force; ``expert_error`` -- the eps_{i,j} of
+  Sec. 2.2.2 (layer output with one expert quantised against the unquantised
+  layer).
 * ``stack``                     -- pre-norm residual layers h <- h + MoE(RMSNorm(h)),
   each result rounded to bf16 where the stacked workload stores bf16.
 
@@ -67,7 +69,9 @@ def _load():
     global _lib
     with _lock:
         if _lib is None:
-            lib = ctypes.CDLL(build())
+            # MC_ORACLE_SO: load that build of mc_oracle.c instead (the mutant
+            # tests point it at deliberately broken copies)
+            lib = ctypes.CDLL(os.environ.get("MC_ORACLE_SO") or build())
             P = ctypes.c_void_p
             I = ctypes.c_int
             D = ctypes.c_double
@@ -309,6 +313,25 @@ def expert_significance(idx, w, pruned, E: int):
             phi[idx[t, s]] += 1
             wact[idx[t, s]] += w[t, s]
     return phi / T, wact / T
+
+
+def expert_error(x, wg, dense_mats, quant_mats, mu: float = 0.0, protect=None):
+    """Sec. 2.2.2: eps[i][j-1] = || F(theta) - F(theta[e_i -> Q(e_i, j)]) ||_F over
+    the calibration tokens x [T, H]: the layer output (Eq. 1 with Eq. 5 at mu) with
+    every expert unquantised, against the same layer with only expert i replaced by
+    its j-bit quantisation; the gate is not quantised, so the routing is the same.
+    dense_mats[e] = (w1, w3, w2) QMats with bits 16, quant_mats[e][j-1] = expert e
+    quantised to j bits.  Returns eps fp64 [E, 3]."""
+    E = len(dense_mats)
+    y16, *_ = moe_layer(x, wg, dense_mats, mu, protect)
+    eps = np.zeros((E, 3))
+    for i in range(E):
+        for j in range(3):
+            mats = list(dense_mats)
+            mats[i] = quant_mats[i][j]
+            yq, *_ = moe_layer(x, wg, mats, mu, protect)
+            eps[i, j] = float(np.linalg.norm(yq - y16))
+    return eps
 
 
 def pmq_allocate(phi, wact, eps, bits_total: int, alpha=1.0, beta=1.0, gamma=2.0):

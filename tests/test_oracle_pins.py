@@ -539,3 +539,79 @@ def test_expert_significance_sums():
     for e in range(8):  # brute force count
         n = sum(1 for t in range(90) for s in range(2) if idx[t, s] == e and not ((s and pr[t]) or pr[t] == 2))
         assert phi[e] == pytest.approx(n / 90, rel=1e-12)
+
+
+# ------------------------------------------------------- eps_{i,j} (N3) ----
+
+def _eps_setup(T=10, H=32, F=48, E=4, group=16, seed=51):
+    """Unquantised weights N(0, 0.02) (fp16 values) and their 1/2/3-bit quantisations."""
+    L = synth.make_layer(T, H, F, E, group, [2] * E, seed, gate_std=0.3, experts=False)
+    dense, quant = [], []
+    for e in range(E):
+        ws = [synth.expert_weights_f32(seed, e, m, *L.mat_shape(m)).astype(np.float16).astype(np.float32)
+              for m in range(3)]
+        dense.append([oracle.QMat(*L.mat_shape(m), group, 16, dense=ws[m]) for m in range(3)])
+        quant.append([[oracle.QMat(*L.mat_shape(m), group, j, *synth.rtn_quantize(ws[m], j, group))
+                       for m in range(3)] for j in (1, 2, 3)])
+    return L, dense, quant
+
+
+def test_expert_error_is_the_routing_weighted_expert_difference():
+    """Sec. 2.2.2's eps_{i,j} (two whole layers per (i, j)) equals, by the linearity
+    of Eq. 1 in the expert outputs with the routing unchanged, the F-norm of
+    w_i(t) (E_i^Q(x_t) - E_i^16(x_t)) over the tokens, built from the routing
+    weights and the single-expert function instead."""
+    L, dense, quant = _eps_setup()
+    eps = oracle.expert_error(L.x_f32(), L.gate_f32(), dense, quant)
+    idx, w, pr = oracle.route(L.x_f32(), L.gate_f32(), 0.0)
+    x = L.x_f32().astype(np.float64)
+    for i in range(L.E):
+        for j in range(3):
+            rows = []
+            for t in range(L.T):
+                wi = sum(float(w[t, s]) for s in range(2) if idx[t, s] == i)
+                d = oracle.expert(*quant[i][j], x[t]) - oracle.expert(*dense[i], x[t])
+                rows.append(wi * d)
+            assert eps[i, j] == pytest.approx(np.linalg.norm(np.stack(rows)), rel=1e-9, abs=1e-12)
+
+
+def test_expert_error_invariants():
+    """An expert no token is routed to has eps = 0; a 'quantisation' equal to the
+    dense expert gives eps = 0; doubling an expert's W2 (dense and quantised alike)
+    doubles its eps and leaves the others'."""
+    L, dense, quant = _eps_setup(seed=52)
+    idx, _, _ = oracle.route(L.x_f32(), L.gate_f32(), 0.0)
+    unused = [e for e in range(L.E) if e not in set(idx.reshape(-1).tolist())]
+    eps = oracle.expert_error(L.x_f32(), L.gate_f32(), dense, quant)
+    for e in unused:
+        assert np.all(eps[e] == 0.0)
+    same = [[dense[e]] * 3 for e in range(L.E)]
+    assert np.all(oracle.expert_error(L.x_f32(), L.gate_f32(), dense, same) == 0.0)
+    i = int(idx[0, 0])
+    d2 = [list(m) for m in dense]
+    q2 = [[list(m) for m in qe] for qe in quant]
+    d2[i][2] = oracle.QMat(*L.mat_shape(2), L.group, 16, dense=2.0 * dense[i][2].dense)
+    for j in range(3):
+        c, s_, z = quant[i][j][2].codes, quant[i][j][2].scale, quant[i][j][2].zero
+        q2[i][j][2] = oracle.QMat(*L.mat_shape(2), L.group, j + 1, c, 2.0 * s_, z)
+    eps2 = oracle.expert_error(L.x_f32(), L.gate_f32(), d2, q2)
+    np.testing.assert_allclose(eps2[i], 2.0 * eps[i], rtol=1e-9)
+    others = [e for e in range(L.E) if e != i]
+    np.testing.assert_allclose(eps2[others], eps[others], rtol=1e-12)
+
+
+def test_odp_threshold_is_strict_at_equality():
+    """Eq. 5 prunes when w1/w0 < mu, strictly.  Two identical gate rows give a
+    token bit-equal top-2 logits, so w0 = w1 and w1/w0 = 1 exactly: at mu = 1 the
+    secondary is kept (weights 1/2, 1/2), just above 1 it is pruned."""
+    L = _rand_layer(T=6, H=24, E=4, experts=False)
+    g = L.gate_f32().copy()
+    g[1] = g[0]
+    x = np.abs(L.x_f32()) + 0.1  # logits of experts 0 and 1 the largest
+    g[0] = g[1] = 0.5
+    g[2:] = -0.5
+    idx, w, pr = oracle.route(x, g, 1.0)
+    assert (idx[:, 0] == 0).all() and (idx[:, 1] == 1).all()
+    assert (w[:, 0] == w[:, 1]).all() and (pr == 0).all()
+    _, w2, pr2 = oracle.route(x, g, np.nextafter(1.0, 2.0))
+    assert (pr2 == 1).all() and (w2[:, 0] == 1.0).all() and (w2[:, 1] == 0.0).all()
