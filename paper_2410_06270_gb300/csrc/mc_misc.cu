@@ -76,6 +76,83 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const __nv_bfloat16 *x, co
             __float2bfloat16_rn(__bfloat162float(xr[c]) * inv * __bfloat162float(gamma[c]));
 }
 
+// The same with 16-byte accesses (H % 8 == 0, 16-byte aligned rows, H <= 16384):
+// the row is loaded once into registers, every load issued before the first use,
+// and normalised from there (an in-place call is safe: all loads precede the
+// block barrier).
+constexpr int kRmsPer = 8;  // 16-byte chunks per thread: 256 x 8 x 8 = 16384 columns
+__global__ void __launch_bounds__(256) rmsnorm_vec_kernel(const __nv_bfloat16 *x, const __nv_bfloat16 *gamma,
+                                                          int H, float eps, __nv_bfloat16 *out)
+{
+    pdl_trigger();
+    pdl_wait();
+    const int n8 = H >> 3;
+    const uint4 *xr = reinterpret_cast<const uint4 *>(x + (size_t)blockIdx.x * H);
+    const uint4 *g4 = reinterpret_cast<const uint4 *>(gamma);
+    uint4 *orow = reinterpret_cast<uint4 *>(out + (size_t)blockIdx.x * H);
+    __shared__ float red[8];
+    uint4 v[kRmsPer];
+#pragma unroll
+    for (int i = 0; i < kRmsPer; ++i) {
+        const int c = threadIdx.x + 256 * i;
+        v[i] = c < n8 ? xr[c] : make_uint4(0, 0, 0, 0);
+    }
+    float ss = 0.f;
+#pragma unroll
+    for (int i = 0; i < kRmsPer; ++i) {
+        const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&v[i]);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float2 f = __bfloat1622float2(b2[k]);
+            ss = fmaf(f.x, f.x, ss);
+            ss = fmaf(f.y, f.y, ss);
+        }
+    }
+    for (int m = 16; m >= 1; m >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, m);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+    __syncthreads();
+    float tot = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) tot += red[w];
+    const float inv = rsqrtf(tot / H + eps);
+#pragma unroll
+    for (int i = 0; i < kRmsPer; ++i) {
+        const int c = threadIdx.x + 256 * i;
+        if (c >= n8) continue;
+        const uint4 gv = g4[c];
+        const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&v[i]);
+        const __nv_bfloat162 *gg = reinterpret_cast<const __nv_bfloat162 *>(&gv);
+        uint4 o;
+        __nv_bfloat162 *o2 = reinterpret_cast<__nv_bfloat162 *>(&o);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float2 f = __bfloat1622float2(b2[k]), g = __bfloat1622float2(gg[k]);
+            o2[k] = __floats2bfloat162_rn(f.x * inv * g.x, f.y * inv * g.y);
+        }
+        orow[c] = o;
+    }
+}
+
+// out = a + b, eight bf16 per thread (n % 8 == 0, 16-byte aligned).
+__global__ void add_vec_kernel(const uint4 *a, const uint4 *b, size_t n8, uint4 *out)
+{
+    pdl_trigger();
+    pdl_wait();
+    const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= n8) return;
+    const uint4 x = a[i], y = b[i];
+    const __nv_bfloat162 *x2 = reinterpret_cast<const __nv_bfloat162 *>(&x);
+    const __nv_bfloat162 *y2 = reinterpret_cast<const __nv_bfloat162 *>(&y);
+    uint4 o;
+    __nv_bfloat162 *o2 = reinterpret_cast<__nv_bfloat162 *>(&o);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const float2 f = __bfloat1622float2(x2[k]), g = __bfloat1622float2(y2[k]);
+        o2[k] = __floats2bfloat162_rn(f.x + g.x, f.y + g.y);
+    }
+    out[i] = o;
+}
+
 __global__ void add_kernel(const __nv_bfloat16 *a, const __nv_bfloat16 *b, size_t n, __nv_bfloat16 *out)
 {
     pdl_trigger();
@@ -120,8 +197,9 @@ int mc_rmsnorm(const void *x, const void *gamma, int T, int H, float eps, void *
     if (T < 0 || H <= 0 || !(eps >= 0.f)) return set_error(MC_ERR_INVALID_ARG, "bad T/H/eps");
     if (T == 0) return MC_OK;
     if (!x || !gamma || !out) return set_error(MC_ERR_INVALID_ARG, "NULL pointer argument");
-    cudaError_t e = launch_k(rmsnorm_kernel, dim3(T), dim3(256), 0, (cudaStream_t)stream, (const __nv_bfloat16 *)x,
-                             (const __nv_bfloat16 *)gamma, H, eps, (__nv_bfloat16 *)out);
+    const bool vec = H % 8 == 0 && H <= 256 * 8 * kRmsPer && aligned(x, 16) && aligned(gamma, 16) && aligned(out, 16);
+    cudaError_t e = launch_k(vec ? rmsnorm_vec_kernel : rmsnorm_kernel, dim3(T), dim3(256), 0, (cudaStream_t)stream,
+                             (const __nv_bfloat16 *)x, (const __nv_bfloat16 *)gamma, H, eps, (__nv_bfloat16 *)out);
     if (e != cudaSuccess) return set_error(MC_ERR_CUDA, "rmsnorm launch: %s", cudaGetErrorString(e));
     return MC_OK;
 }
@@ -131,8 +209,13 @@ int mc_add(const void *a, const void *b, size_t n, void *out, void *stream)
     clear_error();
     if (n == 0) return MC_OK;
     if (!a || !b || !out) return set_error(MC_ERR_INVALID_ARG, "NULL pointer argument");
-    cudaError_t e = launch_k(add_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, (cudaStream_t)stream,
-                             (const __nv_bfloat16 *)a, (const __nv_bfloat16 *)b, n, (__nv_bfloat16 *)out);
+    cudaError_t e;
+    if (n % 8 == 0 && aligned(a, 16) && aligned(b, 16) && aligned(out, 16))
+        e = launch_k(add_vec_kernel, dim3((unsigned)((n / 8 + 255) / 256)), dim3(256), 0, (cudaStream_t)stream,
+                     (const uint4 *)a, (const uint4 *)b, n / 8, (uint4 *)out);
+    else
+        e = launch_k(add_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, (cudaStream_t)stream,
+                     (const __nv_bfloat16 *)a, (const __nv_bfloat16 *)b, n, (__nv_bfloat16 *)out);
     if (e != cudaSuccess) return set_error(MC_ERR_CUDA, "add launch: %s", cudaGetErrorString(e));
     return MC_OK;
 }

@@ -421,10 +421,13 @@ def test_activation_outside_fp16_range_is_reported(mc):
 
 # ------------------------------------------------------------- rmsnorm ----
 
-def test_rmsnorm_and_add(mc):
+@pytest.mark.parametrize("H", [4096, 16384, 1001])
+def test_rmsnorm_and_add(mc, H):
+    """RMSNorm against the oracle (16-byte rows up to H 16384 take the vector
+    kernel, H 1001 the scalar one), in place too; the residual add exactly."""
     r = np.random.default_rng(5)
-    xs = synth.f32_to_bf16_bits(r.standard_normal((6, 4096)).astype(np.float32) * 3)
-    gs = synth.f32_to_bf16_bits(r.uniform(0.5, 1.5, 4096).astype(np.float32))
+    xs = synth.f32_to_bf16_bits(r.standard_normal((6, H)).astype(np.float32) * 3)
+    gs = synth.f32_to_bf16_bits(r.uniform(0.5, 1.5, H).astype(np.float32))
     x = torch.from_numpy(xs.view(np.int16)).view(torch.bfloat16).cuda()
     g = torch.from_numpy(gs.view(np.int16)).view(torch.bfloat16).cuda()
     y = mc.rmsnorm(x, g, 1e-5).float().cpu().numpy()
@@ -432,8 +435,14 @@ def test_rmsnorm_and_add(mc):
         ref = oracle.rmsnorm(synth.bf16_bits_to_f32(xs[t]), synth.bf16_bits_to_f32(gs), 1e-5)
         rel, mx = errors(y[t], ref)
         assert rel < 4e-3 and mx < 8e-3
+    xi = x.clone()
+    mc.rmsnorm(xi, g, 1e-5, out=xi)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(xi.float().cpu().numpy(), y)
     s = mc.add(x, x).float().cpu().numpy()
     np.testing.assert_array_equal(s, 2 * synth.bf16_bits_to_f32(xs))
+    s1 = mc.add(x.view(-1)[1:], x.view(-1)[1:]).float().cpu().numpy()  # odd length, unaligned: scalar kernel
+    np.testing.assert_array_equal(s1, 2 * synth.bf16_bits_to_f32(xs).reshape(-1)[1:])
 
 
 @pytest.mark.parametrize("path", [1, 2])
