@@ -69,20 +69,26 @@ __host__ __device__ inline size_t gemv_smem(int nslots, int group, bool dense)
     return kRingOff + (size_t)nslots * slot_bytes(group, dense) + 2 * kHsBytes + 8 * 32 * sizeof(uint2);
 }
 
-// Bounded wait that gives up as soon as another thread of the CTA aborted.
-__device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, const ExpertParams &p, RingShared *sh)
+// Bounded wait that gives up as soon as another thread of the CTA aborted
+// (*abort, the CTA's abort flag).
+__device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, const ExpertParams &p,
+                                              volatile int *abort)
 {
     if (mbar_try_wait(bar, parity)) return true;
     uint64_t t0 = globaltimer_ns();
     while (true) {
         if (mbar_try_wait_sleep(bar, parity, kWaitHintNs)) return true;
-        if (sh->abort) return false;
+        if (*abort) return false;
         if (globaltimer_ns() - t0 > p.timeout_ns) {
             set_status(p.status, MC_ERR_TIMEOUT);
-            sh->abort = 1;
+            *abort = 1;
             return false;
         }
     }
+}
+__device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, const ExpertParams &p, RingShared *sh)
+{
+    return wait_or_abort(bar, parity, p, &sh->abort);
 }
 
 // The packed buffer must carry the header written for this shape and bit table:
@@ -416,13 +422,23 @@ struct Ring {
     const uint2 *afr;  // A fragments of the table matrix
 };
 
-// All consumer warps meet at the CTA's consumer barrier (bounded); false once
-// the CTA aborted.
-__device__ __forceinline__ bool consumer_sync(const ExpertParams &p, RingShared *sh, int lane, int &uses)
+// What one group of consumer warps shares: the CTA's abort flag, the group's
+// epilogue barrier, the column steps of each of its ring's stages, and the
+// thread's index within the group.
+struct GroupCtx {
+    volatile int *abort;
+    uint64_t *cbar;
+    const int *slot_kc;
+    int gtid;
+};
+
+// All consumer warps of a group meet at its barrier (bounded); false once the
+// CTA aborted.
+__device__ __forceinline__ bool consumer_sync(const ExpertParams &p, const GroupCtx &G, int lane, int &uses)
 {
     __syncwarp();
-    if (lane == 0) mbar_arrive(&sh->cbar);
-    return wait_or_abort(&sh->cbar, (uses++) & 1, p, sh);
+    if (lane == 0) mbar_arrive(G.cbar);
+    return wait_or_abort(G.cbar, (uses++) & 1, p, G.abort);
 }
 
 // One work item for one consumer warp: all its stages, then the epilogue.  The
@@ -433,13 +449,12 @@ __device__ __forceinline__ bool consumer_sync(const ExpertParams &p, RingShared 
 //        (double-buffered by item parity), then the consumer warps together
 //        write W2's vector blocks of this 128-row block.
 //   W2:  fp32 outputs of the split.
-template <bool W13, int NT, int BITS, int GPT>
-__device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, const Ring &R, const Item &I, int nrb,
-                                         int tl, int lane, int &slot, uint32_t &phase, __half *hs2, int &items,
-                                         int &cbar_uses)
+template <bool W13, int NT, int BITS, int GPT, int KPS>
+__device__ __forceinline__ bool run_item(const ExpertParams &p, const GroupCtx &G, const Ring &R, const Item &I,
+                                         int nrb, int tl, int lane, int &slot, uint32_t &phase, __half *hs2,
+                                         int &items, int &cbar_uses)
 {
     constexpr int group = kTileK / GPT;
-    constexpr int KPS = BITS == 16 ? 1 : kKPS;  // stage_steps
     const int STB = supertile_bytes(BITS, group), TB = tile_bytes(BITS, group);
     const int pw = W13 ? 2 : w2_pair_width(I.blkA >> 1, nrb);
     const int step_bytes = pw * STB;
@@ -454,9 +469,9 @@ __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, 
 #pragma unroll
             for (int c = 0; c < 4; ++c) y[u][j][c] = 0.f;
     for (int i = 0; i < I.nkt; i += KPS) {
-        if (i > 0 && !wait_or_abort(&R.full[slot], phase, p, sh)) return false;
+        if (i > 0 && !wait_or_abort(&R.full[slot], phase, p, G.abort)) return false;
         const uint8_t *base = R.base + (size_t)slot * R.SB;
-        const int kc = sh->slot_kc[slot];
+        const int kc = G.slot_kc[slot];
         const uint8_t *v0 = base + R.vec_off0, *v1 = v0 + KPS * R.VB;
         auto step = [&](int kk) {
             const uint8_t *st = base + kk * step_bytes;
@@ -505,11 +520,11 @@ __device__ __forceinline__ bool run_item(const ExpertParams &p, RingShared *sh, 
         if (bad) set_status(p.status, MC_ERR_RANGE);
         // every warp finished the previous item's vector blocks before it got
         // here, so after this barrier the other h buffer is free again
-        if (!consumer_sync(p, sh, lane, cbar_uses)) return false;
+        if (!consumer_sync(p, G, lane, cbar_uses)) return false;
         // the item's 128 rows are W2's column step I.u
         const int KT2 = p.F / kTileK;
         write_vec_blocks(hs, NT, group, p.hvec + vec_off(I.k, 0, I.u, KT2, group), vec_off(0, 1, 0, KT2, group),
-                         R.afr, threadIdx.x, kCW * 32);
+                         R.afr, G.gtid, kCW * 32);
     } else {
         float *out = p.opart + (size_t)I.ks * p.Pmax * p.H;
 #pragma unroll
@@ -665,6 +680,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
     } else {
         // --------------------------------------------------------- consumers --
         const Ring R{full, empty, ring, S, SB, vec_off0, VB, afr};
+        const GroupCtx G{&sh->abort, &sh->cbar, sh->slot_kc, (int)threadIdx.x};
         const int tl = warp;
         int slot = 0, items = 0, cbar_uses = 0;
         uint32_t phase = 0;
@@ -676,7 +692,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
             const int sel = (I.ci.bits - 1) * 2 + (I.ci.nv > 8 ? 1 : 0);
             bool ok;
 #define MC_RUN(NT_, B_) \
-    run_item<W13, NT_, B_, GPT>(p, sh, R, I, nrb, tl, lane, slot, phase, hs2, items, cbar_uses)
+    run_item<W13, NT_, B_, GPT, (B_ == 16 ? 1 : kKPS)>(p, G, R, I, nrb, tl, lane, slot, phase, hs2, items, cbar_uses)
             if constexpr (DENSE) {
                 ok = I.ci.nv > 8 ? MC_RUN(2, 16) : MC_RUN(1, 16);
             } else switch (sel) {
@@ -699,6 +715,235 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
             const uint64_t t0 = globaltimer_ns();
             while (!mbar_try_wait(&full[it % S], (it / S) & 1))
                 if (globaltimer_ns() - t0 > p.timeout_ns) break;
+        }
+    }
+}
+
+// -------------------------------------------------------------- ping-pong --
+// gemv_pp_kernel: the quantised-expert GEMV with two consumer groups per CTA.
+// Each group (8 consumer warps owning tile tl of both streams, as above, and a
+// producer warp) has its own ring of two-step stages and its own epilogue
+// barrier and h tiles; both producers claim whole items from the same counter.
+// The two groups' warps share the SM's schedulers, so while one group's warps
+// drain at a stage boundary or run an item's epilogue, the other group's decode
+// and mma keep the pipes issuing.
+constexpr int kPPKPS = 2;                  // 128-column steps per stage
+constexpr int kPPSlots = 2;                // ring slots per group
+constexpr int kPPThreads = 2 * (kCW + 1) * 32;
+constexpr int kPPMinPairs = 32;            // 2 T from which a quantised layer takes this kernel
+
+struct PPGroup {
+    uint64_t full[kPPSlots], empty[kPPSlots];
+    uint64_t cbar;
+    volatile int issued;
+    int slot_item[kPPSlots], slot_kc[kPPSlots];
+    ChunkInfo slot_ci[kPPSlots];
+};
+struct PPShared {
+    PPGroup g[2];
+    volatile int abort;
+    int producers_done;
+};
+static_assert(sizeof(PPShared) <= kRingOff, "ping-pong header");
+
+__host__ __device__ inline int pp_slot_bytes(int group)
+{
+    return kPPKPS * 2 * supertile_bytes(3, group) + 2 * kPPKPS * vec_bytes(group);
+}
+__host__ __device__ inline size_t pp_smem(int group)
+{
+    return kRingOff + (size_t)2 * kPPSlots * pp_slot_bytes(group) + 2 * 2 * kHsBytes + 8 * 32 * sizeof(uint2);
+}
+
+// One group's producer: claims items from the shared counter (the first one
+// already claimed by the caller) and streams them into the group's ring, then
+// one end-marker stage.  Counts itself done on the CTA's counter when it takes
+// no further item; the second producer to do so lets the next kernel launch.
+template <bool W13>
+__device__ __forceinline__ void pp_produce(const ExpertParams &p, PPShared *sh, PPGroup &G, uint8_t *ring, int SB,
+                                           int VB, int vec_off0, int item, ChunkInfo ci, int total, int U, int nrb,
+                                           int KTm, const uint8_t *vbase, int *counter)
+{
+    const int group = p.group;
+    const uint64_t pol = policy_evict_first();
+    int it = 0, pslot = 0;
+    uint32_t pphase = 0;  // phase of the ring round being filled
+    bool ok = true, done = false;
+    auto signal_done = [&]() {
+        if (!done) {
+            done = true;
+            if (atomicAdd(&sh->producers_done, 1) == 1) pdl_trigger();
+        }
+    };
+    if (item >= total) signal_done();
+    while (item < total) {
+        // the next item is claimed with this item's second-to-last stage and its
+        // chunk read with the last one (both round trips overlap copies in flight)
+        int next = total;
+        ChunkInfo next_ci = ci;
+        bool have_ci = false;
+        const Item I = decode_item<W13>(p, item, U, ci);
+        const int nst = (I.nkt + kPPKPS - 1) / kPPKPS, claim_at = nst > 1 ? nst - 2 : 0;
+        const int bits = I.ci.bits, NT = I.ci.nv > 8 ? 2 : 1;
+        const int STB = supertile_bytes(bits, group);
+        const int pw = W13 ? 2 : w2_pair_width(I.blkA >> 1, nrb);
+        const uint8_t *wsrc =
+            p.packed + p.mat_off[I.ci.e][W13 ? 0 : 2] + supertile_off(W13 ? 0 : 2, I.blkA, I.kt0, KTm, nrb, STB);
+        for (int i = 0, st = 0; i < I.nkt; i += kPPKPS, ++it, ++st) {
+            const int slot = pslot;
+            if (it >= kPPSlots && !wait_or_abort(&G.empty[slot], pphase ^ 1u, p, &sh->abort)) {
+                ok = false;
+                break;
+            }
+            if (++pslot == kPPSlots) {
+                pslot = 0;
+                pphase ^= 1u;
+            }
+            const int kc = min(kPPKPS, I.nkt - i);
+            G.slot_item[slot] = item;
+            G.slot_ci[slot] = I.ci;
+            G.slot_kc[slot] = kc;
+            uint8_t *dst = ring + (size_t)slot * SB;
+            const uint32_t wb = (uint32_t)(kc * pw * STB), vb = (uint32_t)(kc * VB);
+            mbar_arrive_expect_tx(&G.full[slot], wb + NT * vb);
+            bulk_g2s_stream(dst, wsrc + (size_t)i * pw * STB, wb, &G.full[slot], pol);
+            for (int j = 0; j < NT; ++j)
+                bulk_g2s(dst + vec_off0 + j * kPPKPS * VB, vbase + vec_off(I.k, j, I.kt0 + i, KTm, group), vb,
+                         &G.full[slot]);
+            G.issued = it + 1;
+            if (st == claim_at) {
+                next = atomicAdd(counter, 1);
+            } else if (st == nst - 1 && next < total) {
+                next_ci = p.chunks[next / U];
+                have_ci = true;
+            }
+        }
+        if (!ok) return;
+        if (!have_ci && next < total) next_ci = p.chunks[next / U];
+        if (next >= total) signal_done();
+        item = next;
+        ci = next_ci;
+    }
+    // end marker: one more stage with item -1 and no data
+    const int slot = pslot;
+    if (it < kPPSlots || wait_or_abort(&G.empty[slot], pphase ^ 1u, p, &sh->abort)) {
+        G.slot_item[slot] = -1;
+        mbar_arrive(&G.full[slot]);
+    }
+}
+
+template <bool W13, int GPT>
+__global__ void __launch_bounds__(kPPThreads, 1) gemv_pp_kernel(ExpertParams p)
+{
+    extern __shared__ __align__(1024) uint8_t smem[];
+    PPShared *sh = reinterpret_cast<PPShared *>(smem);
+    const int group = p.group;
+    const int SB = pp_slot_bytes(group), VB = vec_bytes(group);
+    const int vec_off0 = kPPKPS * 2 * supertile_bytes(3, group);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int g = warp / (kCW + 1), lw = warp % (kCW + 1);  // group, warp within the group (kCW: producer)
+    PPGroup &G = sh->g[g];
+    uint8_t *ring = smem + kRingOff + (size_t)g * kPPSlots * SB;
+    __half *hs2 = reinterpret_cast<__half *>(smem + kRingOff + (size_t)2 * kPPSlots * SB + (size_t)g * 2 * kHsBytes);
+    uint2 *afr = reinterpret_cast<uint2 *>(smem + kRingOff + (size_t)2 * kPPSlots * SB + 4 * kHsBytes);
+    const int nrb = W13 ? p.F / kBlockRows : p.H / kBlockRows;  // 128-row blocks of the matrix
+    const int U = W13 ? nrb : ((nrb + 1) / 2) * p.KS;
+    const int KTm = W13 ? p.H / kTileK : p.F / kTileK;  // column steps of the matrix and its vectors
+    const uint8_t *vbase = W13 ? p.xvec : p.hvec;
+
+    if (threadIdx.x == 0) {
+        for (int gg = 0; gg < 2; ++gg) {
+            for (int s = 0; s < kPPSlots; ++s) {
+                mbar_init(&sh->g[gg].full[s], 1);
+                mbar_init(&sh->g[gg].empty[s], kCW);
+            }
+            mbar_init(&sh->g[gg].cbar, kCW);
+            sh->g[gg].issued = 0;
+        }
+        sh->abort = 0;
+        sh->producers_done = 0;
+        fence_mbar_init();
+    }
+    if (W13) build_tab_afrag(afr, threadIdx.x, kPPThreads);
+    __syncthreads();
+
+    // Each producer's first claim and the header check read only the routing
+    // outputs and the packed weights (complete before this kernel was let
+    // launch), so they overlap the end of the launch before; so does an L2
+    // prefetch of the first stages of each first item.
+    const bool producer = lw == kCW && lane == 0 && !(p.debug & kDebugNoProducer);
+    int *counter = &p.counters[W13 ? 0 : 1];
+    int item = 0, total = 0;
+    bool ok = true;
+    ChunkInfo ci{};
+    if (producer) {
+        const int nchunks = *p.nchunks;
+        item = atomicAdd(counter, 1);
+        ok = header_ok(p);
+        total = nchunks * U;
+        if (ok && item < total) {
+            ci = p.chunks[item / U];
+            const Item I = decode_item<W13>(p, item, U, ci);
+            const int STB = supertile_bytes(I.ci.bits, group);
+            const int pw = W13 ? 2 : w2_pair_width(I.blkA >> 1, nrb);
+            const uint8_t *wsrc =
+                p.packed + p.mat_off[I.ci.e][W13 ? 0 : 2] + supertile_off(W13 ? 0 : 2, I.blkA, I.kt0, KTm, nrb, STB);
+            const int nk = min(I.nkt, kPPSlots * kPPKPS);
+            for (int i = 0; i < nk; i += kPPKPS)
+                bulk_prefetch_l2(wsrc + (size_t)i * pw * STB, (uint32_t)(min(kPPKPS, nk - i) * pw * STB));
+        }
+    }
+    pdl_wait();
+
+    if (lw == kCW) {
+        // ---------------------------------------------------------- producer --
+        if (producer) {
+            if (!ok) {
+                set_status(p.status, MC_ERR_BAD_PACK);
+                sh->abort = 1;
+            } else {
+                pp_produce<W13>(p, sh, G, ring, SB, VB, vec_off0, item, ci, total, U, nrb, KTm, vbase, counter);
+            }
+        }
+    } else {
+        // --------------------------------------------------------- consumers --
+        const Ring R{G.full, G.empty, ring, kPPSlots, SB, vec_off0, VB, afr};
+        const GroupCtx Gc{&sh->abort, &G.cbar, G.slot_kc, lw * 32 + lane};
+        const int tl = lw;
+        int slot = 0, items = 0, cbar_uses = 0;
+        uint32_t phase = 0;
+        while (true) {
+            if (!wait_or_abort(&G.full[slot], phase, p, &sh->abort)) break;
+            const int it_id = G.slot_item[slot];
+            if (it_id < 0) break;
+            const Item I = decode_item<W13>(p, it_id, U, G.slot_ci[slot]);
+            const int sel = (I.ci.bits - 1) * 2 + (I.ci.nv > 8 ? 1 : 0);
+            bool run_ok;
+#define MC_RUN(NT_, B_) \
+    run_item<W13, NT_, B_, GPT, kPPKPS>(p, Gc, R, I, nrb, tl, lane, slot, phase, hs2, items, cbar_uses)
+            switch (sel) {
+            case 0: run_ok = MC_RUN(1, 1); break;
+            case 1: run_ok = MC_RUN(2, 1); break;
+            case 2: run_ok = MC_RUN(1, 2); break;
+            case 3: run_ok = MC_RUN(2, 2); break;
+            case 4: run_ok = MC_RUN(1, 3); break;
+            default: run_ok = MC_RUN(2, 3); break;
+            }
+#undef MC_RUN
+            if (!run_ok) break;
+        }
+    }
+    __syncthreads();
+    // On an abort, let copies that were issued but never consumed land before the
+    // CTA's shared memory is released (bounded).
+    if (threadIdx.x == 0 && sh->abort) {
+        for (int gg = 0; gg < 2; ++gg) {
+            PPGroup &Q = sh->g[gg];
+            for (int it = max(0, Q.issued - kPPSlots); it < Q.issued; ++it) {
+                const uint64_t t0 = globaltimer_ns();
+                while (!mbar_try_wait(&Q.full[it % kPPSlots], (it / kPPSlots) & 1))
+                    if (globaltimer_ns() - t0 > p.timeout_ns) break;
+            }
         }
     }
 }
@@ -755,8 +1000,37 @@ int launch_gemv(ExpertParams ep, cudaStream_t st)
     if (err == cudaSuccess) err = cudaDeviceGetAttribute(&maxsm, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
     if (err == cudaSuccess) err = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "device query: %s", cudaGetErrorString(err));
-    // 16-bit experts are all or none of a layer (check_bits)
+    // 16-bit experts are all or none of a layer (check_bits).  Quantised layers of
+    // >= 16 tokens run the two-group kernel: measured on the Mixtral-8x7b layer at
+    // 16 tokens 127.9 K against 120.8 K tokens/s; at 1 and 4 tokens it was slower
+    // (15.3 / 33.2 K against 17.2 / 36.3 K: with about one item per SM one group
+    // idles and the other's two-slot ring is too shallow to keep the stream busy)
     const bool dense = ep.bits[0] == 16;
+    if (!dense && ep.Pmax >= kPPMinPairs) {
+        const size_t smp = pp_smem(ep.group);
+        if ((size_t)maxsm < smp) return set_error(MC_ERR_UNSUPPORTED, "not enough shared memory for the GEMV rings");
+        auto p13 = ep.group == 64 ? gemv_pp_kernel<true, 2> : gemv_pp_kernel<true, 1>;
+        auto p2 = ep.group == 64 ? gemv_pp_kernel<false, 2> : gemv_pp_kernel<false, 1>;
+        err = cudaFuncSetAttribute(p13, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smp);
+        if (err == cudaSuccess) err = cudaFuncSetAttribute(p2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smp);
+        if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(err));
+        ep.nslots = kPPSlots;
+        profile_begin(kKFragX, st);
+        err = launch_k(frag_x_kernel, dim3(ep.max_chunks, ep.H / kTileK), dim3(256), 0, st, ep);
+        profile_end(kKFragX, st);
+        if (err == cudaSuccess) {
+            profile_begin(kKGemvW13, st);
+            err = launch_k(p13, dim3(nsm), dim3(kPPThreads), smp, st, ep);
+            profile_end(kKGemvW13, st);
+        }
+        if (err == cudaSuccess) {
+            profile_begin(kKGemvW2, st);
+            err = launch_k(p2, dim3(nsm), dim3(kPPThreads), smp, st, ep);
+            profile_end(kKGemvW2, st);
+        }
+        if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "GEMV launch: %s", cudaGetErrorString(err));
+        return MC_OK;
+    }
     int nslots = (int)((maxsm - gemv_smem(0, ep.group, dense)) / slot_bytes(ep.group, dense));
     nslots = nslots > kMaxSlots ? kMaxSlots : nslots;
     if (nslots < 2) return set_error(MC_ERR_UNSUPPORTED, "not enough shared memory for the GEMV ring");

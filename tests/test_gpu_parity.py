@@ -278,7 +278,7 @@ def test_one_workspace_serves_every_token_count(mc):
         assert torch.equal(y, y_fresh), "shared vs fresh workspace, T=%d" % T
 
 
-@pytest.mark.parametrize("T,path", [(8, 1), (8, 2), (130, 0)])
+@pytest.mark.parametrize("T,path", [(8, 1), (40, 1), (8, 2), (130, 0)])
 def test_forward_every_token_dropped(mc, T, path):
     """The degenerate batch: every token dropped (mask byte 2).  No pair reaches
     an expert, every expert kernel runs with zero work items, and the output is
@@ -359,8 +359,10 @@ def test_profile_events_inside_a_captured_graph(mc):
 
 # ---------------------------------------------------------- device faults ----
 
-def test_bounded_wait_reports_timeout_and_context_survives(mc):
-    L = synth.make_layer(4, 256, 256, 8, 64, [2] * 8, 90, gate_std=0.1)
+@pytest.mark.parametrize("T", [4, 20])
+def test_bounded_wait_reports_timeout_and_context_survives(mc, T):
+    """Both GEMV kernels (one consumer group below 16 tokens, two from 16)."""
+    L = synth.make_layer(T, 256, 256, 8, 64, [2] * 8, 90, gate_std=0.1)
     shape, packed = _pack(mc, L)
     x, g, p = to_dev(L)
     ws = mc.alloc_workspace(shape, L.T)
@@ -378,8 +380,9 @@ def test_bounded_wait_reports_timeout_and_context_survives(mc):
     assert torch.isfinite(y.float()).all()
 
 
-def test_corrupt_pack_header_is_reported(mc):
-    L = synth.make_layer(4, 256, 256, 8, 64, [2] * 8, 91, gate_std=0.1)
+@pytest.mark.parametrize("T", [4, 20])
+def test_corrupt_pack_header_is_reported(mc, T):
+    L = synth.make_layer(T, 256, 256, 8, 64, [2] * 8, 91, gate_std=0.1)
     shape, packed = _pack(mc, L)
     x, g, p = to_dev(L)
     bad = packed.clone()
