@@ -290,6 +290,7 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     ep.Pmax = 2 * T;
     ep.max_chunks = ws.max_chunks;
     ep.status = ws.status;
+    ep.hdr_ok = ws.status + kHdrOkWord;
     ep.timeout_ns = g_timeout_ns;
     ep.debug = g_debug;
     rc = path == kPathGemm ? launch_gemm(ep, st) : launch_gemv(ep, st);

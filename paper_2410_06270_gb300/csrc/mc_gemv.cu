@@ -196,11 +196,21 @@ __global__ void __launch_bounds__(256) frag_x_kernel(ExpertParams p)
     __shared__ __align__(16) __half xs[kChunk * kTileK];
     __shared__ uint2 afr[8 * 32];
     const int k = blockIdx.x, kt = blockIdx.y, KT = p.H / kTileK;
+    // CTA (0, 0) checks the packed header for the expert kernels that follow (they
+    // read only its verdict): the header's loads go out before the wait (the packed
+    // buffer is complete before the layer starts), the verdict is written after it,
+    // when the expert kernels of the call before have completed
+    const bool hdr_thread = k == 0 && kt == 0 && threadIdx.x == 0;
+    const bool hok = hdr_thread ? header_ok(p) : true;
     build_tab_afrag(afr, threadIdx.x, 256);
     // trigger only after the routing launch has completed: the expert kernel that
     // follows reads the routing outputs before its own wait
     pdl_wait();
     pdl_trigger();
+    if (hdr_thread) {
+        *p.hdr_ok = hok ? 1 : 0;
+        if (!hok) set_status(p.status, MC_ERR_BAD_PACK);
+    }
     // both loads in flight together (entry k < max_chunks exists even when unused)
     const int nchunks = *p.nchunks;
     const ChunkInfo ci = p.chunks[k];
@@ -589,25 +599,17 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
     if (producer) {
         const int nchunks = *p.nchunks;
         item = atomicAdd(counter, 1);
-        ok = header_ok(p);
         total = nchunks * U;
-        if (ok && item < total) {
-            ci = p.chunks[item / U];
-            const Item I = decode_item<W13>(p, item, U, ci);
-            const int STB = supertile_bytes(I.ci.bits, group);
-            const int pw = W13 ? 2 : w2_pair_width(I.blkA >> 1, nrb);
-            const uint8_t *wsrc =
-                p.packed + p.mat_off[I.ci.e][W13 ? 0 : 2] + supertile_off(W13 ? 0 : 2, I.blkA, I.kt0, KTm, nrb, STB);
-            const int nk = min(I.nkt, S * KPS);
-            for (int i = 0; i < nk; i += KPS)
-                bulk_prefetch_l2(wsrc + (size_t)i * pw * STB, (uint32_t)(min(KPS, nk - i) * pw * STB));
-        }
+        if (item < total) ci = p.chunks[item / U];
     }
     pdl_wait();
 
     if (warp == kCW) {
         // ---------------------------------------------------------- producer --
         if (producer) {
+            // no copy before the packed header's verdict (published by frag_x_kernel,
+            // which completed before this wait returned)
+            ok = __ldcg(p.hdr_ok) == 1;
             const uint64_t pol = policy_evict_first();
             int it = 0, pslot = 0;
             uint32_t pphase = 0;  // phase of the ring round being filled
@@ -867,10 +869,8 @@ __global__ void __launch_bounds__(kPPThreads, 1) gemv_pp_kernel(ExpertParams p)
     if (W13) build_tab_afrag(afr, threadIdx.x, kPPThreads);
     __syncthreads();
 
-    // Each producer's first claim and the header check read only the routing
-    // outputs and the packed weights (complete before this kernel was let
-    // launch), so they overlap the end of the launch before; so does an L2
-    // prefetch of the first stages of each first item.
+    // Each producer's first claim reads only the routing outputs (complete before
+    // this kernel was let launch), so it overlaps the end of the launch before.
     const bool producer = lw == kCW && lane == 0 && !(p.debug & kDebugNoProducer);
     int *counter = &p.counters[W13 ? 0 : 1];
     int item = 0, total = 0;
@@ -879,25 +879,17 @@ __global__ void __launch_bounds__(kPPThreads, 1) gemv_pp_kernel(ExpertParams p)
     if (producer) {
         const int nchunks = *p.nchunks;
         item = atomicAdd(counter, 1);
-        ok = header_ok(p);
         total = nchunks * U;
-        if (ok && item < total) {
-            ci = p.chunks[item / U];
-            const Item I = decode_item<W13>(p, item, U, ci);
-            const int STB = supertile_bytes(I.ci.bits, group);
-            const int pw = W13 ? 2 : w2_pair_width(I.blkA >> 1, nrb);
-            const uint8_t *wsrc =
-                p.packed + p.mat_off[I.ci.e][W13 ? 0 : 2] + supertile_off(W13 ? 0 : 2, I.blkA, I.kt0, KTm, nrb, STB);
-            const int nk = min(I.nkt, kPPSlots * kPPKPS);
-            for (int i = 0; i < nk; i += kPPKPS)
-                bulk_prefetch_l2(wsrc + (size_t)i * pw * STB, (uint32_t)(min(kPPKPS, nk - i) * pw * STB));
-        }
+        if (item < total) ci = p.chunks[item / U];
     }
     pdl_wait();
 
     if (lw == kCW) {
         // ---------------------------------------------------------- producer --
         if (producer) {
+            // no copy before the packed header's verdict (published by frag_x_kernel,
+            // which completed before this wait returned)
+            ok = __ldcg(p.hdr_ok) == 1;
             if (!ok) {
                 set_status(p.status, MC_ERR_BAD_PACK);
                 sh->abort = 1;

@@ -87,9 +87,14 @@ struct ExpertParams {
     int max_chunks;
     int nslots;              // stages of the shared-memory ring
     int32_t *status;
+    int32_t *hdr_ok;         // the packed header's verdict for this call (1: matches), written by frag_x_kernel
     uint64_t timeout_ns;
     int debug;               // test hooks (kDebugNoProducer)
 };
+
+// Word of the 256-byte status area at the start of a workspace that holds the
+// packed header's verdict (the status word itself is word 0).
+constexpr int kHdrOkWord = 16;
 
 constexpr int kDebugNoProducer = 1;  // the copy producer never issues: waits expire
 constexpr int kDebugNoPdl = 2;       // launch without programmatic dependent launch

@@ -181,6 +181,7 @@ extern "C" int mc_moe_forward_static(const void *x, const void *gate_w, int T, c
     ep.Pmax = 2 * T;
     ep.max_chunks = ws.max_chunks;
     ep.status = status;
+    ep.hdr_ok = ws.status + kHdrOkWord;
     ep.timeout_ns = wait_bound_ns();  // the mc_set_debug hooks apply here as well
     ep.debug = debug_flags();
     if ((rc = launch_gemv(ep, st))) return rc;
