@@ -112,21 +112,37 @@ __device__ __forceinline__ bool g_wait(uint64_t *bar, uint32_t parity, const Exp
     }
 }
 
-__device__ __forceinline__ bool g_header_ok(const ExpertParams &p, int e)
+// The packed buffer carries the header written for this shape and bit table
+// (every expert's bit width and matrix offsets), so no copy reads outside it.
+__device__ __forceinline__ bool g_header_ok(const ExpertParams &p)
 {
     const PackHeader *hd = reinterpret_cast<const PackHeader *>(p.packed);
-    return hd->magic == kMagic && hd->version == kFormatVersion && hd->E == p.E && hd->H == p.H &&
-           hd->F == p.F && hd->group == p.group && hd->bits[e] == p.bits[e] &&
-           hd->mat_off[e][0] == p.mat_off[e][0] && hd->mat_off[e][1] == p.mat_off[e][1] &&
-           hd->mat_off[e][2] == p.mat_off[e][2];
+    bool ok = hd->magic == kMagic && hd->version == kFormatVersion && hd->E == p.E && hd->H == p.H &&
+              hd->F == p.F && hd->group == p.group;
+#pragma unroll
+    for (int e = 0; e < kMaxE; ++e)
+        if (e < p.E)
+            ok &= hd->bits[e] == p.bits[e] && hd->mat_off[e][0] == p.mat_off[e][0] &&
+                  hd->mat_off[e][1] == p.mat_off[e][1] && hd->mat_off[e][2] == p.mat_off[e][2];
+    return ok;
 }
 
 // ------------------------------------------------------------------ x image --
 __global__ void __launch_bounds__(256) x_img_kernel(ExpertParams p)
 {
     const int k = blockIdx.x, kt = blockIdx.y, KT = p.H / kTileK;
+    // CTA (0, 0) checks the packed header for the two GEMM launches that follow
+    // (they read only its verdict): the header's loads go out before the wait (the
+    // packed buffer is complete before the layer starts), the verdict is written
+    // after it, when the expert kernels of the call before have completed
+    const bool hdr_thread = k == 0 && kt == 0 && threadIdx.x == 0;
+    const bool hok = hdr_thread ? g_header_ok(p) : true;
     pdl_trigger();
     pdl_wait();
+    if (hdr_thread) {
+        *p.hdr_ok = hok ? 1 : 0;
+        if (!hok) set_status(p.status, MC_ERR_BAD_PACK);
+    }
     const int nblocks = *p.nchunks;
     const ChunkInfo ci = p.chunks[k];  // entry k < max_blocks exists even when unused
     if (k >= nblocks) return;
@@ -361,10 +377,23 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
         if (lane == 0 && !(p.debug & kDebugNoProducer)) {
             const uint64_t pol = policy_evict_first();
             int it = 0, nitem = 0;
-            bool ok = true;
-            uint32_t verified = 0;
+            // The packed header was checked once for the call by x_img_kernel, which
+            // completed before this launch's wait returned: no copy unless its verdict
+            // says the buffer matches (the verdict's load and the first claim go out
+            // together; the verdict is looked at once the claim returns)
+            const int verdict = __ldcg(p.hdr_ok);
+            bool ok = true, checked = false;
             while (ok) {
                 const int item = atomicAdd(&p.counters[W13 ? 2 : 3], 1);
+                if (!checked) {
+                    checked = true;
+                    if (verdict != 1) {
+                        set_status(p.status, MC_ERR_BAD_PACK);
+                        sh->abort = 1;
+                        ok = false;
+                        break;
+                    }
+                }
                 if (item >= total) {
                     pdl_trigger();  // the CTA takes no further item: the next kernel may launch
                     break;
@@ -381,15 +410,6 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_kernel(ExpertParams p)
                 const int k = sh->run_first[r] + (W13 ? local % nbr : local / U);
                 const ChunkInfo ci = p.chunks[k];
                 const int e = ci.e, bits = ci.bits;
-                if (!((verified >> e) & 1u)) {
-                    if (!g_header_ok(p, e)) {
-                        set_status(p.status, MC_ERR_BAD_PACK);
-                        sh->abort = 1;
-                        ok = false;
-                        break;
-                    }
-                    verified |= 1u << e;
-                }
                 GItem gi;
                 gi.k = k;
                 gi.u = u;
