@@ -983,6 +983,54 @@ __global__ void __launch_bounds__(256) combine_kernel(CombineParams p)
     *reinterpret_cast<uint4 *>(p.y + (size_t)t * p.H + c) = *reinterpret_cast<uint4 *>(r);
 }
 
+// The same for decode-sized calls (T <= 64): one thread per 4 output columns in
+// 128-thread CTAs, so that the grid spreads over the SMs, and every split of
+// both slots loaded before the first is used (one round trip after the routing
+// outputs).  Same summation order as combine_kernel.
+constexpr int kCombine4MaxT = 64;
+
+__global__ void __launch_bounds__(128) combine4_kernel(CombineParams p)
+{
+    pdl_trigger();
+    pdl_wait();
+    const int H4 = p.H / 4;
+    const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= p.T * H4) return;
+    const int t = idx / H4, c = (idx % H4) * 4;
+    const int2 q2 = *reinterpret_cast<const int2 *>(p.inv + 2 * t);
+    const float2 w2 = *reinterpret_cast<const float2 *>(p.w + 2 * t);
+    float4 a[2][kMaxKS];
+#pragma unroll
+    for (int slot = 0; slot < 2; ++slot) {
+        const int q = slot ? q2.y : q2.x;
+#pragma unroll
+        for (int ks = 0; ks < kMaxKS; ++ks)
+            if (ks < p.KS && q >= 0)
+                a[slot][ks] = *reinterpret_cast<const float4 *>(p.opart + ((size_t)ks * p.Pmax + q) * p.H + c);
+    }
+    float out[4] = {0, 0, 0, 0};
+#pragma unroll
+    for (int slot = 0; slot < 2; ++slot) {
+        if ((slot ? q2.y : q2.x) < 0) continue;
+        const float wt = slot ? w2.y : w2.x;
+        float o[4] = {0, 0, 0, 0};
+#pragma unroll
+        for (int ks = 0; ks < kMaxKS; ++ks)
+            if (ks < p.KS) {
+                o[0] += a[slot][ks].x;
+                o[1] += a[slot][ks].y;
+                o[2] += a[slot][ks].z;
+                o[3] += a[slot][ks].w;
+            }
+#pragma unroll
+        for (int k = 0; k < 4; ++k) out[k] = fmaf(wt, o[k], out[k]);
+    }
+    __nv_bfloat16 r[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) r[k] = __float2bfloat16_rn(out[k]);
+    *reinterpret_cast<uint2 *>(p.y + (size_t)t * p.H + c) = *reinterpret_cast<uint2 *>(r);
+}
+
 // -------------------------------------------------------------- launchers --
 
 int launch_gemv(ExpertParams ep, cudaStream_t st)
@@ -1055,10 +1103,16 @@ int launch_gemv(ExpertParams ep, cudaStream_t st)
 
 int launch_combine(const CombineParams &cp, cudaStream_t st)
 {
-    const int n = cp.T * (cp.H / 8);
     if (cp.KS < 1 || cp.KS > kMaxKS) return set_error(MC_ERR_INVALID_ARG, "combine: %d column splits", cp.KS);
     profile_begin(kKCombine, st);
-    cudaError_t err = launch_k(combine_kernel, dim3((n + 255) / 256), dim3(256), 0, st, cp);
+    cudaError_t err;
+    if (cp.T <= kCombine4MaxT) {
+        const int n = cp.T * (cp.H / 4);
+        err = launch_k(combine4_kernel, dim3((n + 127) / 128), dim3(128), 0, st, cp);
+    } else {
+        const int n = cp.T * (cp.H / 8);
+        err = launch_k(combine_kernel, dim3((n + 255) / 256), dim3(256), 0, st, cp);
+    }
     profile_end(kKCombine, st);
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "combine launch: %s", cudaGetErrorString(err));
     return MC_OK;
