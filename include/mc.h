@@ -208,7 +208,8 @@ int mc_moe_forward_static(const void *x, const void *gate_w, int T, const mc_sha
                           const uint8_t *protect, void *y, int32_t *status_dev, void *stream);
 
 /* Workspace bytes of mc_stack_forward for up to T_max tokens: the layer
- * workspace (status word first) followed by two [T_max, H] bf16 activations. */
+ * workspace (status word first) followed by one [T_max, H] bf16 activation (the
+ * normalised layer input). */
 size_t mc_stack_workspace_size(const mc_shape *shape, int T_max);
 
 /* A stack of `layers` pre-norm residual MoE blocks, the structure of the

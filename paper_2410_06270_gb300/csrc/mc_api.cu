@@ -202,9 +202,14 @@ int mc_route(const void *x, const void *gate_w, int T, const mc_shape *shape, fl
     return launch_route(rp, pp, (cudaStream_t)stream);
 }
 
-int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *shape, const int8_t *bits_host,
-                   const void *packed_dev, float mu, const uint8_t *protect, void *y, void *workspace,
-                   size_t ws_bytes, int32_t *topk_idx_out, float *topk_w_out, uint8_t *pruned_out, void *stream)
+}  // extern "C"
+
+// mc_moe_forward with an optional residual added in its last kernel (resid may
+// alias y; the stack's h <- h + MoE(RMSNorm(h)) without a separate add).
+int mc::moe_forward_resid(const void *x, const void *gate_w, int T, const mc_shape *shape, const int8_t *bits_host,
+                          const void *packed_dev, float mu, const uint8_t *protect, void *y, const void *resid,
+                          void *workspace, size_t ws_bytes, int32_t *topk_idx_out, float *topk_w_out,
+                          uint8_t *pruned_out, void *stream)
 {
     clear_error();
     int rc = check_bits(shape, bits_host);
@@ -305,7 +310,18 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
     cp.KS = ep.KS;
     cp.Pmax = 2 * T;
     cp.y = (__nv_bfloat16 *)y;
+    cp.resid = (const __nv_bfloat16 *)resid;
     return launch_combine(cp, st);
+}
+
+extern "C" {
+
+int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *shape, const int8_t *bits_host,
+                   const void *packed_dev, float mu, const uint8_t *protect, void *y, void *workspace,
+                   size_t ws_bytes, int32_t *topk_idx_out, float *topk_w_out, uint8_t *pruned_out, void *stream)
+{
+    return moe_forward_resid(x, gate_w, T, shape, bits_host, packed_dev, mu, protect, y, nullptr, workspace,
+                             ws_bytes, topk_idx_out, topk_w_out, pruned_out, stream);
 }
 
 int mc_check_status(void *workspace, void *stream)

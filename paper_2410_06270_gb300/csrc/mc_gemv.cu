@@ -942,7 +942,9 @@ __global__ void __launch_bounds__(kPPThreads, 1) gemv_pp_kernel(ExpertParams p)
 
 // ---------------------------------------------------------------- combine --
 // y[t] = w0 * o[p(t,0)] + w1 * o[p(t,1)] (second term absent when pruned),
-// summing the column splits of the W2 pass in a fixed order (Eq. 1 with Eq. 5).
+// summing the column splits of the W2 pass in a fixed order (Eq. 1 with Eq. 5);
+// with a residual (the pre-norm stack), y[t] = resid[t] + that, rounded to bf16
+// first (the layer's own output) and once more after the fp32 add.
 //   Every load of a slot's column splits is issued before the first is used.
 __global__ void __launch_bounds__(256) combine_kernel(CombineParams p)
 {
@@ -980,6 +982,12 @@ __global__ void __launch_bounds__(256) combine_kernel(CombineParams p)
     __nv_bfloat16 r[8];
 #pragma unroll
     for (int k = 0; k < 8; ++k) r[k] = __float2bfloat16_rn(out[k]);
+    if (p.resid) {
+        const uint4 rv = *reinterpret_cast<const uint4 *>(p.resid + (size_t)t * p.H + c);
+        const __nv_bfloat16 *rb = reinterpret_cast<const __nv_bfloat16 *>(&rv);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) r[k] = __float2bfloat16_rn(__bfloat162float(rb[k]) + __bfloat162float(r[k]));
+    }
     *reinterpret_cast<uint4 *>(p.y + (size_t)t * p.H + c) = *reinterpret_cast<uint4 *>(r);
 }
 
@@ -999,6 +1007,7 @@ __global__ void __launch_bounds__(128) combine4_kernel(CombineParams p)
     const int t = idx / H4, c = (idx % H4) * 4;
     const int2 q2 = *reinterpret_cast<const int2 *>(p.inv + 2 * t);
     const float2 w2 = *reinterpret_cast<const float2 *>(p.w + 2 * t);
+    const uint2 rv = p.resid ? *reinterpret_cast<const uint2 *>(p.resid + (size_t)t * p.H + c) : make_uint2(0, 0);
     float4 a[2][kMaxKS];
 #pragma unroll
     for (int slot = 0; slot < 2; ++slot) {
@@ -1028,6 +1037,11 @@ __global__ void __launch_bounds__(128) combine4_kernel(CombineParams p)
     __nv_bfloat16 r[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k) r[k] = __float2bfloat16_rn(out[k]);
+    if (p.resid) {
+        const __nv_bfloat16 *rb = reinterpret_cast<const __nv_bfloat16 *>(&rv);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) r[k] = __float2bfloat16_rn(__bfloat162float(rb[k]) + __bfloat162float(r[k]));
+    }
     *reinterpret_cast<uint2 *>(p.y + (size_t)t * p.H + c) = *reinterpret_cast<uint2 *>(r);
 }
 

@@ -108,6 +108,9 @@ struct CombineParams {
     const int32_t *inv;   // [2T]
     int T, H, KS, Pmax;
     __nv_bfloat16 *y;     // [T, H]
+    // optional residual: y = resid + (the layer output rounded to bf16), added in
+    // fp32 and rounded once more (resid may alias y); null: y = the layer output
+    const __nv_bfloat16 *resid;
 };
 
 // Launch with programmatic stream serialisation (unless switched off by
@@ -147,6 +150,12 @@ int32_t *route_done_word();  // mc_route's arrival word for the single-launch ro
 // best, among the divisors of F/128 that leave every item >= 8 column steps).
 int max_ks(const mc_shape *s, int T);
 int choose_ks(const mc_shape *s, int T, int nsm);
+// mc_moe_forward whose last kernel writes y = resid + the layer output (resid may
+// alias y; null: mc_moe_forward itself).  Used by mc_stack_forward.
+int moe_forward_resid(const void *x, const void *gate_w, int T, const mc_shape *shape, const int8_t *bits_host,
+                      const void *packed_dev, float mu, const uint8_t *protect, void *y, const void *resid,
+                      void *workspace, size_t ws_bytes, int32_t *topk_idx_out, float *topk_w_out,
+                      uint8_t *pruned_out, void *stream);
 // The test hooks of mc_set_debug: its flags and the bound on device waits.
 int debug_flags();
 uint64_t wait_bound_ns();

@@ -16,7 +16,7 @@ extern "C" size_t mc_stack_workspace_size(const mc_shape *shape, int T_max)
 {
     const size_t ws = mc_moe_workspace_size(shape, T_max);
     if (!ws) return 0;
-    return align256(ws) + 2 * align256((size_t)T_max * shape->H * 2);
+    return align256(ws) + align256((size_t)T_max * shape->H * 2);
 }
 
 extern "C" int mc_stack_forward(void *h, int T, const mc_shape *shape, int layers, const void *const *gate_w,
@@ -34,17 +34,15 @@ extern "C" int mc_stack_forward(void *h, int T, const mc_shape *shape, int layer
     const size_t need = mc_stack_workspace_size(shape, T);
     if (ws_bytes < need) return set_error(MC_ERR_INVALID_ARG, "workspace has %zu bytes, needs %zu", ws_bytes, need);
     const size_t fw = align256(mc_moe_workspace_size(shape, T));
-    const size_t act = align256((size_t)T * shape->H * 2);
-    uint8_t *base = (uint8_t *)workspace;
-    void *xn = base + fw, *y = base + fw + act;
-    const size_t n = (size_t)T * shape->H;
+    void *xn = (uint8_t *)workspace + fw;
     for (int l = 0; l < layers; ++l) {
         const void *g = (const uint8_t *)gamma + (size_t)l * shape->H * 2;
         if ((rc = mc_rmsnorm(h, g, T, shape->H, eps, xn, stream))) return rc;
-        if ((rc = mc_moe_forward(xn, gate_w[l], T, shape, bits_host + (size_t)l * shape->E, packed_dev[l],
-                                 mu_host[l], protect, y, workspace, fw, nullptr, nullptr, nullptr, stream)))
+        // the layer's combine adds its output to h in place (h + MoE(xn), rounded
+        // like mc_add of the layer's bf16 output)
+        if ((rc = moe_forward_resid(xn, gate_w[l], T, shape, bits_host + (size_t)l * shape->E, packed_dev[l],
+                                    mu_host[l], protect, h, h, workspace, fw, nullptr, nullptr, nullptr, stream)))
             return rc;
-        if ((rc = mc_add(h, y, n, h, stream))) return rc;
     }
     return MC_OK;
 }

@@ -380,8 +380,13 @@ def test_bounded_wait_reports_timeout_and_context_survives(mc, T):
     assert torch.isfinite(y.float()).all()
 
 
-@pytest.mark.parametrize("T", [4, 20])
-def test_corrupt_pack_header_is_reported(mc, T):
+@pytest.mark.parametrize("T,path", [(4, "auto"), (20, "auto"), (20, "gemm")])
+def test_corrupt_pack_header_is_reported(mc, T, path):
+    """The packed header is checked once per call (by the kernel that prepares the
+    activations) and the expert kernels copy nothing unless its verdict says the
+    buffer matches; the verdict is rewritten by every call, so a good call after
+    a bad one runs normally.  Both expert paths: the GEMV kernels (single-group
+    at 4 tokens, two-group at 20) and the GEMM."""
     L = synth.make_layer(T, 256, 256, 8, 64, [2] * 8, 91, gate_std=0.1)
     shape, packed = _pack(mc, L)
     x, g, p = to_dev(L)
@@ -390,24 +395,34 @@ def test_corrupt_pack_header_is_reported(mc, T):
     with pytest.raises(mc.MCError) as ei:
         mc.pack_verify(shape, L.bits, bad)
     assert ei.value.code == mc.ERR_BAD_PACK
-    ws = mc.alloc_workspace(shape, L.T)
-    mc.moe_forward(x, g, shape, L.bits, bad, workspace=ws)
-    with pytest.raises(mc.MCError) as ei:
+    old = mc.set_path(mc.PATH_GEMM if path == "gemm" else mc.PATH_AUTO)
+    try:
+        ws = mc.alloc_workspace(shape, L.T)
+        y_good = mc.moe_forward(x, g, shape, L.bits, packed, workspace=ws).clone()
         mc.check_status(ws)
-    assert ei.value.code == mc.ERR_BAD_PACK
-    # a bit table that disagrees with the buffer is reported the same way, both
-    # when the wrong entry is a routed expert's and when it only shifts the
-    # offsets of the experts after it (expert 0 untouched by these tokens)
-    idx, _, _ = oracle.route(L.x_f32(), L.gate_f32(), 0.0)
-    touched = sorted(set(idx.reshape(-1).tolist()))
-    shifting = [e for e in range(L.E) if e not in touched and any(t > e for t in touched)]
-    for e in [touched[0]] + shifting[:1]:
-        other = np.array(L.bits).copy()
-        other[e] = 3 if other[e] != 3 else 1
-        mc.moe_forward(x, g, shape, other, packed, workspace=ws)
+        mc.moe_forward(x, g, shape, L.bits, bad, workspace=ws)
         with pytest.raises(mc.MCError) as ei:
             mc.check_status(ws)
         assert ei.value.code == mc.ERR_BAD_PACK
+        # the next call with the right buffer is not affected by the bad one
+        y_again = mc.moe_forward(x, g, shape, L.bits, packed, workspace=ws)
+        mc.check_status(ws)
+        assert torch.equal(y_again, y_good)
+        # a bit table that disagrees with the buffer is reported the same way, both
+        # when the wrong entry is a routed expert's and when it only shifts the
+        # offsets of the experts after it (expert 0 untouched by these tokens)
+        idx, _, _ = oracle.route(L.x_f32(), L.gate_f32(), 0.0)
+        touched = sorted(set(idx.reshape(-1).tolist()))
+        shifting = [e for e in range(L.E) if e not in touched and any(t > e for t in touched)]
+        for e in [touched[0]] + shifting[:1]:
+            other = np.array(L.bits).copy()
+            other[e] = 3 if other[e] != 3 else 1
+            mc.moe_forward(x, g, shape, other, packed, workspace=ws)
+            with pytest.raises(mc.MCError) as ei:
+                mc.check_status(ws)
+            assert ei.value.code == mc.ERR_BAD_PACK
+    finally:
+        mc.set_path(old)
 
 
 def test_activation_outside_fp16_range_is_reported(mc):
