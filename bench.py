@@ -797,7 +797,7 @@ def measure_stack(name, args, torch, mc, dev, local, world, cpu=True):
                    "weights": "one seeded expert set shared by the layers (separate copies), per-layer gates",
                    "kept_pairs": pairs},
         "roofline": {"bound": "hbm", "kernel": "stack step (CUDA graph: %d layers of rmsnorm, route, permute, "
-                                                "GEMV W1|W3, GEMV W2, combine with the residual add)" % layers,
+                                                "GEMV W1|W3, GEMV W2, combine; RMSNorm in the routing launch, residual add in the combine)" % layers,
                      "achieved": gbs, "peak": hbm, "unit": "GB/s", "frac": gbs / hbm, "traffic": None,
                      "frac_of_nominal_7900": gbs / HBM_NOMINAL_GBS,
                      "peak_source": "%s (MEASURED_PEAKS.json hbm_gbs)" % src if src == "measured" else src,
@@ -807,9 +807,9 @@ def measure_stack(name, args, torch, mc, dev, local, world, cpu=True):
         "kernels_ms_per_step": {k: v[0] for k, v in breakdown.items()},
         "e2e": {"value": job_throughput(world, T, steps, ms_e2e), "unit": "tokens/s",
                 "h2d_bytes_per_step": int(x0.numel() * 2), "d2h_bytes_per_step": int(hs.numel() * 2)},
-        # the profiled kernels of one call plus one rmsnorm launch per layer (the
-        # residual add is part of each layer's combine)
-        "gpu_launches": (_launches_per_step(breakdown, 1) + layers) * steps,
+        # the profiled kernels of one call (each layer's RMSNorm runs in its routing
+        # launch and its residual add in its combine)
+        "gpu_launches": _launches_per_step(breakdown, 1) * steps,
         "clocks": _clock_note(cl),
     }
     if cpu and not args.no_cpu_baseline:

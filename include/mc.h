@@ -218,7 +218,11 @@ size_t mc_stack_workspace_size(const mc_shape *shape, int T_max);
  * MoE_l is mc_moe_forward with gate_w[l] (device bf16 [E, H]), packed_dev[l],
  * the bit table bits_host[l*E .. l*E+E-1] and threshold mu_host[l]; RMSNorm_l
  * uses gamma + l*H (device bf16 [layers, H]) and eps.  h (device bf16 [T, H]) is
- * updated in place; every intermediate is bf16.  protect (device [T] or NULL)
+ * updated in place; every intermediate is bf16.  With 16-byte aligned h and
+ * gamma each layer's RMSNorm runs inside its routing launch and its residual add
+ * inside its combine, with the arithmetic and rounding of mc_rmsnorm and mc_add
+ * (the result is bit for bit that of mc_rmsnorm, mc_moe_forward and mc_add in
+ * turn).  protect (device [T] or NULL)
  * applies to every layer.  Device-detected faults of any layer go to the status
  * word at the start of `workspace` (mc_check_status).  All launches go to
  * `stream` and none synchronises, so a caller may capture one call into a CUDA

@@ -204,12 +204,12 @@ int mc_route(const void *x, const void *gate_w, int T, const mc_shape *shape, fl
 
 }  // extern "C"
 
-// mc_moe_forward with an optional residual added in its last kernel (resid may
-// alias y; the stack's h <- h + MoE(RMSNorm(h)) without a separate add).
-int mc::moe_forward_resid(const void *x, const void *gate_w, int T, const mc_shape *shape, const int8_t *bits_host,
-                          const void *packed_dev, float mu, const uint8_t *protect, void *y, const void *resid,
-                          void *workspace, size_t ws_bytes, int32_t *topk_idx_out, float *topk_w_out,
-                          uint8_t *pruned_out, void *stream)
+// mc_moe_forward with the stack's pre-norm and residual folded into its first
+// and last launches (LayerPrePost).
+int mc::moe_forward_ex(const void *x, const void *gate_w, int T, const mc_shape *shape, const int8_t *bits_host,
+                       const void *packed_dev, float mu, const uint8_t *protect, void *y, const LayerPrePost *lpp,
+                       void *workspace, size_t ws_bytes, int32_t *topk_idx_out, float *topk_w_out,
+                       uint8_t *pruned_out, void *stream)
 {
     clear_error();
     int rc = check_bits(shape, bits_host);
@@ -250,6 +250,13 @@ int mc::moe_forward_resid(const void *x, const void *gate_w, int T, const mc_sha
     rp.idx_out = topk_idx_out;
     rp.w_out = topk_w_out;
     rp.pruned_out = pruned_out;
+    if (lpp && lpp->norm_in) {
+        if (shape->H > 16384 || !aligned(lpp->norm_in, 16) || !aligned(lpp->gamma, 16))
+            return set_error(MC_ERR_INVALID_ARG, "pre-norm input and gamma need 16-byte alignment, H <= 16384");
+        rp.h_in = (const __nv_bfloat16 *)lpp->norm_in;
+        rp.gamma = (const __nv_bfloat16 *)lpp->gamma;
+        rp.eps = lpp->eps;
+    }
     PermuteParams pp{};
     memset(&pp, 0, sizeof pp);
     pp.idx = ws.idx;
@@ -310,7 +317,7 @@ int mc::moe_forward_resid(const void *x, const void *gate_w, int T, const mc_sha
     cp.KS = ep.KS;
     cp.Pmax = 2 * T;
     cp.y = (__nv_bfloat16 *)y;
-    cp.resid = (const __nv_bfloat16 *)resid;
+    cp.resid = lpp ? (const __nv_bfloat16 *)lpp->resid : nullptr;
     return launch_combine(cp, st);
 }
 
@@ -320,8 +327,8 @@ int mc_moe_forward(const void *x, const void *gate_w, int T, const mc_shape *sha
                    const void *packed_dev, float mu, const uint8_t *protect, void *y, void *workspace,
                    size_t ws_bytes, int32_t *topk_idx_out, float *topk_w_out, uint8_t *pruned_out, void *stream)
 {
-    return moe_forward_resid(x, gate_w, T, shape, bits_host, packed_dev, mu, protect, y, nullptr, workspace,
-                             ws_bytes, topk_idx_out, topk_w_out, pruned_out, stream);
+    return moe_forward_ex(x, gate_w, T, shape, bits_host, packed_dev, mu, protect, y, nullptr, workspace, ws_bytes,
+                          topk_idx_out, topk_w_out, pruned_out, stream);
 }
 
 int mc_check_status(void *workspace, void *stream)

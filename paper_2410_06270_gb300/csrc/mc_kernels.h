@@ -49,6 +49,11 @@ struct RouteParams {
     int32_t *idx_out;           // optional copies
     float *w_out;
     uint8_t *pruned_out;
+    // optional pre-norm (the stack): x = RMSNorm(h_in) with gamma and eps, computed
+    // here, written to x (which the expert kernels then read) and routed on
+    const __nv_bfloat16 *h_in;  // [T, H] or null
+    const __nv_bfloat16 *gamma; // [H]
+    float eps;
 };
 
 struct PermuteParams {
@@ -150,12 +155,21 @@ int32_t *route_done_word();  // mc_route's arrival word for the single-launch ro
 // best, among the divisors of F/128 that leave every item >= 8 column steps).
 int max_ks(const mc_shape *s, int T);
 int choose_ks(const mc_shape *s, int T, int nsm);
-// mc_moe_forward whose last kernel writes y = resid + the layer output (resid may
-// alias y; null: mc_moe_forward itself).  Used by mc_stack_forward.
-int moe_forward_resid(const void *x, const void *gate_w, int T, const mc_shape *shape, const int8_t *bits_host,
-                      const void *packed_dev, float mu, const uint8_t *protect, void *y, const void *resid,
-                      void *workspace, size_t ws_bytes, int32_t *topk_idx_out, float *topk_w_out,
-                      uint8_t *pruned_out, void *stream);
+// The pre-norm residual form of one layer, for mc_stack_forward: with norm_in,
+// the routing launch computes x = RMSNorm(norm_in) (gamma, eps; bit for bit
+// mc_rmsnorm) into the buffer x and routes on it; with resid, the last kernel
+// writes y = resid + the layer output (resid may alias y).  Both null:
+// mc_moe_forward itself.
+struct LayerPrePost {
+    const void *norm_in;  // bf16 [T, H] or null (16-byte aligned)
+    const void *gamma;    // bf16 [H] (16-byte aligned)
+    float eps;
+    const void *resid;    // bf16 [T, H] or null
+};
+int moe_forward_ex(const void *x, const void *gate_w, int T, const mc_shape *shape, const int8_t *bits_host,
+                   const void *packed_dev, float mu, const uint8_t *protect, void *y, const LayerPrePost *pp,
+                   void *workspace, size_t ws_bytes, int32_t *topk_idx_out, float *topk_w_out, uint8_t *pruned_out,
+                   void *stream);
 // The test hooks of mc_set_debug: its flags and the bound on device waits.
 int debug_flags();
 uint64_t wait_bound_ns();

@@ -20,14 +20,56 @@ namespace mc {
 
 constexpr int kRouteThreads = 512;
 
+// The pre-norm of token t's row (the stack): h_in[t] staged in shared memory and
+// its sum of squares accumulated in the order of rmsnorm_vec_kernel (256
+// threads, thread i over the 16-byte chunks i + 256 j, j < 8; warp xor
+// reductions; the 8 warp partials added in order), so that inv and every
+// normalised element f * inv * g are bit for bit those of mc_rmsnorm.
+__device__ __forceinline__ float route_row_inv(const RouteParams &p, int t, uint4 *row_s, float *red)
+{
+    const int tid = threadIdx.x, n8 = p.H >> 3;
+    const uint4 *hr = reinterpret_cast<const uint4 *>(p.h_in + (size_t)t * p.H);
+    for (int c = tid; c < n8; c += kRouteThreads) row_s[c] = hr[c];
+    __syncthreads();
+    if (tid < 256) {
+        float ss = 0.f;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const int c = tid + 256 * i;
+            if (c >= n8) continue;
+            const uint4 v = row_s[c];
+            const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&v);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float2 f = __bfloat1622float2(b2[k]);
+                ss = fmaf(f.x, f.x, ss);
+                ss = fmaf(f.y, f.y, ss);
+            }
+        }
+        for (int m = 16; m >= 1; m >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, m);
+        if ((tid & 31) == 0) red[tid >> 5] = ss;
+    }
+    __syncthreads();
+    float tot = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) tot += red[w];
+    return rsqrtf(tot / p.H + p.eps);
+}
+
 // The logits of token t by the whole CTA; thread 0 takes the decision and writes
 // the outputs.
+template <bool NORM>
 __device__ __forceinline__ void route_token(const RouteParams &p, int t)
 {
     __shared__ float part[kRouteThreads / 32][kMaxE];
+    __shared__ float red[8];
+    // the pre-norm row: dynamic shared memory, H * 2 bytes, given only with h_in
+    extern __shared__ uint4 row_s[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int H = p.H, E = p.E;
     const __nv_bfloat16 *xr = p.x + (size_t)t * H;
+    float inv = 0.f;
+    if constexpr (NORM) inv = route_row_inv(p, t, row_s, red);
     // the mask byte is needed only by thread 0's decision; load it now
     // (0: prunable, 2: dropped, anything else: protected)
     const int mask = threadIdx.x == 0 && p.protect != nullptr ? p.protect[t] : 0;
@@ -35,7 +77,23 @@ __device__ __forceinline__ void route_token(const RouteParams &p, int t)
 #pragma unroll
     for (int e = 0; e < kMaxE; ++e) acc[e] = 0.f;
     for (int c0 = 8 * threadIdx.x; c0 < H; c0 += 8 * kRouteThreads) {
-        const uint4 raw = *reinterpret_cast<const uint4 *>(xr + c0);
+        uint4 raw;
+        if constexpr (NORM) {
+            // x = h * inv * gamma rounded to bf16 (mc_rmsnorm's expression), written
+            // for the expert kernels and routed on as written
+            const uint4 hv = row_s[c0 >> 3], gv = *reinterpret_cast<const uint4 *>(p.gamma + c0);
+            const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&hv);
+            const __nv_bfloat162 *g2 = reinterpret_cast<const __nv_bfloat162 *>(&gv);
+            __nv_bfloat162 *o2 = reinterpret_cast<__nv_bfloat162 *>(&raw);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float2 f = __bfloat1622float2(h2[k]), g = __bfloat1622float2(g2[k]);
+                o2[k] = __floats2bfloat162_rn(f.x * inv * g.x, f.y * inv * g.y);
+            }
+            *reinterpret_cast<uint4 *>(const_cast<__nv_bfloat16 *>(xr) + c0) = raw;
+        } else {
+            raw = *reinterpret_cast<const uint4 *>(xr + c0);
+        }
         uint4 gr[kMaxE];
 #pragma unroll
         for (int e = 0; e < kMaxE; ++e)
@@ -124,11 +182,12 @@ __device__ __forceinline__ void route_token(const RouteParams &p, int t)
     if (p.pruned_out) p.pruned_out[t] = (uint8_t)prune;
 }
 
+template <bool NORM>
 __global__ void __launch_bounds__(kRouteThreads) route_kernel(RouteParams p)
 {
     pdl_trigger();
     pdl_wait();
-    route_token(p, blockIdx.x);
+    route_token<NORM>(p, blockIdx.x);
 }
 
 // Histogram, scan, stable placement and work-chunk list by one CTA of any size
@@ -314,12 +373,13 @@ __device__ __forceinline__ void permute_warp(const PermuteParams &p)
 
 // Routing of token blockIdx.x, then the last CTA to finish (counted on *done,
 // which it resets) places the pairs: one launch instead of two for small T.
+template <bool NORM>
 __global__ void __launch_bounds__(kRouteThreads) route_permute_kernel(RouteParams rp, PermuteParams pp, int32_t *done)
 {
     __shared__ int last;
     pdl_trigger();
     pdl_wait();
-    route_token(rp, blockIdx.x);
+    route_token<NORM>(rp, blockIdx.x);
     __syncthreads();
     if (threadIdx.x == 0) {
         // thread 0 wrote this CTA's routing outputs: the release orders them before
@@ -349,16 +409,20 @@ int max_chunks_for(int T, int E) { return (2 * T + kChunk - 1) / kChunk + E; }
 
 int launch_route(const RouteParams &rp, const PermuteParams &pp, cudaStream_t st, int32_t *done)
 {
+    // the pre-norm row (mc_stack_forward's layers) in dynamic shared memory
+    const size_t norm_smem = rp.h_in ? (size_t)rp.H * 2 : 0;
     cudaError_t err;
     if (done && rp.T <= 64) {
         profile_begin(kKRoute, st);
-        err = launch_k(route_permute_kernel, dim3(rp.T), dim3(kRouteThreads), 0, st, rp, pp, done);
+        err = rp.h_in ? launch_k(route_permute_kernel<true>, dim3(rp.T), dim3(kRouteThreads), norm_smem, st, rp, pp, done)
+                      : launch_k(route_permute_kernel<false>, dim3(rp.T), dim3(kRouteThreads), 0, st, rp, pp, done);
         profile_end(kKRoute, st);
         if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "route launch: %s", cudaGetErrorString(err));
         return MC_OK;
     }
     profile_begin(kKRoute, st);
-    err = launch_k(route_kernel, dim3(rp.T), dim3(kRouteThreads), 0, st, rp);
+    err = rp.h_in ? launch_k(route_kernel<true>, dim3(rp.T), dim3(kRouteThreads), norm_smem, st, rp)
+                  : launch_k(route_kernel<false>, dim3(rp.T), dim3(kRouteThreads), 0, st, rp);
     profile_end(kKRoute, st);
     if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "route launch: %s", cudaGetErrorString(err));
     profile_begin(kKPermute, st);

@@ -35,13 +35,17 @@ extern "C" int mc_stack_forward(void *h, int T, const mc_shape *shape, int layer
     if (ws_bytes < need) return set_error(MC_ERR_INVALID_ARG, "workspace has %zu bytes, needs %zu", ws_bytes, need);
     const size_t fw = align256(mc_moe_workspace_size(shape, T));
     void *xn = (uint8_t *)workspace + fw;
+    // With 16-byte aligned rows the layer's routing launch computes its RMSNorm (bit
+    // for bit mc_rmsnorm) into xn and routes on it; otherwise mc_rmsnorm runs first.
+    const bool fused_norm = ((uintptr_t)h % 16 == 0) && ((uintptr_t)gamma % 16 == 0) && shape->H % 8 == 0;
     for (int l = 0; l < layers; ++l) {
         const void *g = (const uint8_t *)gamma + (size_t)l * shape->H * 2;
-        if ((rc = mc_rmsnorm(h, g, T, shape->H, eps, xn, stream))) return rc;
+        if (!fused_norm && (rc = mc_rmsnorm(h, g, T, shape->H, eps, xn, stream))) return rc;
         // the layer's combine adds its output to h in place (h + MoE(xn), rounded
         // like mc_add of the layer's bf16 output)
-        if ((rc = moe_forward_resid(xn, gate_w[l], T, shape, bits_host + (size_t)l * shape->E, packed_dev[l],
-                                    mu_host[l], protect, h, h, workspace, fw, nullptr, nullptr, nullptr, stream)))
+        LayerPrePost lpp{fused_norm ? h : nullptr, g, eps, h};
+        if ((rc = moe_forward_ex(xn, gate_w[l], T, shape, bits_host + (size_t)l * shape->E, packed_dev[l], mu_host[l],
+                                 protect, h, &lpp, workspace, fw, nullptr, nullptr, nullptr, stream)))
             return rc;
     }
     return MC_OK;
