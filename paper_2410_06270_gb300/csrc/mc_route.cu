@@ -68,6 +68,14 @@ __device__ __forceinline__ void route_token(const RouteParams &p, int t)
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int H = p.H, E = p.E;
     const __nv_bfloat16 *xr = p.x + (size_t)t * H;
+    // the gate's first column round goes out before the pre-norm's reduction
+    uint4 gr[kMaxE];
+    if constexpr (NORM) {
+        const int c0 = 8 * threadIdx.x;
+#pragma unroll
+        for (int e = 0; e < kMaxE; ++e)
+            if (e < E && c0 < H) gr[e] = *reinterpret_cast<const uint4 *>(p.gate + (size_t)e * H + c0);
+    }
     float inv = 0.f;
     if constexpr (NORM) inv = route_row_inv(p, t, row_s, red);
     // the mask byte is needed only by thread 0's decision; load it now
@@ -94,10 +102,11 @@ __device__ __forceinline__ void route_token(const RouteParams &p, int t)
         } else {
             raw = *reinterpret_cast<const uint4 *>(xr + c0);
         }
-        uint4 gr[kMaxE];
+        if (!NORM || c0 != 8 * (int)threadIdx.x) {
 #pragma unroll
-        for (int e = 0; e < kMaxE; ++e)
-            if (e < E) gr[e] = *reinterpret_cast<const uint4 *>(p.gate + (size_t)e * H + c0);
+            for (int e = 0; e < kMaxE; ++e)
+                if (e < E) gr[e] = *reinterpret_cast<const uint4 *>(p.gate + (size_t)e * H + c0);
+        }
         const __nv_bfloat162 *x2 = reinterpret_cast<const __nv_bfloat162 *>(&raw);
         float xf[8];
 #pragma unroll
