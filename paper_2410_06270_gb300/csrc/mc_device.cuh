@@ -127,13 +127,6 @@ __device__ __forceinline__ void bulk_g2s_stream(void *dst_smem, const void *src_
         : "memory");
 }
 
-// Bring [src, src + bytes) into L2 (16-byte aligned, bytes a multiple of 16); no
-// destination, nothing to wait for.
-__device__ __forceinline__ void bulk_prefetch_l2(const void *src, uint32_t bytes)
-{
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
-}
-
 __device__ __forceinline__ uint64_t policy_evict_first()
 {
     uint64_t p;

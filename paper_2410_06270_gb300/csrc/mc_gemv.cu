@@ -92,11 +92,11 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity, co
 }
 
 // The packed buffer must carry the header written for this shape and bit table:
-// the expert's bit width and the byte offsets of its matrices (which depend on
-// every earlier expert's width) must match what the host computed, so no copy
-// ever reads outside the region the buffer was packed with.
-// The packed buffer's header matches the shape, bit table and matrix offsets the
-// kernel was launched with, for every expert (its loads are all in flight together).
+// every expert's bit width and the byte offsets of its matrices (which depend on
+// every earlier expert's width) must match what the host computed, so that no
+// copy ever reads outside the region the buffer was packed with.  Checked once per
+// call by frag_x_kernel (all loads in flight together); the expert kernels read
+// its verdict.
 __device__ __forceinline__ bool header_ok(const ExpertParams &p)
 {
     const PackHeader *hd = reinterpret_cast<const PackHeader *>(p.packed);
@@ -586,11 +586,10 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(ExpertParams p)
     if (W13) build_tab_afrag(afr, threadIdx.x, kGemvThreads);
     __syncthreads();
 
-    // The producer's first claim, the header check and an L2 prefetch of its first
-    // item's weights read only the routing outputs and the packed weights: the
-    // routing launch completed before the launch before this one triggered this
-    // kernel, so this overlaps that launch's end.  Everything after the wait may
-    // read what that launch wrote.
+    // The producer's first claim reads only the routing outputs: the routing launch
+    // completed before the launch before this one triggered this kernel, so it
+    // overlaps that launch's end.  Everything after the wait may read what that
+    // launch wrote (the packed header's verdict among it).
     const bool producer = warp == kCW && lane == 0 && !(p.debug & kDebugNoProducer);
     int *counter = &p.counters[W13 ? 0 : 1];
     int item = 0, total = 0;
