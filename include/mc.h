@@ -208,8 +208,8 @@ int mc_moe_forward_static(const void *x, const void *gate_w, int T, const mc_sha
                           const uint8_t *protect, void *y, int32_t *status_dev, void *stream);
 
 /* Workspace bytes of mc_stack_forward for up to T_max tokens: the layer
- * workspace (status word first) followed by one [T_max, H] bf16 activation (the
- * normalised layer input). */
+ * workspace (status word first) followed by two [T_max, H] bf16 activations (the
+ * normalised layer input; the layer output when h is not 16-byte aligned). */
 size_t mc_stack_workspace_size(const mc_shape *shape, int T_max);
 
 /* A stack of `layers` pre-norm residual MoE blocks, the structure of the
@@ -222,7 +222,8 @@ size_t mc_stack_workspace_size(const mc_shape *shape, int T_max);
  * gamma each layer's RMSNorm runs inside its routing launch and its residual add
  * inside its combine, with the arithmetic and rounding of mc_rmsnorm and mc_add
  * (the result is bit for bit that of mc_rmsnorm, mc_moe_forward and mc_add in
- * turn).  protect (device [T] or NULL)
+ * turn, which is what runs for an h of any other alignment).  protect (device
+ * [T] or NULL)
  * applies to every layer.  Device-detected faults of any layer go to the status
  * word at the start of `workspace` (mc_check_status).  All launches go to
  * `stream` and none synchronises, so a caller may capture one call into a CUDA

@@ -51,7 +51,10 @@ __global__ void unpack_kernel(const uint8_t *packed, uint64_t mat_off, int mat, 
     }
 }
 
-// One CTA of 256 threads per row; fp32 statistics.
+// One CTA of 256 threads per row; fp32 statistics.  For H % 8 == 0 the sum of
+// squares takes the order of rmsnorm_vec_kernel (thread i over the 8-element
+// chunks i, i + 256, ..., each chunk's elements in turn), so that the result does
+// not depend on which of the two kernels the alignment of the arguments picks.
 __global__ void __launch_bounds__(256) rmsnorm_kernel(const __nv_bfloat16 *x, const __nv_bfloat16 *gamma, int H,
                                                       float eps, __nv_bfloat16 *out)
 {
@@ -60,9 +63,18 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const __nv_bfloat16 *x, co
     const __nv_bfloat16 *xr = x + (size_t)blockIdx.x * H;
     __shared__ float red[8];
     float ss = 0.f;
-    for (int c = threadIdx.x; c < H; c += blockDim.x) {
-        float v = __bfloat162float(xr[c]);
-        ss = fmaf(v, v, ss);
+    if (H % 8 == 0) {
+        for (int c = threadIdx.x; c < H / 8; c += blockDim.x)
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const float v = __bfloat162float(xr[8 * c + e]);
+                ss = fmaf(v, v, ss);
+            }
+    } else {
+        for (int c = threadIdx.x; c < H; c += blockDim.x) {
+            const float v = __bfloat162float(xr[c]);
+            ss = fmaf(v, v, ss);
+        }
     }
     for (int m = 16; m >= 1; m >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, m);
     if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;

@@ -16,7 +16,7 @@ extern "C" size_t mc_stack_workspace_size(const mc_shape *shape, int T_max)
 {
     const size_t ws = mc_moe_workspace_size(shape, T_max);
     if (!ws) return 0;
-    return align256(ws) + align256((size_t)T_max * shape->H * 2);
+    return align256(ws) + 2 * align256((size_t)T_max * shape->H * 2);
 }
 
 extern "C" int mc_stack_forward(void *h, int T, const mc_shape *shape, int layers, const void *const *gate_w,
@@ -34,19 +34,28 @@ extern "C" int mc_stack_forward(void *h, int T, const mc_shape *shape, int layer
     const size_t need = mc_stack_workspace_size(shape, T);
     if (ws_bytes < need) return set_error(MC_ERR_INVALID_ARG, "workspace has %zu bytes, needs %zu", ws_bytes, need);
     const size_t fw = align256(mc_moe_workspace_size(shape, T));
-    void *xn = (uint8_t *)workspace + fw;
+    const size_t act = align256((size_t)T * shape->H * 2);
+    void *xn = (uint8_t *)workspace + fw, *y = (uint8_t *)workspace + fw + act;
     // With 16-byte aligned rows the layer's routing launch computes its RMSNorm (bit
-    // for bit mc_rmsnorm) into xn and routes on it; otherwise mc_rmsnorm runs first.
-    const bool fused_norm = ((uintptr_t)h % 16 == 0) && ((uintptr_t)gamma % 16 == 0) && shape->H % 8 == 0;
+    // for bit mc_rmsnorm) into xn and routes on it, and its combine adds the layer
+    // output to h in place (rounded like mc_add of the layer's bf16 output).  An
+    // unaligned h takes mc_rmsnorm, the layer into y and mc_add: the same result.
+    const bool h_aligned = (uintptr_t)h % 16 == 0;
+    const bool fused_norm = h_aligned && ((uintptr_t)gamma % 16 == 0) && shape->H % 8 == 0;
     for (int l = 0; l < layers; ++l) {
         const void *g = (const uint8_t *)gamma + (size_t)l * shape->H * 2;
+        const int8_t *bl = bits_host + (size_t)l * shape->E;
         if (!fused_norm && (rc = mc_rmsnorm(h, g, T, shape->H, eps, xn, stream))) return rc;
-        // the layer's combine adds its output to h in place (h + MoE(xn), rounded
-        // like mc_add of the layer's bf16 output)
-        LayerPrePost lpp{fused_norm ? h : nullptr, g, eps, h};
-        if ((rc = moe_forward_ex(xn, gate_w[l], T, shape, bits_host + (size_t)l * shape->E, packed_dev[l], mu_host[l],
-                                 protect, h, &lpp, workspace, fw, nullptr, nullptr, nullptr, stream)))
-            return rc;
+        if (h_aligned) {
+            LayerPrePost lpp{fused_norm ? h : nullptr, g, eps, h};
+            rc = moe_forward_ex(xn, gate_w[l], T, shape, bl, packed_dev[l], mu_host[l], protect, h, &lpp, workspace,
+                                fw, nullptr, nullptr, nullptr, stream);
+        } else {
+            rc = mc_moe_forward(xn, gate_w[l], T, shape, bl, packed_dev[l], mu_host[l], protect, y, workspace, fw,
+                                nullptr, nullptr, nullptr, stream);
+            if (!rc) rc = mc_add(h, y, (size_t)T * shape->H, h, stream);
+        }
+        if (rc) return rc;
     }
     return MC_OK;
 }

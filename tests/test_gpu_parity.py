@@ -461,6 +461,14 @@ def test_rmsnorm_and_add(mc, H):
     np.testing.assert_array_equal(s, 2 * synth.bf16_bits_to_f32(xs))
     s1 = mc.add(x.view(-1)[1:], x.view(-1)[1:]).float().cpu().numpy()  # odd length, unaligned: scalar kernel
     np.testing.assert_array_equal(s1, 2 * synth.bf16_bits_to_f32(xs).reshape(-1)[1:])
+    if H % 8 == 0:
+        # an unaligned row takes the scalar kernel, which sums in the vector
+        # kernel's order for H % 8 == 0: the same bits
+        buf = torch.empty(6 * H + 8, dtype=torch.bfloat16, device="cuda")
+        xu = buf[1:1 + 6 * H].view(6, H)
+        xu.copy_(x)
+        yu = mc.rmsnorm(xu, g, 1e-5).float().cpu().numpy()
+        np.testing.assert_array_equal(yu, y)
 
 
 @pytest.mark.parametrize("path", [1, 2])

@@ -112,6 +112,38 @@ def test_stack_graph_replay_equals_eager(mc, shape_name):
     assert torch.equal(h_eager.view(torch.int16), h_graph.view(torch.int16))
 
 
+def test_stack_fused_pre_norm_equals_separate_launches(mc):
+    """With 16-byte aligned h and gamma each layer's RMSNorm runs in its routing
+    launch and its residual add in its combine; an unaligned h (or gamma) takes
+    mc_rmsnorm, the layer and mc_add as separate launches.  The results are bit
+    for bit the same, with random (non-unit) gamma."""
+    L, gates = synth.config_stack(T=24, layers=5, seed=405, H=256, F=512, E=8, group=64, gate_std=0.1)
+    mus = [0.2] * len(gates)
+    shape, args, gamma, ws, prot = _setup(mc, L, gates, mus, copies=True)
+    rng = np.random.default_rng(405)
+    gvals = torch.from_numpy((1.0 + 0.25 * rng.standard_normal(gamma.shape)).astype(np.float32)).to(torch.bfloat16)
+    gamma.copy_(gvals.cuda())
+    n = L.T * L.H
+    h_fused = _dev_bf16(L.x)
+    mc.stack_forward(h_fused, shape, args, gamma, ws, prot)
+    # h two bytes past an aligned address: the separate-launch path
+    buf = torch.empty(n + 8, dtype=torch.bfloat16, device="cuda")
+    h_sep = buf[1:1 + n].view(L.T, L.H)
+    h_sep.copy_(_dev_bf16(L.x))
+    assert h_sep.data_ptr() % 16 != 0
+    mc.stack_forward(h_sep, shape, args, gamma, ws, prot)
+    # aligned h, unaligned gamma: separate RMSNorm, residual add in the combine
+    gbuf = torch.empty(gamma.numel() + 8, dtype=torch.bfloat16, device="cuda")
+    g_un = gbuf[1:1 + gamma.numel()].view(gamma.shape)
+    g_un.copy_(gamma)
+    h_gun = _dev_bf16(L.x)
+    mc.stack_forward(h_gun, shape, args, g_un, ws, prot)
+    torch.cuda.synchronize()
+    mc.check_status(ws)
+    assert torch.equal(h_fused.view(torch.int16), h_sep.view(torch.int16))
+    assert torch.equal(h_fused.view(torch.int16), h_gun.view(torch.int16))
+
+
 def test_stack_same_without_programmatic_launch(mc):
     """The stack with every kernel launched without programmatic dependent
     launch is bit-identical to the default (overlapped launches)."""
