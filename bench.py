@@ -219,14 +219,17 @@ def _timed_rounds(torch, replay, steps, stream, world, min_s=MIN_TIMED_S, max_ro
 
 
 def _e2e_pipelined(torch, step, nsets, x, y, steps, stream, min_s=MIN_TIMED_S / 2, max_rounds=2000):
-    """End to end: every step copies its input from pinned host memory to the
-    device and its output back, over two device buffer pairs, so that step i+1's
-    input copy and step i's output copy (copy stream) overlap step i's layer
-    (launching stream).  A round is `steps` such steps, timed from before the
-    first input copy to after the last output copy; each graph is replayed once
-    before the first round (its first launch uploads it), and rounds repeat (at
-    least 3) until `min_s` seconds have passed.  Returns the median round's
-    milliseconds."""
+    """End to end: every step copies an input from pinned host memory to the
+    device and an output back, over two device buffer pairs.  A step is one graph
+    replay with three branches: the layer on pair b, the host->device copy of the
+    next step's input into pair 1-b and the device->host copy of the previous
+    step's output out of pair 1-b, so the copies overlap the layer with no
+    cross-stream synchronisation between steps.  A round is `steps` such steps
+    plus the first input's copy before them and the last output's copy after
+    them, timed from before the first copy to after the last; each graph is
+    replayed once before the first round (its first launch uploads it), and
+    rounds repeat (at least 3) until `min_s` seconds have passed.  Returns the
+    median round's milliseconds."""
     xh = [torch.empty(x.shape, dtype=x.dtype, pin_memory=True) for _ in range(2)]
     yh = [torch.empty(y.shape, dtype=y.dtype, pin_memory=True) for _ in range(2)]
     for b in range(2):
@@ -237,46 +240,33 @@ def _e2e_pipelined(torch, step, nsets, x, y, steps, stream, min_s=MIN_TIMED_S / 
     for k in range(nsets):
         for b in range(2):
             gr = torch.cuda.CUDAGraph()
-            cs = torch.cuda.Stream()
+            cs, side = torch.cuda.Stream(), torch.cuda.Stream()
             cs.wait_stream(torch.cuda.current_stream())
             with torch.cuda.stream(cs):
                 with torch.cuda.graph(gr, stream=cs):
+                    fork, join = torch.cuda.Event(), torch.cuda.Event()
+                    fork.record(cs)
+                    side.wait_event(fork)
+                    with torch.cuda.stream(side):
+                        xd[1 - b].copy_(xh[1 - b], non_blocking=True)  # the next step's input
+                        yh[1 - b].copy_(yd[1 - b], non_blocking=True)  # the previous step's output
+                        join.record(side)
                     step(k, xd[b], yd[b])
+                    cs.wait_event(join)
             torch.cuda.current_stream().wait_stream(cs)
             graphs[k, b] = gr
     for gr in graphs.values():
         gr.replay()
     torch.cuda.synchronize()
-    copy = torch.cuda.Stream()
-    ev_in = [torch.cuda.Event() for _ in range(2)]
-    ev_done = [torch.cuda.Event() for _ in range(2)]
-    ev_out = [torch.cuda.Event() for _ in range(2)]
     e2, e3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    last = (steps - 1) % 2
 
     def one_round():
         e2.record(stream)
-        copy.wait_event(e2)
-        with torch.cuda.stream(copy):
-            xd[0].copy_(xh[0], non_blocking=True)
-            ev_in[0].record(copy)
+        xd[0].copy_(xh[0], non_blocking=True)
         for i in range(steps):
-            b = i % 2
-            if i + 1 < steps:
-                # buffer 1-b was last read by step i-1, whose output copy the copy
-                # stream already waited for
-                with torch.cuda.stream(copy):
-                    xd[1 - b].copy_(xh[1 - b], non_blocking=True)
-                    ev_in[1 - b].record(copy)
-            stream.wait_event(ev_in[b])
-            if i >= 2:
-                stream.wait_event(ev_out[b])  # step i-2's output has left yd[b]
-            graphs[i % nsets, b].replay()
-            ev_done[b].record(stream)
-            copy.wait_event(ev_done[b])
-            with torch.cuda.stream(copy):
-                yh[b].copy_(yd[b], non_blocking=True)
-                ev_out[b].record(copy)
-        stream.wait_stream(copy)
+            graphs[i % nsets, i % 2].replay()
+        yh[last].copy_(yd[last], non_blocking=True)
         e3.record(stream)
         torch.cuda.synchronize()
         return e2.elapsed_time(e3)
@@ -687,8 +677,9 @@ def measure_layer(name, args, torch, mc, dev, local, world, cpu=True):
                   "overlap, so the sum exceeds ms_per_step)" % (nsets * max(3, min(steps, 200))),
         "e2e": {"value": e2e, "unit": "tokens/s", "h2d_bytes_per_step": int(x.numel() * 2),
                 "d2h_bytes_per_step": int(y.numel() * 2),
-                "copies": "cudaMemcpyAsync from / to pinned host buffers every step, on a copy stream, two "
-                          "device buffer pairs: step i+1's input and step i's output move while step i runs"},
+                "copies": "pinned host buffers, two device buffer pairs; every step is one graph replay "
+                          "whose branches copy step i+1's input in and step i-1's output out while step i's "
+                          "layer runs (plus the first input before and the last output after the steps)"},
         "gpu_launches": int(round(sum(n for _, n in breakdown.values()))) * steps,
         "clocks": _clock_note(cl),
     }
