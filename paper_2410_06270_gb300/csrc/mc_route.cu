@@ -8,10 +8,14 @@
 //   rows, 16 bytes each) before it uses any, so a round costs one memory round
 //   trip; the partial logits meet in shared memory, warp 0 adds them up and
 //   thread 0 takes the decision in fp32.
+// route_cluster_kernel (T <= 16): the same as one thread-block cluster, the
+//   decisions gathered in CTA 0's shared memory and placed by its first warp.
 // permute_kernel: one CTA; histogram, exclusive scan and a stable placement with
 //   __match_any_sync ranks, so the permutation is unique (ascending token within
 //   an expert) and identical run to run.  It also lists the work chunks of the
 //   expert kernels (one thread per expert) and resets their work counters.
+#include <cooperative_groups.h>
+
 #include "mc_host.h"
 #include "mc_kernels.h"
 #include "mc_profile.h"
@@ -59,7 +63,9 @@ __device__ __forceinline__ float route_row_inv(const RouteParams &p, int t, uint
 // The logits of token t by the whole CTA; thread 0 takes the decision and writes
 // the outputs.
 template <bool NORM>
-__device__ __forceinline__ void route_token(const RouteParams &p, int t)
+//   sink (optional): where thread 0 also leaves the decision (e0, e1, pruned) of
+//   token t, three ints at 3 t (the cluster routing: CTA 0's shared memory).
+__device__ __forceinline__ void route_token(const RouteParams &p, int t, int *sink = nullptr)
 {
     __shared__ float part[kRouteThreads / 32][kMaxE];
     __shared__ float red[8];
@@ -174,6 +180,11 @@ __device__ __forceinline__ void route_token(const RouteParams &p, int t)
     if (drop) {  // no expert: weights (0, 0), pruned = 2
         w0 = w1 = 0.f;
         prune = 2;
+    }
+    if (sink) {
+        sink[3 * t] = e0;
+        sink[3 * t + 1] = e1;
+        sink[3 * t + 2] = prune;
     }
     p.idx[2 * t] = e0;
     p.idx[2 * t + 1] = e1;
@@ -304,7 +315,9 @@ __global__ void __launch_bounds__(1024) permute_kernel(PermuteParams p)
 // expert's count, a warp scan over the lanes gives the offsets, and a pair's
 // place is its expert's start of the slice plus the lanes of that expert below
 // it in the slice.  Same result as permute_block.
-__device__ __forceinline__ void permute_warp(const PermuteParams &p)
+//   dec (optional): the tokens' decisions in shared memory (e0, e1, pruned at 3 t)
+//   instead of the routing outputs in global memory.
+__device__ __forceinline__ void permute_warp(const PermuteParams &p, const int *dec = nullptr)
 {
     const unsigned full = 0xffffffffu, lt = (1u << (threadIdx.x & 31)) - 1;
     const int lane = threadIdx.x & 31, NP = 2 * p.T, nk = (NP + 31) / 32, E = p.E;
@@ -314,8 +327,8 @@ __device__ __forceinline__ void permute_warp(const PermuteParams &p)
         const int i = 32 * k + lane;
         key[k] = -1;
         if (i < NP) {
-            const uint8_t pr = __ldcg(p.pruned + (i >> 1));
-            const int e = __ldcg(p.idx + i);
+            const int pr = dec ? dec[3 * (i >> 1) + 2] : (int)__ldcg(p.pruned + (i >> 1));
+            const int e = dec ? dec[3 * (i >> 1) + (i & 1)] : __ldcg(p.idx + i);
             key[k] = ((i & 1) && pr) || pr == 2 ? -1 : e;
         }
     }
@@ -403,6 +416,27 @@ __global__ void __launch_bounds__(kRouteThreads) route_permute_kernel(RouteParam
     if (threadIdx.x == 0) *done = 0;
 }
 
+// Routing and placement of up to kClusterMaxT tokens as one thread-block cluster
+// (one CTA per token): each CTA's decision also goes into CTA 0's shared memory,
+// a cluster barrier (release / acquire) replaces the global arrival count, and
+// CTA 0 places the pairs from its shared memory.
+constexpr int kClusterMaxT = 16;
+
+template <bool NORM>
+__global__ void __launch_bounds__(kRouteThreads) route_cluster_kernel(RouteParams rp, PermuteParams pp)
+{
+    __shared__ int dec_s[3 * kClusterMaxT];
+    namespace cg = cooperative_groups;
+    cg::cluster_group cl = cg::this_cluster();
+    int *sink = cl.map_shared_rank(dec_s, 0);
+    pdl_trigger();
+    pdl_wait();
+    route_token<NORM>(rp, blockIdx.x, sink);
+    cl.sync();
+    if (cl.block_rank() != 0 || threadIdx.x >= 32) return;
+    permute_warp(pp, dec_s);
+}
+
 // The arrival count of mc_route's single-launch routing (kDebugRouteFused): one
 // word owned by the library, zero between launches (the last CTA resets it), so
 // such calls must not overlap in time on one device.
@@ -416,11 +450,41 @@ int32_t *route_done_word()
 
 int max_chunks_for(int T, int E) { return (2 * T + kChunk - 1) / kChunk + E; }
 
+// One cluster of T CTAs (T <= kClusterMaxT; above 8 a non-portable cluster size).
+template <bool NORM>
+static cudaError_t launch_route_cluster(const RouteParams &rp, const PermuteParams &pp, size_t smem, cudaStream_t st)
+{
+    cudaError_t err = cudaFuncSetAttribute(route_cluster_kernel<NORM>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (err != cudaSuccess) return err;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(rp.T);
+    cfg.blockDim = dim3(kRouteThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)rp.T;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl_enabled() ? 2 : 1;
+    return cudaLaunchKernelEx(&cfg, route_cluster_kernel<NORM>, rp, pp);
+}
+
 int launch_route(const RouteParams &rp, const PermuteParams &pp, cudaStream_t st, int32_t *done)
 {
     // the pre-norm row (mc_stack_forward's layers) in dynamic shared memory
     const size_t norm_smem = rp.h_in ? (size_t)rp.H * 2 : 0;
     cudaError_t err;
+    if (done && rp.T <= kClusterMaxT) {
+        profile_begin(kKRoute, st);
+        err = rp.h_in ? launch_route_cluster<true>(rp, pp, norm_smem, st) : launch_route_cluster<false>(rp, pp, 0, st);
+        profile_end(kKRoute, st);
+        if (err != cudaSuccess) return set_error(MC_ERR_CUDA, "route launch: %s", cudaGetErrorString(err));
+        return MC_OK;
+    }
     if (done && rp.T <= 64) {
         profile_begin(kKRoute, st);
         err = rp.h_in ? launch_k(route_permute_kernel<true>, dim3(rp.T), dim3(kRouteThreads), norm_smem, st, rp, pp, done)
